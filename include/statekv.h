@@ -1,0 +1,167 @@
+/*
+ * statekv.h -- C ABI of the GB300 (sm_103a) StateKV per-frame cache-builder step.
+ *
+ * StateKV (Eyzaguirre, Wu, Niebles, "Linear Scaling Video VLMs for Long Video
+ * Understanding") builds a video VLM's KV cache one frame at a time.  Per layer
+ * it keeps two states (Sec. 3.2, Eq. 4):
+ *   - the compressed state C (capacity B tokens), the only cross-frame context
+ *     a new frame can attend to while the cache is built;
+ *   - the detailed state D (every frame's K and V), used only for decoding.
+ * For each new frame n and each layer (Sec. 3.3):
+ *   (a1) the frame's T queries attend, GQA-style, to [C ; frame] (Eq. 5) with
+ *        every state token visible and causal order inside the frame;
+ *   (a2) fused with it, each pool token's importance -- the attention it
+ *        receives, summed over the frame's queries (Eq. 1) and over the query
+ *        heads of its KV head (App. A: sinks are kept per layer and KV head) --
+ *        is recovered from the saved log-sum-exp (App. B.1);
+ *   (a3) the B best-scoring tokens of the pool C + frame become the new C
+ *        (Eq. 6); ties keep the older token;
+ *   (a4) evicted state slots receive the admitted frame rows (bit copies);
+ *   (a5) the frame's K and V are appended to D, and the virtual length
+ *        L_n = n * T advances (Sec. 3.3, "virtual sequence length").
+ *
+ * Memory: the caller allocates one device arena (statekv_arena_bytes) and the
+ * per-call input/output buffers.  The library never allocates device memory
+ * and never frees caller memory.  Every call is asynchronous on the given
+ * CUDA stream; argument errors are reported synchronously and enqueue nothing.
+ *
+ * Layouts (all row-major, bf16 = IEEE bfloat16, 16-byte aligned pointers):
+ *   per-call Q      [stream_count][layer_count][T][Hq][d]
+ *   per-call K, V   [stream_count][layer_count][T][Hkv][d]   (token-major)
+ *   per-call out    [stream_count][layer_count][T][Hq][d]
+ *   importance      fp32 [stream_count][layer_count][Hkv][B + T]
+ * Query head h belongs to KV head h / (Hq / Hkv).  Token t of frame n (1-based)
+ * sits at virtual position (n - 1) * T + t; rotary embeddings are expected to
+ * be applied by the caller at those positions (Sec. 3.3).
+ *
+ * Threading: one host thread per handle.  Calls on one stream run in order.
+ */
+#ifndef STATEKV_H
+#define STATEKV_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* A cudaStream_t (struct CUstream_st*), declared here without CUDA headers.
+ * NULL means the legacy default stream. */
+typedef struct CUstream_st* statekv_stream;
+
+typedef enum {
+    STATEKV_OK = 0,
+    STATEKV_ERR_INVALID_ARG = 1,     /* null/misaligned pointer, bad range or shape */
+    STATEKV_ERR_UNSUPPORTED = 2,     /* valid but not built (e.g. head_dim not 64/128) */
+    STATEKV_ERR_CACHE_FULL = 3,      /* a stream/layer already holds max_frames frames */
+    STATEKV_ERR_CUDA = 4,            /* a CUDA runtime call failed */
+    STATEKV_ERR_DEVICE_TIMEOUT = 5,  /* a kernel's bounded wait expired (sticky) */
+    STATEKV_ERR_ARENA_TOO_SMALL = 6  /* arena smaller than statekv_arena_bytes() */
+} statekv_status;
+
+typedef struct statekv_handle statekv_handle;
+
+typedef struct {
+    int32_t num_streams;      /* independent videos sharing the handle (>= 1) */
+    int32_t num_layers;       /* layers per stream (>= 1) */
+    int32_t num_q_heads;      /* Hq */
+    int32_t num_kv_heads;     /* Hkv, Hq % Hkv == 0 */
+    int32_t head_dim;         /* d: 64 or 128 */
+    int32_t tokens_per_frame; /* T >= 1 */
+    int32_t state_capacity;   /* B >= 0 (B = 0: no cross-frame context) */
+    int32_t max_frames;       /* decode-cache capacity per stream/layer, in frames */
+    int32_t causal_in_frame;  /* 1: key t visible to query i iff t <= i (Eq. 5's M_n);
+                                 0: every frame key visible (variant) */
+    int32_t host_staging;     /* 1: reserve arena space for statekv_prefill_frame_host */
+    float softmax_scale;      /* 0 -> 1 / sqrt(head_dim) (Eq. 5) */
+    uint32_t watchdog_ms;     /* bound on every device-side wait; 0 -> 2000 ms */
+} statekv_config;
+
+/* Bytes of device arena the configuration needs.  Returns INVALID_ARG or
+ * UNSUPPORTED for a bad configuration. */
+statekv_status statekv_arena_bytes(const statekv_config* cfg, size_t* bytes);
+
+/* Creates a handle over a caller-owned device arena of at least
+ * statekv_arena_bytes() bytes (256-byte aligned).  Zeroes the states
+ * (synchronously); every stream/layer starts at frame 1 with an empty state.
+ * The arena must outlive the handle. */
+statekv_status statekv_init(const statekv_config* cfg, void* device_arena, size_t arena_bytes,
+                            statekv_handle** out);
+
+typedef struct {
+    int32_t stream_begin, stream_count; /* streams [begin, begin + count) */
+    int32_t layer_begin, layer_count;   /* layers  [begin, begin + count) */
+    const void* q;                      /* bf16, layout above (device) */
+    const void* k;
+    const void* v;
+    void* out;                          /* bf16 attention output (device) */
+    float* importance;                  /* nullable fp32 (device): per KV head, columns
+                                           0..B-1 = state slots in their pre-call slot
+                                           order (empty slots 0), columns B..B+T-1 =
+                                           the frame's tokens */
+} statekv_frame_args;
+
+/* Processes the next frame of every (stream, layer) in the ranges: steps
+ * (a1)-(a5) above.  Each covered (stream, layer) advances by one frame.
+ * Returns CACHE_FULL (and enqueues nothing) if any of them already holds
+ * max_frames frames, and DEVICE_TIMEOUT if an earlier call's kernel reported
+ * an expired wait. */
+statekv_status statekv_prefill_frame(statekv_handle* h, const statekv_frame_args* args,
+                                     statekv_stream stream);
+
+/* Same step with HOST buffers (pinned memory recommended): q/k/v are copied
+ * into the arena's staging area, the step runs, and out (and importance if
+ * non-null) are copied back, all asynchronously on `stream`.  Host buffers
+ * must stay valid until the stream is synchronised.  Needs host_staging = 1. */
+statekv_status statekv_prefill_frame_host(statekv_handle* h, const statekv_frame_args* args,
+                                          statekv_stream stream);
+
+typedef struct {
+    const void* k;            /* bf16 [Hkv][B][d] (device); slot order is arbitrary */
+    const void* v;            /* bf16 [Hkv][B][d] (device) */
+    const int32_t* positions; /* int32 [Hkv][B] (device); virtual position, -1 = empty */
+    int32_t count;            /* valid slots per KV head: min(B, frames * T) */
+    int32_t frames;           /* frames processed */
+    int64_t virtual_len;      /* L_n = frames * T */
+} statekv_state_info;
+
+typedef struct {
+    const void* k;            /* bf16 [Hkv][capacity][d] (device) */
+    const void* v;
+    int64_t length;           /* rows written: frames * T */
+    int64_t capacity;         /* max_frames * T */
+} statekv_cache_info;
+
+/* Borrowed device pointers into the arena, valid until statekv_destroy.  The
+ * contents are current once the stream of the last prefill call is
+ * synchronised; the counters are host-side and current immediately. */
+statekv_status statekv_state_view(const statekv_handle* h, int32_t stream, int32_t layer,
+                                  statekv_state_info* out);
+statekv_status statekv_cache_view(const statekv_handle* h, int32_t stream, int32_t layer,
+                                  statekv_cache_info* out);
+
+/* Optional per-kernel timing with CUDA events recorded on the call's stream
+ * around each launch.  enable != 0 starts a new record; read synchronises on
+ * the recorded events and returns, per kernel kind (0 = decode-cache append,
+ * 1 = frame attention + importance, 2 = state select/gather), the number of
+ * launches and their summed device milliseconds. */
+typedef struct {
+    int64_t launches[3];
+    double milliseconds[3];
+} statekv_profile;
+statekv_status statekv_profile_enable(statekv_handle* h, int32_t enable);
+statekv_status statekv_profile_read(statekv_handle* h, statekv_profile* out);
+
+/* Synchronises the device and reports a device error (DEVICE_TIMEOUT) if a
+ * kernel recorded one. */
+statekv_status statekv_sync(statekv_handle* h);
+
+void statekv_destroy(statekv_handle* h);
+const char* statekv_status_string(statekv_status s);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* STATEKV_H */

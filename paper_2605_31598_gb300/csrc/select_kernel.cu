@@ -1,0 +1,263 @@
+// K3: importance reduction, top-B state selection and evict/admit gather
+//     (Sec. 3.3, Eq. 6; per layer and KV head as in App. A).
+// K4: decode-cache append (Sec. 3.2 detailed state; Sec. 3.3 "append").
+//
+// K3 runs one CTA per (unit, KV head):
+//   1. importance of every pool member = the fixed-order sum of the attention
+//      kernel's per-query-tile partials (deterministic);
+//   2. if the pool (count + T) fits in B, every frame token is admitted;
+//      otherwise the B best members by (score desc, position asc) are found
+//      with an MSB-first radix select over the 64-bit key
+//      (score bits << 32 | ~position) -- scores are non-negative floats, whose
+//      bit patterns order like the values, and positions are unique, so the
+//      keys are distinct and exactly B members are kept;
+//   3. evicted / empty slots (ascending) receive the admitted frame tokens
+//      (ascending) as 128-bit row copies, and their positions are updated.
+#include "statekv_kernels.cuh"
+
+namespace statekv {
+namespace {
+
+constexpr int kSelThreads = 512;
+constexpr int kSelWarps = kSelThreads / 32;
+
+// Exclusive block-wide scan of one int per thread; returns the total.
+__device__ __forceinline__ int block_exclusive_scan(int x, int* warp_sums, int& excl)
+{
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    int incl = x;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+    }
+    if (lane == 31) warp_sums[warp] = incl;
+    __syncthreads();
+    if (warp == 0) {
+        int w = lane < kSelWarps ? warp_sums[lane] : 0;
+        int wi = w;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, wi, o);
+            if (lane >= o) wi += y;
+        }
+        if (lane < kSelWarps) warp_sums[lane] = wi - w;  // exclusive warp offsets
+        if (lane == kSelWarps - 1) warp_sums[kSelWarps] = wi;
+    }
+    __syncthreads();
+    excl = warp_sums[warp] + incl - x;
+    const int total = warp_sums[kSelWarps];
+    __syncthreads();
+    return total;
+}
+
+__global__ void __launch_bounds__(kSelThreads)
+    state_select_gather(const SelectParams p)
+{
+    extern __shared__ __align__(16) uint8_t smem_raw[];
+    const int T = p.T, B = p.B, P = p.P, D = p.D;
+    uint64_t* key = reinterpret_cast<uint64_t*>(smem_raw);            // [P]
+    int* free_slot = reinterpret_cast<int*>(key + P);                  // [T]
+    int* adm_tok = free_slot + T;                                      // [T]
+    __shared__ unsigned hist[256];
+    __shared__ int warp_sums[kSelWarps + 1];
+    __shared__ unsigned long long sh_prefix, sh_mask;
+    __shared__ int sh_k, sh_done;
+
+    const int hkv = blockIdx.x, u = blockIdx.y;
+    const int ua = p.units.unit_abs(u);
+    const int tid = threadIdx.x, lane = tid & 31;
+    const size_t head = static_cast<size_t>(ua) * p.Hkv + hkv;
+    const int count = p.counts[head];
+    const int nf = p.frames[head];
+    const int L = nf * T;  // virtual length before this frame
+    int32_t* pos = p.positions + head * B;
+    const float* part = p.partials + (static_cast<size_t>(u) * p.Hkv + hkv) * p.MT * P;
+    float* imp_out =
+        p.importance ? p.importance + (static_cast<size_t>(u) * p.Hkv + hkv) * P : nullptr;
+    const int n = count + T;
+
+    // 1. importance (fixed-order sum over query tiles) and selection keys
+    for (int i = tid; i < n; i += kSelThreads) {
+        const int col = i < count ? i : B + (i - count);
+        float s = 0.f;
+        for (int mt = 0; mt < p.MT; ++mt) s += part[static_cast<size_t>(mt) * P + col];
+        const int ps = i < count ? pos[i] : L + (i - count);
+        key[i] = (static_cast<uint64_t>(__float_as_uint(s)) << 32) |
+                 static_cast<uint32_t>(0xFFFFFFFFu - static_cast<uint32_t>(ps));
+        if (imp_out) imp_out[col] = s;
+    }
+    if (imp_out)
+        for (int c = count + tid; c < B; c += kSelThreads) imp_out[c] = 0.f;
+    if (B == 0) {  // no compressed state: nothing is kept
+        if (tid == 0) p.frames[head] = nf + 1;
+        return;
+    }
+
+    // 2. top-B selection: kept(i) <=> (key[i] & mask) >= prefix
+    unsigned long long prefix = 0, mask = 0;
+    if (n > B) {
+        if (tid == 0) {
+            sh_k = B;
+            sh_done = 0;
+        }
+        __syncthreads();
+        for (int shift = 56; shift >= 0; shift -= 8) {
+            for (int i = tid; i < 256; i += kSelThreads) hist[i] = 0;
+            __syncthreads();
+            for (int i0 = 0; i0 < n; i0 += kSelThreads) {
+                const int i = i0 + tid;
+                int digit = -1;
+                if (i < n && (key[i] & mask) == prefix) digit = (key[i] >> shift) & 0xFF;
+                const unsigned peers = __match_any_sync(0xffffffffu, digit);
+                if (digit >= 0 && lane == __ffs(peers) - 1) atomicAdd(&hist[digit], __popc(peers));
+            }
+            __syncthreads();
+            if (tid < 32) {
+                // lane owns digits 255 - 8*lane - j, j = 0..7 (descending)
+                unsigned c[8], local = 0;
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    c[j] = hist[255 - 8 * lane - j];
+                    local += c[j];
+                }
+                unsigned incl = local;
+#pragma unroll
+                for (int o = 1; o < 32; o <<= 1) {
+                    const unsigned y = __shfl_up_sync(0xffffffffu, incl, o);
+                    if (lane >= o) incl += y;
+                }
+                const unsigned excl = incl - local;
+                const int k = sh_k;
+                const bool mine = excl < static_cast<unsigned>(k) && incl >= static_cast<unsigned>(k);
+                if (mine) {
+                    unsigned above = excl;
+#pragma unroll 1
+                    for (int j = 0; j < 8; ++j) {
+                        if (above + c[j] >= static_cast<unsigned>(k)) {
+                            const unsigned d = 255 - 8 * lane - j;
+                            const int k_rem = k - static_cast<int>(above);
+                            sh_prefix = prefix | (static_cast<unsigned long long>(d) << shift);
+                            sh_mask = mask | (0xFFull << shift);
+                            sh_k = k_rem;
+                            sh_done = (c[j] == static_cast<unsigned>(k_rem)) ? 1 : 0;
+                            break;
+                        }
+                        above += c[j];
+                    }
+                }
+            }
+            __syncthreads();
+            prefix = sh_prefix;
+            mask = sh_mask;
+            if (sh_done) break;
+        }
+        __syncthreads();
+    } else {
+        mask = 0;
+        prefix = 0;  // every member kept
+    }
+
+    // 3. free slots (evicted or empty, ascending) and admitted tokens (ascending)
+    const int per = (B + kSelThreads - 1) / kSelThreads;
+    int local_free = 0;
+    for (int s = tid * per; s < min(B, (tid + 1) * per); ++s)
+        local_free += (s >= count || (key[s] & mask) < prefix) ? 1 : 0;
+    int excl;
+    const int nfree = block_exclusive_scan(local_free, warp_sums, excl);
+    int slot_rank = excl;
+    for (int s = tid * per; s < min(B, (tid + 1) * per); ++s)
+        if (s >= count || (key[s] & mask) < prefix) {
+            if (slot_rank < T) free_slot[slot_rank] = s;
+            ++slot_rank;
+        }
+    const int tper = (T + kSelThreads - 1) / kSelThreads;
+    int local_adm = 0;
+    for (int t = tid * tper; t < min(T, (tid + 1) * tper); ++t)
+        local_adm += ((key[count + t] & mask) >= prefix) ? 1 : 0;
+    const int nadm = block_exclusive_scan(local_adm, warp_sums, excl);
+    int tok_rank = excl;
+    for (int t = tid * tper; t < min(T, (tid + 1) * tper); ++t)
+        if ((key[count + t] & mask) >= prefix) adm_tok[tok_rank++] = t;
+    __syncthreads();
+    const int npairs = min(nadm, nfree);
+    if (tid == 0 && nadm > nfree) *reinterpret_cast<volatile int32_t*>(p.status) = DEV_BAD_SELECT;
+
+    // 4. gather: 16-byte vector copies of the admitted K and V rows
+    const int chunks = D / 8;
+    const size_t src_stride = static_cast<size_t>(p.Hkv) * D;
+    const __nv_bfloat16* ksrc = p.k + (static_cast<size_t>(u) * T * p.Hkv + hkv) * D;
+    const __nv_bfloat16* vsrc = p.v + (static_cast<size_t>(u) * T * p.Hkv + hkv) * D;
+    __nv_bfloat16* kdst = p.state_k + head * B * D;
+    __nv_bfloat16* vdst = p.state_v + head * B * D;
+    for (int w = tid; w < npairs * chunks * 2; w += kSelThreads) {
+        const int which = w / (npairs * chunks);
+        const int r = w % (npairs * chunks);
+        const int i = r / chunks, ch = r % chunks;
+        const int t = adm_tok[i], s = free_slot[i];
+        const __nv_bfloat16* src = (which ? vsrc : ksrc) + t * src_stride + ch * 8;
+        __nv_bfloat16* dst = (which ? vdst : kdst) + static_cast<size_t>(s) * D + ch * 8;
+        *reinterpret_cast<uint4*>(dst) = *reinterpret_cast<const uint4*>(src);
+    }
+    for (int i = tid; i < npairs; i += kSelThreads) pos[free_slot[i]] = L + adm_tok[i];
+    if (tid == 0) {
+        p.counts[head] = min(B, count + T);
+        p.frames[head] = nf + 1;
+    }
+}
+
+// K4: D[hkv][L + t][:] = K[t][hkv][:] (and V), one 16-byte chunk per thread.
+__global__ void __launch_bounds__(256) decode_cache_append(const AppendParams p)
+{
+    const int chunks = p.D / 8;
+    const long long per_unit = static_cast<long long>(p.T) * p.Hkv * chunks;
+    const long long total = 2ll * p.U * per_unit;
+    for (long long w = blockIdx.x * 256ll + threadIdx.x; w < total; w += 256ll * gridDim.x) {
+        const int which = static_cast<int>(w / (p.U * per_unit));
+        const long long r = w % (p.U * per_unit);
+        const int u = static_cast<int>(r / per_unit);
+        const long long rr = r % per_unit;  // source order [t][hkv][chunk]
+        const int t = static_cast<int>(rr / (p.Hkv * chunks));
+        const int hkv = static_cast<int>((rr / chunks) % p.Hkv);
+        const int ch = static_cast<int>(rr % chunks);
+        const int ua = p.units.unit_abs(u);
+        const size_t head = static_cast<size_t>(ua) * p.Hkv + hkv;
+        const long long row = static_cast<long long>(p.frames[head]) * p.T + t;
+        const __nv_bfloat16* src = (which ? p.v : p.k) + static_cast<size_t>(u) * per_unit * 8 +
+                                   static_cast<size_t>(rr) * 8;
+        __nv_bfloat16* dst = (which ? p.cache_v : p.cache_k) +
+                             (head * p.cap + row) * p.D + ch * 8;
+        *reinterpret_cast<uint4*>(dst) = *reinterpret_cast<const uint4*>(src);
+    }
+}
+
+}  // namespace
+
+size_t select_smem_bytes(int P, int T)
+{
+    return static_cast<size_t>(P) * 8 + static_cast<size_t>(T) * 8;
+}
+
+cudaError_t select_prepare()
+{
+    return cudaFuncSetAttribute(state_select_gather, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                static_cast<int>(select_smem_bytes(kMaxPool, kMaxFrameTokens)));
+}
+
+cudaError_t launch_select(const SelectParams& p, int U, cudaStream_t st)
+{
+    const dim3 grid(p.Hkv, U);
+    state_select_gather<<<grid, kSelThreads, select_smem_bytes(p.P, p.T), st>>>(p);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_append(const AppendParams& p, cudaStream_t st)
+{
+    const long long total = 2ll * p.U * p.T * p.Hkv * (p.D / 8);
+    const long long blocks = (total + 255) / 256;
+    const int grid = static_cast<int>(blocks < 152ll * 64 ? blocks : 152ll * 64);
+    decode_cache_append<<<grid, 256, 0, st>>>(p);
+    return cudaGetLastError();
+}
+
+}  // namespace statekv

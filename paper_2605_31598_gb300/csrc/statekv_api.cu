@@ -1,0 +1,498 @@
+// Host runtime behind include/statekv.h: configuration checks, arena
+// carve-up, TMA descriptor encoding, launch sequencing and profiling.
+//
+// Per call, in stream order:  K4 append -> K1 attention -> K3 select/gather.
+// K4 reads the per-head frame counter before K3 advances it; K1 reads the
+// state before K3 rewrites it.
+#include "../../include/statekv.h"
+#include "statekv_kernels.cuh"
+
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstring>
+#include <mutex>
+#include <new>
+#include <vector>
+
+using namespace statekv;
+
+namespace {
+
+constexpr size_t kAlign = 256;
+constexpr int kProfPairs = 3 * 4096;
+
+size_t round_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
+
+struct Layout {
+    size_t state_k, state_v, positions, counts, frames, cache_k, cache_v, partials;
+    size_t stg_q, stg_k, stg_v, stg_out, stg_imp;
+    size_t total;
+};
+
+struct Derived {
+    int G, MT, P, SL;
+    long long cap;
+    float scale;
+};
+
+statekv_status check_config(const statekv_config* c, Derived* d)
+{
+    if (!c) return STATEKV_ERR_INVALID_ARG;
+    if (c->num_streams < 1 || c->num_layers < 1 || c->num_q_heads < 1 || c->num_kv_heads < 1 ||
+        c->num_q_heads % c->num_kv_heads != 0 || c->head_dim < 1 || c->tokens_per_frame < 1 ||
+        c->state_capacity < 0 || c->max_frames < 1 ||
+        (c->causal_in_frame != 0 && c->causal_in_frame != 1) ||
+        (c->host_staging != 0 && c->host_staging != 1) || !(c->softmax_scale >= 0.f) ||
+        !std::isfinite(c->softmax_scale))
+        return STATEKV_ERR_INVALID_ARG;
+    if (static_cast<long long>(c->max_frames) * c->tokens_per_frame > 0x7FFFFFFFll)
+        return STATEKV_ERR_INVALID_ARG;  // positions are int32
+    if (c->head_dim != 64 && c->head_dim != 128) return STATEKV_ERR_UNSUPPORTED;
+    if (c->tokens_per_frame > kMaxFrameTokens) return STATEKV_ERR_UNSUPPORTED;
+    if (static_cast<long long>(c->state_capacity) + c->tokens_per_frame > kMaxPool)
+        return STATEKV_ERR_UNSUPPORTED;
+    if (c->num_kv_heads > 65535 || static_cast<long long>(c->num_streams) * c->num_layers > 65535)
+        return STATEKV_ERR_UNSUPPORTED;
+    d->G = c->num_q_heads / c->num_kv_heads;
+    d->MT = static_cast<int>((static_cast<long long>(d->G) * c->tokens_per_frame + kBM - 1) / kBM);
+    d->P = c->state_capacity + c->tokens_per_frame;
+    d->SL = c->num_streams * c->num_layers;
+    d->cap = static_cast<long long>(c->max_frames) * c->tokens_per_frame;
+    d->scale = c->softmax_scale > 0.f ? c->softmax_scale
+                                      : 1.0f / std::sqrt(static_cast<float>(c->head_dim));
+    return STATEKV_OK;
+}
+
+Layout make_layout(const statekv_config& c, const Derived& d)
+{
+    Layout L{};
+    const size_t heads = static_cast<size_t>(d.SL) * c.num_kv_heads;
+    const size_t D = c.head_dim, B = c.state_capacity, T = c.tokens_per_frame;
+    size_t off = 0;
+    auto take = [&](size_t bytes) {
+        const size_t at = off;
+        off += round_up(bytes);
+        return at;
+    };
+    L.state_k = take(heads * B * D * 2);
+    L.state_v = take(heads * B * D * 2);
+    L.positions = take(heads * B * 4);
+    L.counts = take(heads * 4);
+    L.frames = take(heads * 4);
+    L.cache_k = take(heads * static_cast<size_t>(d.cap) * D * 2);
+    L.cache_v = take(heads * static_cast<size_t>(d.cap) * D * 2);
+    L.partials = take(heads * d.MT * static_cast<size_t>(d.P) * 4);
+    if (c.host_staging) {
+        L.stg_q = take(static_cast<size_t>(d.SL) * T * c.num_q_heads * D * 2);
+        L.stg_k = take(heads * T * D * 2);
+        L.stg_v = take(heads * T * D * 2);
+        L.stg_out = take(static_cast<size_t>(d.SL) * T * c.num_q_heads * D * 2);
+        L.stg_imp = take(heads * static_cast<size_t>(d.P) * 4);
+    }
+    L.total = off;
+    return L;
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn()
+{
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000,
+                                             cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    });
+    return fn;
+}
+
+// 4-D bf16 tensor map with a (64, b1, b2, 1) box and 128-byte swizzle; OOB
+// elements read as zero.
+bool encode_4d(CUtensorMap* m, const void* base, const cuuint64_t dims[4],
+               const cuuint64_t strides_bytes[3], const cuuint32_t box[4])
+{
+    auto fn = encode_fn();
+    if (!fn) return false;
+    const cuuint32_t es[4] = {1, 1, 1, 1};
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides_bytes,
+              box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+struct ProfRec {
+    cudaEvent_t a, b;
+    int kind;
+};
+
+}  // namespace
+
+struct statekv_handle {
+    statekv_config cfg;
+    Derived d;
+    Layout lay;
+    uint8_t* arena;
+    std::vector<int32_t> frames_host;  // [S*L]
+    CUtensorMap tm_sk, tm_sv;
+    volatile int32_t* status_host;
+    int32_t* status_dev;
+    bool prof_on;
+    size_t prof_used;
+    std::vector<ProfRec> prof;
+
+    template <class T>
+    T* at(size_t off) const { return reinterpret_cast<T*>(arena + off); }
+};
+
+namespace {
+
+statekv_status check_args(const statekv_handle* h, const statekv_frame_args* a, bool host)
+{
+    if (!h || !a) return STATEKV_ERR_INVALID_ARG;
+    const statekv_config& c = h->cfg;
+    if (a->stream_count < 1 || a->layer_count < 1 || a->stream_begin < 0 || a->layer_begin < 0 ||
+        a->stream_begin + a->stream_count > c.num_streams ||
+        a->layer_begin + a->layer_count > c.num_layers)
+        return STATEKV_ERR_INVALID_ARG;
+    if (!a->q || !a->k || !a->v || !a->out) return STATEKV_ERR_INVALID_ARG;
+    if (!host) {
+        if (!aligned(a->q, 16) || !aligned(a->k, 16) || !aligned(a->v, 16) || !aligned(a->out, 16) ||
+            (a->importance && !aligned(a->importance, 4)))
+            return STATEKV_ERR_INVALID_ARG;
+    }
+    if (host && !c.host_staging) return STATEKV_ERR_INVALID_ARG;
+    if (*h->status_host != 0) return STATEKV_ERR_DEVICE_TIMEOUT;
+    for (int s = a->stream_begin; s < a->stream_begin + a->stream_count; ++s)
+        for (int l = a->layer_begin; l < a->layer_begin + a->layer_count; ++l)
+            if (h->frames_host[static_cast<size_t>(s) * c.num_layers + l] >= c.max_frames)
+                return STATEKV_ERR_CACHE_FULL;
+    return STATEKV_OK;
+}
+
+template <class F>
+cudaError_t timed(statekv_handle* h, int kind, cudaStream_t st, F&& launch)
+{
+    ProfRec* r = nullptr;
+    if (h->prof_on && h->prof_used < h->prof.size()) {
+        r = &h->prof[h->prof_used++];
+        r->kind = kind;
+        cudaEventRecord(r->a, st);
+    }
+    cudaError_t e = launch();
+    if (r) cudaEventRecord(r->b, st);
+    return e;
+}
+
+statekv_status run_step(statekv_handle* h, const statekv_frame_args& a, cudaStream_t st)
+{
+    const statekv_config& c = h->cfg;
+    const Derived& d = h->d;
+    const int U = a.stream_count * a.layer_count;
+    const int D = c.head_dim, T = c.tokens_per_frame, Hkv = c.num_kv_heads;
+    const UnitRange ur{a.stream_begin, a.layer_begin, a.layer_count, c.num_layers};
+
+    CUtensorMap tm_fk, tm_fv;
+    {
+        const cuuint64_t dims[4] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(Hkv),
+                                    static_cast<cuuint64_t>(T), static_cast<cuuint64_t>(U)};
+        const cuuint64_t strides[3] = {static_cast<cuuint64_t>(D) * 2,
+                                       static_cast<cuuint64_t>(Hkv) * D * 2,
+                                       static_cast<cuuint64_t>(T) * Hkv * D * 2};
+        const cuuint32_t box[4] = {64, 1, static_cast<cuuint32_t>(kBN), 1};
+        if (!encode_4d(&tm_fk, a.k, dims, strides, box) ||
+            !encode_4d(&tm_fv, a.v, dims, strides, box))
+            return STATEKV_ERR_CUDA;
+    }
+    int32_t* counts = h->at<int32_t>(h->lay.counts);
+    int32_t* frames = h->at<int32_t>(h->lay.frames);
+    float* partials = h->at<float>(h->lay.partials);
+
+    AppendParams ap{};
+    ap.k = static_cast<const __nv_bfloat16*>(a.k);
+    ap.v = static_cast<const __nv_bfloat16*>(a.v);
+    ap.cache_k = h->at<__nv_bfloat16>(h->lay.cache_k);
+    ap.cache_v = h->at<__nv_bfloat16>(h->lay.cache_v);
+    ap.frames = frames;
+    ap.units = ur;
+    ap.U = U;
+    ap.T = T;
+    ap.Hkv = Hkv;
+    ap.D = D;
+    ap.cap = d.cap;
+    if (timed(h, 0, st, [&] { return launch_append(ap, st); }) != cudaSuccess)
+        return STATEKV_ERR_CUDA;
+
+    AttnParams pa{};
+    pa.q = static_cast<const __nv_bfloat16*>(a.q);
+    pa.out = static_cast<__nv_bfloat16*>(a.out);
+    pa.partials = partials;
+    pa.counts = counts;
+    pa.status = h->status_dev;
+    pa.units = ur;
+    pa.T = T;
+    pa.Hq = c.num_q_heads;
+    pa.Hkv = Hkv;
+    pa.G = d.G;
+    pa.B = c.state_capacity;
+    pa.P = d.P;
+    pa.MT = d.MT;
+    pa.causal = c.causal_in_frame;
+    pa.scale_log2 = d.scale * 1.4426950408889634f;
+    pa.watchdog_ns = 1000000ull * (c.watchdog_ms ? c.watchdog_ms : 2000u);
+    if (timed(h, 1, st, [&] { return launch_attn(D, h->tm_sk, h->tm_sv, tm_fk, tm_fv, pa, U, st); }) !=
+        cudaSuccess)
+        return STATEKV_ERR_CUDA;
+
+    SelectParams ps{};
+    ps.partials = partials;
+    ps.importance = a.importance;
+    ps.k = ap.k;
+    ps.v = ap.v;
+    ps.state_k = h->at<__nv_bfloat16>(h->lay.state_k);
+    ps.state_v = h->at<__nv_bfloat16>(h->lay.state_v);
+    ps.positions = h->at<int32_t>(h->lay.positions);
+    ps.counts = counts;
+    ps.frames = frames;
+    ps.status = h->status_dev;
+    ps.units = ur;
+    ps.T = T;
+    ps.Hkv = Hkv;
+    ps.D = D;
+    ps.B = c.state_capacity;
+    ps.P = d.P;
+    ps.MT = d.MT;
+    if (timed(h, 2, st, [&] { return launch_select(ps, U, st); }) != cudaSuccess)
+        return STATEKV_ERR_CUDA;
+
+    for (int s = a.stream_begin; s < a.stream_begin + a.stream_count; ++s)
+        for (int l = a.layer_begin; l < a.layer_begin + a.layer_count; ++l)
+            ++h->frames_host[static_cast<size_t>(s) * c.num_layers + l];
+    return STATEKV_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+statekv_status statekv_arena_bytes(const statekv_config* cfg, size_t* bytes)
+{
+    Derived d;
+    const statekv_status s = check_config(cfg, &d);
+    if (s != STATEKV_OK) return s;
+    if (!bytes) return STATEKV_ERR_INVALID_ARG;
+    *bytes = make_layout(*cfg, d).total;
+    return STATEKV_OK;
+}
+
+statekv_status statekv_init(const statekv_config* cfg, void* device_arena, size_t arena_bytes,
+                            statekv_handle** out)
+{
+    Derived d;
+    statekv_status s = check_config(cfg, &d);
+    if (s != STATEKV_OK) return s;
+    if (!out || !device_arena || !aligned(device_arena, kAlign)) return STATEKV_ERR_INVALID_ARG;
+    const Layout lay = make_layout(*cfg, d);
+    if (arena_bytes < lay.total) return STATEKV_ERR_ARENA_TOO_SMALL;
+    if (!encode_fn()) return STATEKV_ERR_CUDA;
+
+    statekv_handle* h = new (std::nothrow) statekv_handle();
+    if (!h) return STATEKV_ERR_CUDA;
+    h->cfg = *cfg;
+    h->d = d;
+    h->lay = lay;
+    h->arena = static_cast<uint8_t*>(device_arena);
+    h->frames_host.assign(static_cast<size_t>(d.SL), 0);
+    h->prof_on = false;
+    h->prof_used = 0;
+    std::memset(&h->tm_sk, 0, sizeof(CUtensorMap));
+    std::memset(&h->tm_sv, 0, sizeof(CUtensorMap));
+
+    void* st_host = nullptr;
+    if (cudaHostAlloc(&st_host, 64, cudaHostAllocMapped) != cudaSuccess) {
+        delete h;
+        return STATEKV_ERR_CUDA;
+    }
+    h->status_host = static_cast<volatile int32_t*>(st_host);
+    *h->status_host = 0;
+    void* st_dev = nullptr;
+    if (cudaHostGetDevicePointer(&st_dev, st_host, 0) != cudaSuccess) {
+        cudaFreeHost(st_host);
+        delete h;
+        return STATEKV_ERR_CUDA;
+    }
+    h->status_dev = static_cast<int32_t*>(st_dev);
+
+    const int D = cfg->head_dim, B = cfg->state_capacity, Hkv = cfg->num_kv_heads;
+    bool ok = attn_prepare(D) == cudaSuccess && select_prepare() == cudaSuccess;
+    if (ok && B > 0) {
+        const cuuint64_t dims[4] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(B),
+                                    static_cast<cuuint64_t>(Hkv), static_cast<cuuint64_t>(d.SL)};
+        const cuuint64_t strides[3] = {static_cast<cuuint64_t>(D) * 2,
+                                       static_cast<cuuint64_t>(B) * D * 2,
+                                       static_cast<cuuint64_t>(Hkv) * B * D * 2};
+        const cuuint32_t box[4] = {64, static_cast<cuuint32_t>(kBN), 1, 1};
+        ok = encode_4d(&h->tm_sk, h->arena + lay.state_k, dims, strides, box) &&
+             encode_4d(&h->tm_sv, h->arena + lay.state_v, dims, strides, box);
+    }
+    // Empty states: zero rows (masked keys must still be finite), positions -1.
+    ok = ok && cudaMemset(h->arena + lay.state_k, 0, lay.positions - lay.state_k) == cudaSuccess &&
+         cudaMemset(h->arena + lay.positions, 0xFF, lay.counts - lay.positions) == cudaSuccess &&
+         cudaMemset(h->arena + lay.counts, 0, lay.cache_k - lay.counts) == cudaSuccess &&
+         cudaDeviceSynchronize() == cudaSuccess;
+    if (!ok) {
+        cudaFreeHost(st_host);
+        delete h;
+        return STATEKV_ERR_CUDA;
+    }
+    *out = h;
+    return STATEKV_OK;
+}
+
+statekv_status statekv_prefill_frame(statekv_handle* h, const statekv_frame_args* args,
+                                     statekv_stream stream)
+{
+    const statekv_status s = check_args(h, args, false);
+    if (s != STATEKV_OK) return s;
+    return run_step(h, *args, reinterpret_cast<cudaStream_t>(stream));
+}
+
+statekv_status statekv_prefill_frame_host(statekv_handle* h, const statekv_frame_args* args,
+                                          statekv_stream stream)
+{
+    const statekv_status s = check_args(h, args, true);
+    if (s != STATEKV_OK) return s;
+    const statekv_config& c = h->cfg;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    const size_t U = static_cast<size_t>(args->stream_count) * args->layer_count;
+    const size_t T = c.tokens_per_frame, D = c.head_dim;
+    const size_t qbytes = U * T * c.num_q_heads * D * 2;
+    const size_t kvbytes = U * T * c.num_kv_heads * D * 2;
+    const size_t impbytes = U * c.num_kv_heads * static_cast<size_t>(h->d.P) * 4;
+    statekv_frame_args dev = *args;
+    dev.q = h->arena + h->lay.stg_q;
+    dev.k = h->arena + h->lay.stg_k;
+    dev.v = h->arena + h->lay.stg_v;
+    dev.out = h->arena + h->lay.stg_out;
+    dev.importance = args->importance ? h->at<float>(h->lay.stg_imp) : nullptr;
+    if (cudaMemcpyAsync(const_cast<void*>(dev.q), args->q, qbytes, cudaMemcpyHostToDevice, st) !=
+            cudaSuccess ||
+        cudaMemcpyAsync(const_cast<void*>(dev.k), args->k, kvbytes, cudaMemcpyHostToDevice, st) !=
+            cudaSuccess ||
+        cudaMemcpyAsync(const_cast<void*>(dev.v), args->v, kvbytes, cudaMemcpyHostToDevice, st) !=
+            cudaSuccess)
+        return STATEKV_ERR_CUDA;
+    const statekv_status r = run_step(h, dev, st);
+    if (r != STATEKV_OK) return r;
+    if (cudaMemcpyAsync(args->out, dev.out, qbytes, cudaMemcpyDeviceToHost, st) != cudaSuccess)
+        return STATEKV_ERR_CUDA;
+    if (args->importance &&
+        cudaMemcpyAsync(args->importance, dev.importance, impbytes, cudaMemcpyDeviceToHost, st) !=
+            cudaSuccess)
+        return STATEKV_ERR_CUDA;
+    return STATEKV_OK;
+}
+
+statekv_status statekv_state_view(const statekv_handle* h, int32_t stream, int32_t layer,
+                                  statekv_state_info* out)
+{
+    if (!h || !out || stream < 0 || layer < 0 || stream >= h->cfg.num_streams ||
+        layer >= h->cfg.num_layers)
+        return STATEKV_ERR_INVALID_ARG;
+    const size_t unit = static_cast<size_t>(stream) * h->cfg.num_layers + layer;
+    const size_t per = static_cast<size_t>(h->cfg.num_kv_heads) * h->cfg.state_capacity;
+    out->k = h->arena + h->lay.state_k + unit * per * h->cfg.head_dim * 2;
+    out->v = h->arena + h->lay.state_v + unit * per * h->cfg.head_dim * 2;
+    out->positions = h->at<int32_t>(h->lay.positions) + unit * per;
+    const int32_t f = h->frames_host[unit];
+    const long long filled = static_cast<long long>(f) * h->cfg.tokens_per_frame;
+    out->frames = f;
+    out->count = static_cast<int32_t>(filled < h->cfg.state_capacity ? filled : h->cfg.state_capacity);
+    out->virtual_len = filled;
+    return STATEKV_OK;
+}
+
+statekv_status statekv_cache_view(const statekv_handle* h, int32_t stream, int32_t layer,
+                                  statekv_cache_info* out)
+{
+    if (!h || !out || stream < 0 || layer < 0 || stream >= h->cfg.num_streams ||
+        layer >= h->cfg.num_layers)
+        return STATEKV_ERR_INVALID_ARG;
+    const size_t unit = static_cast<size_t>(stream) * h->cfg.num_layers + layer;
+    const size_t per = static_cast<size_t>(h->cfg.num_kv_heads) * h->d.cap * h->cfg.head_dim * 2;
+    out->k = h->arena + h->lay.cache_k + unit * per;
+    out->v = h->arena + h->lay.cache_v + unit * per;
+    out->length = static_cast<int64_t>(h->frames_host[unit]) * h->cfg.tokens_per_frame;
+    out->capacity = h->d.cap;
+    return STATEKV_OK;
+}
+
+statekv_status statekv_profile_enable(statekv_handle* h, int32_t enable)
+{
+    if (!h) return STATEKV_ERR_INVALID_ARG;
+    if (enable && h->prof.empty()) {
+        h->prof.resize(kProfPairs);
+        for (auto& r : h->prof)
+            if (cudaEventCreate(&r.a) != cudaSuccess || cudaEventCreate(&r.b) != cudaSuccess)
+                return STATEKV_ERR_CUDA;
+    }
+    if (enable) h->prof_used = 0;
+    h->prof_on = enable != 0;
+    return STATEKV_OK;
+}
+
+statekv_status statekv_profile_read(statekv_handle* h, statekv_profile* out)
+{
+    if (!h || !out) return STATEKV_ERR_INVALID_ARG;
+    std::memset(out, 0, sizeof(*out));
+    for (size_t i = 0; i < h->prof_used; ++i) {
+        const ProfRec& r = h->prof[i];
+        float ms = 0.f;
+        if (cudaEventSynchronize(r.b) != cudaSuccess ||
+            cudaEventElapsedTime(&ms, r.a, r.b) != cudaSuccess)
+            return STATEKV_ERR_CUDA;
+        out->launches[r.kind] += 1;
+        out->milliseconds[r.kind] += ms;
+    }
+    return STATEKV_OK;
+}
+
+statekv_status statekv_sync(statekv_handle* h)
+{
+    if (!h) return STATEKV_ERR_INVALID_ARG;
+    if (cudaDeviceSynchronize() != cudaSuccess) return STATEKV_ERR_CUDA;
+    return *h->status_host != 0 ? STATEKV_ERR_DEVICE_TIMEOUT : STATEKV_OK;
+}
+
+void statekv_destroy(statekv_handle* h)
+{
+    if (!h) return;
+    for (auto& r : h->prof) {
+        cudaEventDestroy(r.a);
+        cudaEventDestroy(r.b);
+    }
+    cudaFreeHost(const_cast<int32_t*>(h->status_host));
+    delete h;
+}
+
+const char* statekv_status_string(statekv_status s)
+{
+    switch (s) {
+    case STATEKV_OK: return "ok";
+    case STATEKV_ERR_INVALID_ARG: return "invalid argument";
+    case STATEKV_ERR_UNSUPPORTED: return "unsupported configuration";
+    case STATEKV_ERR_CACHE_FULL: return "decode cache full (max_frames reached)";
+    case STATEKV_ERR_CUDA: return "CUDA runtime error";
+    case STATEKV_ERR_DEVICE_TIMEOUT: return "device wait timed out";
+    case STATEKV_ERR_ARENA_TOO_SMALL: return "arena too small";
+    }
+    return "unknown status";
+}
+
+}  // extern "C"

@@ -1,0 +1,92 @@
+// Kernel parameter blocks and launchers of the StateKV per-frame step.
+//
+//   K4  decode-cache append   (Sec. 3.2 / 3.3: D_n = D_{n-1} + (K_n, V_n))
+//   K1  frame attention + LSE + fused importance partials (Eq. 5, Eq. 1, App. B.1)
+//   K3  importance reduction, top-B select, evict/admit gather (Eq. 6)
+//
+// A "unit" is one (stream, layer) of the current call; `unit_abs` indexes the
+// arena (stream * num_layers + layer), `u` indexes the call's buffers.
+#pragma once
+
+#include <cstdint>
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+namespace statekv {
+
+// Device error codes written to the status word (0 = no error).
+enum DeviceError : int32_t {
+    DEV_OK = 0,
+    DEV_TIMEOUT_ATTN = 1,
+    DEV_BAD_SELECT = 2,
+};
+
+// Tile sizes of the attention kernel: 128 query rows x 128 keys per MMA tile.
+constexpr int kBM = 128;
+constexpr int kBN = 128;
+
+struct UnitRange {
+    int stream_begin, layer_begin, layer_count, num_layers;
+    __host__ __device__ int unit_abs(int u) const
+    {
+        return (stream_begin + u / layer_count) * num_layers + layer_begin + u % layer_count;
+    }
+};
+
+struct AttnParams {
+    const __nv_bfloat16* q;   // [U][T][Hq][D]
+    __nv_bfloat16* out;       // [U][T][Hq][D]
+    float* partials;          // [U][Hkv][MT][P]
+    const int32_t* counts;    // arena [S*L][Hkv]
+    int32_t* status;          // device-visible status word
+    UnitRange units;
+    int T, Hq, Hkv, G, B, P, MT;
+    int causal;
+    float scale_log2;         // softmax scale * log2(e)
+    unsigned long long watchdog_ns;
+};
+
+struct SelectParams {
+    const float* partials;      // [U][Hkv][MT][P]
+    float* importance;          // nullable [U][Hkv][P]
+    const __nv_bfloat16* k;     // [U][T][Hkv][D]
+    const __nv_bfloat16* v;
+    __nv_bfloat16* state_k;     // arena [S*L][Hkv][B][D]
+    __nv_bfloat16* state_v;
+    int32_t* positions;         // arena [S*L][Hkv][B]
+    int32_t* counts;            // arena [S*L][Hkv]
+    int32_t* frames;            // arena [S*L][Hkv]
+    int32_t* status;
+    UnitRange units;
+    int T, Hkv, D, B, P, MT;
+};
+
+struct AppendParams {
+    const __nv_bfloat16* k;     // [U][T][Hkv][D]
+    const __nv_bfloat16* v;
+    __nv_bfloat16* cache_k;     // arena [S*L][Hkv][cap][D]
+    __nv_bfloat16* cache_v;
+    const int32_t* frames;      // arena [S*L][Hkv]
+    UnitRange units;
+    int U, T, Hkv, D;
+    long long cap;
+};
+
+// Shared-memory bytes the attention kernel needs for head dim D.
+size_t attn_smem_bytes(int D);
+// Largest pool (B + T) the select kernel keeps in shared memory, and the
+// largest frame (T) it lists.
+constexpr int kMaxPool = 24576;
+constexpr int kMaxFrameTokens = 4096;
+size_t select_smem_bytes(int P, int T);
+
+cudaError_t attn_prepare(int D);
+cudaError_t select_prepare();
+cudaError_t launch_attn(int D, const CUtensorMap& tm_sk, const CUtensorMap& tm_sv,
+                        const CUtensorMap& tm_fk, const CUtensorMap& tm_fv, const AttnParams& p,
+                        int U, cudaStream_t st);
+cudaError_t launch_select(const SelectParams& p, int U, cudaStream_t st);
+cudaError_t launch_append(const AppendParams& p, cudaStream_t st);
+
+}  // namespace statekv

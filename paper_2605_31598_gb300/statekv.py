@@ -1,0 +1,279 @@
+"""ctypes binding of ``include/statekv.h`` (argument marshalling only).
+
+Every function of the C ABI is exposed under its own name; ``StateKV`` is a
+small convenience owner that allocates the device arena with torch (PyTorch
+is used for device memory and streams only) and passes raw pointers through.
+Every step of the path runs in the CUDA library; there is no fallback: if the
+library is missing the first call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(PKG, "libstatekv.so")
+
+STATEKV_OK = 0
+STATUS_NAMES = {
+    0: "STATEKV_OK", 1: "STATEKV_ERR_INVALID_ARG", 2: "STATEKV_ERR_UNSUPPORTED",
+    3: "STATEKV_ERR_CACHE_FULL", 4: "STATEKV_ERR_CUDA", 5: "STATEKV_ERR_DEVICE_TIMEOUT",
+    6: "STATEKV_ERR_ARENA_TOO_SMALL",
+}
+EXPORTED = ("statekv_arena_bytes", "statekv_init", "statekv_prefill_frame",
+            "statekv_prefill_frame_host", "statekv_state_view", "statekv_cache_view",
+            "statekv_profile_enable", "statekv_profile_read", "statekv_sync",
+            "statekv_destroy", "statekv_status_string")
+
+
+class statekv_config(ctypes.Structure):
+    _fields_ = [("num_streams", ctypes.c_int32), ("num_layers", ctypes.c_int32),
+                ("num_q_heads", ctypes.c_int32), ("num_kv_heads", ctypes.c_int32),
+                ("head_dim", ctypes.c_int32), ("tokens_per_frame", ctypes.c_int32),
+                ("state_capacity", ctypes.c_int32), ("max_frames", ctypes.c_int32),
+                ("causal_in_frame", ctypes.c_int32), ("host_staging", ctypes.c_int32),
+                ("softmax_scale", ctypes.c_float), ("watchdog_ms", ctypes.c_uint32)]
+
+
+class statekv_frame_args(ctypes.Structure):
+    _fields_ = [("stream_begin", ctypes.c_int32), ("stream_count", ctypes.c_int32),
+                ("layer_begin", ctypes.c_int32), ("layer_count", ctypes.c_int32),
+                ("q", ctypes.c_void_p), ("k", ctypes.c_void_p), ("v", ctypes.c_void_p),
+                ("out", ctypes.c_void_p), ("importance", ctypes.c_void_p)]
+
+
+class statekv_state_info(ctypes.Structure):
+    _fields_ = [("k", ctypes.c_void_p), ("v", ctypes.c_void_p), ("positions", ctypes.c_void_p),
+                ("count", ctypes.c_int32), ("frames", ctypes.c_int32),
+                ("virtual_len", ctypes.c_int64)]
+
+
+class statekv_cache_info(ctypes.Structure):
+    _fields_ = [("k", ctypes.c_void_p), ("v", ctypes.c_void_p), ("length", ctypes.c_int64),
+                ("capacity", ctypes.c_int64)]
+
+
+class statekv_profile(ctypes.Structure):
+    _fields_ = [("launches", ctypes.c_int64 * 3), ("milliseconds", ctypes.c_double * 3)]
+
+
+_lock = threading.Lock()
+_lib = None
+
+
+def lib() -> ctypes.CDLL:
+    """The loaded C library (raises if it has not been built)."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            if not os.path.exists(LIB_PATH):
+                raise RuntimeError(
+                    f"{LIB_PATH} is missing: build the CUDA library first "
+                    "(python -c 'import __graft_entry__ as g; g.build()')")
+            L = ctypes.CDLL(LIB_PATH)
+            P = ctypes.POINTER
+            st = ctypes.c_int
+            L.statekv_arena_bytes.argtypes = [P(statekv_config), P(ctypes.c_size_t)]
+            L.statekv_arena_bytes.restype = st
+            L.statekv_init.argtypes = [P(statekv_config), ctypes.c_void_p, ctypes.c_size_t,
+                                       P(ctypes.c_void_p)]
+            L.statekv_init.restype = st
+            for name in ("statekv_prefill_frame", "statekv_prefill_frame_host"):
+                fn = getattr(L, name)
+                fn.argtypes = [ctypes.c_void_p, P(statekv_frame_args), ctypes.c_void_p]
+                fn.restype = st
+            L.statekv_state_view.argtypes = [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32,
+                                             P(statekv_state_info)]
+            L.statekv_state_view.restype = st
+            L.statekv_cache_view.argtypes = [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32,
+                                             P(statekv_cache_info)]
+            L.statekv_cache_view.restype = st
+            L.statekv_profile_enable.argtypes = [ctypes.c_void_p, ctypes.c_int32]
+            L.statekv_profile_enable.restype = st
+            L.statekv_profile_read.argtypes = [ctypes.c_void_p, P(statekv_profile)]
+            L.statekv_profile_read.restype = st
+            L.statekv_sync.argtypes = [ctypes.c_void_p]
+            L.statekv_sync.restype = st
+            L.statekv_destroy.argtypes = [ctypes.c_void_p]
+            L.statekv_destroy.restype = None
+            L.statekv_status_string.argtypes = [ctypes.c_int]
+            L.statekv_status_string.restype = ctypes.c_char_p
+            _lib = L
+    return _lib
+
+
+class StateKVError(RuntimeError):
+    def __init__(self, status: int, what: str):
+        self.status = status
+        msg = lib().statekv_status_string(status).decode()
+        super().__init__(f"{what}: {STATUS_NAMES.get(status, status)} ({msg})")
+
+
+def check(status: int, what: str):
+    if status != STATEKV_OK:
+        raise StateKVError(status, what)
+
+
+# ---------------------------------------------------------------- C ABI names
+def statekv_arena_bytes(cfg: statekv_config) -> int:
+    n = ctypes.c_size_t(0)
+    check(lib().statekv_arena_bytes(ctypes.byref(cfg), ctypes.byref(n)), "statekv_arena_bytes")
+    return n.value
+
+
+def statekv_init(cfg: statekv_config, arena_ptr: int, arena_bytes: int) -> int:
+    h = ctypes.c_void_p(0)
+    check(lib().statekv_init(ctypes.byref(cfg), ctypes.c_void_p(arena_ptr), arena_bytes,
+                             ctypes.byref(h)), "statekv_init")
+    return h.value
+
+
+def statekv_prefill_frame(handle: int, args: statekv_frame_args, stream: int) -> int:
+    return lib().statekv_prefill_frame(handle, ctypes.byref(args), ctypes.c_void_p(stream))
+
+
+def statekv_prefill_frame_host(handle: int, args: statekv_frame_args, stream: int) -> int:
+    return lib().statekv_prefill_frame_host(handle, ctypes.byref(args), ctypes.c_void_p(stream))
+
+
+def statekv_state_view(handle: int, stream: int, layer: int) -> statekv_state_info:
+    info = statekv_state_info()
+    check(lib().statekv_state_view(handle, stream, layer, ctypes.byref(info)),
+          "statekv_state_view")
+    return info
+
+
+def statekv_cache_view(handle: int, stream: int, layer: int) -> statekv_cache_info:
+    info = statekv_cache_info()
+    check(lib().statekv_cache_view(handle, stream, layer, ctypes.byref(info)),
+          "statekv_cache_view")
+    return info
+
+
+def statekv_profile_enable(handle: int, enable: bool):
+    check(lib().statekv_profile_enable(handle, 1 if enable else 0), "statekv_profile_enable")
+
+
+def statekv_profile_read(handle: int) -> statekv_profile:
+    prof = statekv_profile()
+    check(lib().statekv_profile_read(handle, ctypes.byref(prof)), "statekv_profile_read")
+    return prof
+
+
+def statekv_sync(handle: int) -> int:
+    return lib().statekv_sync(handle)
+
+
+def statekv_destroy(handle: int):
+    lib().statekv_destroy(handle)
+
+
+def statekv_status_string(status: int) -> str:
+    return lib().statekv_status_string(status).decode()
+
+
+# ---------------------------------------------------------------- owner object
+def make_config(shape, *, causal=True, host_staging=False, softmax_scale=0.0,
+                watchdog_ms=0) -> statekv_config:
+    """statekv_config from an ``inputs.Shape``-like object."""
+    return statekv_config(shape.num_streams, shape.num_layers, shape.num_q_heads,
+                          shape.num_kv_heads, shape.head_dim, shape.tokens_per_frame,
+                          shape.state_capacity, shape.max_frames, 1 if causal else 0,
+                          1 if host_staging else 0, softmax_scale, watchdog_ms)
+
+
+class StateKV:
+    """Owns a handle and its torch-allocated device arena."""
+
+    def __init__(self, cfg: statekv_config, device="cuda"):
+        import torch
+
+        self.cfg = cfg
+        self.nbytes = statekv_arena_bytes(cfg)
+        self.arena = torch.empty(max(self.nbytes, 256), dtype=torch.uint8, device=device)
+        self.handle = statekv_init(cfg, self.arena.data_ptr(), self.nbytes)
+
+    def close(self):
+        if getattr(self, "handle", None):
+            statekv_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def _args(self, q, k, v, out, importance, stream_begin, stream_count, layer_begin,
+              layer_count):
+        return statekv_frame_args(stream_begin, stream_count, layer_begin, layer_count,
+                                  q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr(),
+                                  importance.data_ptr() if importance is not None else None)
+
+    def prefill_frame(self, q, k, v, out, importance=None, *, stream_begin=0, stream_count=None,
+                      layer_begin=0, layer_count=None, stream=None) -> int:
+        """Enqueue one frame step on ``stream`` (torch current stream by default).
+
+        Returns the C status code (0 = OK); the caller decides how to react."""
+        import torch
+
+        sc = self.cfg.num_streams - stream_begin if stream_count is None else stream_count
+        lc = self.cfg.num_layers - layer_begin if layer_count is None else layer_count
+        st = (stream or torch.cuda.current_stream()).cuda_stream
+        args = self._args(q, k, v, out, importance, stream_begin, sc, layer_begin, lc)
+        return statekv_prefill_frame(self.handle, args, st)
+
+    def prefill_frame_host(self, q, k, v, out, importance=None, *, stream_begin=0,
+                           stream_count=None, layer_begin=0, layer_count=None,
+                           stream=None) -> int:
+        import torch
+
+        sc = self.cfg.num_streams - stream_begin if stream_count is None else stream_count
+        lc = self.cfg.num_layers - layer_begin if layer_count is None else layer_count
+        st = (stream or torch.cuda.current_stream()).cuda_stream
+        args = self._args(q, k, v, out, importance, stream_begin, sc, layer_begin, lc)
+        return statekv_prefill_frame_host(self.handle, args, st)
+
+    def _arena_view(self, ptr, nbytes, dtype, shape):
+        import torch
+
+        off = ptr - self.arena.data_ptr()
+        assert 0 <= off and off + nbytes <= self.arena.numel()
+        return self.arena[off: off + nbytes].view(dtype).view(shape)
+
+    def state(self, stream: int, layer: int):
+        """(k [Hkv][B][d] bf16, v, positions [Hkv][B] int32, info) views into the arena."""
+        import torch
+
+        c = self.cfg
+        info = statekv_state_view(self.handle, stream, layer)
+        H, B, d = c.num_kv_heads, c.state_capacity, c.head_dim
+        if B == 0:
+            e = torch.empty((H, 0, d), dtype=torch.bfloat16, device=self.arena.device)
+            return e, e, torch.empty((H, 0), dtype=torch.int32, device=self.arena.device), info
+        kk = self._arena_view(info.k, H * B * d * 2, torch.bfloat16, (H, B, d))
+        vv = self._arena_view(info.v, H * B * d * 2, torch.bfloat16, (H, B, d))
+        pp = self._arena_view(info.positions, H * B * 4, torch.int32, (H, B))
+        return kk, vv, pp, info
+
+    def cache(self, stream: int, layer: int):
+        """(k [Hkv][capacity][d] bf16, v, info) views into the arena."""
+        import torch
+
+        c = self.cfg
+        info = statekv_cache_view(self.handle, stream, layer)
+        H, cap, d = c.num_kv_heads, info.capacity, c.head_dim
+        kk = self._arena_view(info.k, H * cap * d * 2, torch.bfloat16, (H, cap, d))
+        vv = self._arena_view(info.v, H * cap * d * 2, torch.bfloat16, (H, cap, d))
+        return kk, vv, info
+
+    def profile(self, enable: bool):
+        statekv_profile_enable(self.handle, enable)
+
+    def profile_read(self):
+        p = statekv_profile_read(self.handle)
+        return [(int(p.launches[i]), float(p.milliseconds[i])) for i in range(3)]
+
+    def sync(self) -> int:
+        return statekv_sync(self.handle)
