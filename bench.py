@@ -1,0 +1,461 @@
+"""Benchmark of the StateKV per-frame video-prefill step on GB300.
+
+A step is one frame of the workload: every layer (and stream) runs the whole
+hot path -- frame attention with fused importance, top-B state selection and
+gather, decode-cache append -- through ``statekv_prefill_frame``.  Before the
+timed steps the state is filled (the frames whose pool still fits in B run
+untimed), so the timed frames are the steady state: "given the preceding
+cache, process one more frame" (App. B's protocol).
+
+Prints one JSON line.  ``--impl reference`` times the CPU oracle instead (the
+paper ships no implementation; the oracle is the reference arm).
+"""
+from __future__ import annotations
+
+import argparse
+import dataclasses
+import hashlib
+import json
+import math
+import os
+import re
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+DEFAULT_WORKLOAD = "qwen7b_stack"
+METRIC = "frames/s and p50 per-frame \u00b5s at 7B shape; % of BF16 tensor peak"
+WORKLOAD_TEXT = {
+    "qwen7b_stack": "28-layer Qwen2-7B-shaped stack: 28 q / 4 kv heads, head_dim 128, bf16, "
+                    "196 tokens/frame, state capacity 2048, 256-frame video",
+    "qwen7b_layer": "one Qwen2-7B-shaped attention layer: 28 q / 4 kv heads, head_dim 128, bf16, "
+                    "196 tokens/frame, state capacity 1568, 64-frame video",
+    "qwen72b_stack": "80-layer 72B-shaped stack: 64 q / 8 kv heads, head_dim 128, bf16, "
+                     "196 tokens/frame, state capacity 4096, 512-frame video",
+    "qwen7b_8streams": "8 concurrent 7B-shaped streams x 28 layers, 28 q / 4 kv heads, head_dim 128, "
+                       "bf16, 196 tokens/frame, state capacity 2048, 1024 frames each",
+    "toy": "toy layer: 4 q / 1 kv heads, head_dim 64, 16 tokens/frame, state capacity 32",
+}
+KERNEL_SOURCE = os.path.join(ROOT, "paper_2605_31598_gb300", "csrc", "attn_kernel.cu")
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "frame_attn_qwen7b_stack.md")
+
+
+def log(*a):
+    print(*a, file=sys.stderr, flush=True)
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            p = json.load(f)
+        return p["hbm_gbs"], p["bf16_tflops"], p.get("bf16_tflops_sustained"), "measured"
+    return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+def attn_flops(shape, count):
+    """Algorithmic FLOPs of the frame attention for one (stream, layer):
+    QK^T and PV over the visible pairs, 4 d Hq (T count + T (T + 1) / 2).
+    The QK^T recompute of the two-pass design is not counted."""
+    T, d, Hq = shape.tokens_per_frame, shape.head_dim, shape.num_q_heads
+    return 4.0 * d * Hq * (T * count + T * (T + 1) / 2)
+
+
+def kernel_source_hash():
+    with open(KERNEL_SOURCE, "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+def recorded_traffic():
+    """DRAM bytes per attention launch from the committed ncu summary, or None
+    if the summary is missing or was taken on a different kernel source."""
+    if not os.path.exists(TRAFFIC_FILE):
+        return None
+    txt = open(TRAFFIC_FILE).read()
+    m = re.search(r"dram_bytes_per_full_launch:\s*([0-9.eE+]+)", txt)
+    h = re.search(r"kernel_source_sha256_16:\s*([0-9a-f]+)", txt)
+    if not m or not h or h.group(1) != kernel_source_hash():
+        return None
+    return float(m.group(1))
+
+
+class ClockSampler:
+    """nvidia-smi clocks / throttle reasons sampled in the background."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id: str):
+        self.samples = []
+        self.proc = None
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", gpu_id, f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "50"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.samples.append((time.time(), [x.strip() for x in line.split(",")]))
+
+    def stop(self):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self, t0, t1):
+        if not self.samples:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no nvidia-smi samples"],
+                    "samples": 0}
+        win = [s for (t, s) in self.samples if t0 - 0.3 <= t <= t1 + 0.3]
+        if not win:  # timed region shorter than the sampling period: nearest samples
+            mid = 0.5 * (t0 + t1)
+            win = [min(self.samples, key=lambda x: abs(x[0] - mid))[1]]
+        sm = [float(s[0]) for s in win if s[0].replace(".", "").isdigit()]
+        mx = [float(s[1]) for s in win if s[1].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for s in win for i in range(4)
+                          if len(s) > 4 + i and s[4 + i].lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons,
+                "samples": len(win),
+                "power_w_max": max((float(s[2]) for s in win
+                                    if s[2].replace(".", "").isdigit()), default=None)}
+
+
+def dist_setup():
+    import torch
+    import torch.distributed as dist
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if backend == "nccl":
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend)
+    return world, rank, local
+
+
+def max_over_ranks(x: float, world: int, device) -> float:
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.barrier()
+
+
+# ---------------------------------------------------------------- oracle legs
+def oracle_units_timing(shape, n_units, seed=0, q_heads=None):
+    """Times the CPU oracle on ``n_units`` (layer, KV head) units of one
+    steady-state frame (state full with B entries).  Each unit is the oracle
+    called on one KV head's query group; ``q_heads`` < G restricts the group.
+    Returns (seconds, fraction of a whole frame step processed)."""
+    import numpy as np
+    import torch
+
+    import oracle
+    from paper_2605_31598_gb300.inputs import frame_qkv
+
+    T, Hq, Hkv, d, B, L = (shape.tokens_per_frame, shape.num_q_heads, shape.num_kv_heads,
+                           shape.head_dim, shape.state_capacity, shape.num_layers)
+    G = Hq // Hkv
+    g = G if q_heads is None else q_heads
+    n_frame = math.ceil(B / T) + 1 if B > 0 else 1
+    total = 0.0
+    for i in range(n_units):
+        layer, h = (i // Hkv) % L, i % Hkv
+        q, k, v = frame_qkv(shape, n_frame, layer=layer, seed=seed)
+        qb = np.ascontiguousarray(oracle.as_bf16_bits(q)[:, h * G: h * G + g])
+        kb = np.ascontiguousarray(oracle.as_bf16_bits(k)[:, h: h + 1])
+        vb = np.ascontiguousarray(oracle.as_bf16_bits(v)[:, h: h + 1])
+        lay = oracle.OracleLayer(g, 1, d, T, B, n_frame)
+        gen = torch.Generator().manual_seed(seed + i)
+        sk = oracle.as_bf16_bits((torch.randn((1, B, d), generator=gen) * d ** -0.5).bfloat16())
+        sv = oracle.as_bf16_bits((torch.randn((1, B, d), generator=gen) * d ** -0.5).bfloat16())
+        lay.set_state(np.array([B], np.int32), np.arange(B, dtype=np.int64)[None], sk, sv,
+                      (n_frame - 1) * T)
+        t0 = time.perf_counter()
+        lay.prefill_frame(qb, kb, vb)
+        total += time.perf_counter() - t0
+    frac = n_units * g / float(L * Hkv * G)
+    return total, frac
+
+
+def run_reference(args, world, rank):
+    """The reference arm: the CPU oracle, timed on the host cores."""
+    if rank != 0:
+        return
+    import oracle
+    from paper_2605_31598_gb300.inputs import WORKLOADS
+
+    oracle.build()
+    shape = WORKLOADS[args.workload]
+    G = shape.num_q_heads // shape.num_kv_heads
+    # size each step so the whole run stays within about two minutes
+    t_one, _ = oracle_units_timing(shape, 1, q_heads=1)
+    budget = 120.0 / max(1, args.steps + args.warmup)
+    g = max(1, min(G, int(budget / max(t_one, 1e-6))))
+    for _ in range(args.warmup):
+        oracle_units_timing(shape, 1, q_heads=g)
+    secs, frac = 0.0, 0.0
+    for _ in range(args.steps):
+        s, f = oracle_units_timing(shape, 1, q_heads=g)
+        secs += s
+        frac += f
+    value = shape.num_streams * frac / secs
+    sample = (f"each step: the oracle on {g} of the {G} query heads of one (layer, KV head) unit "
+              f"of a steady-state frame (state full, B={shape.state_capacity}); "
+              f"frames/s = fraction of a frame processed / time")
+    line = {
+        "impl": "reference", "metric": METRIC,
+        "value": value, "unit": "frames/s", "n_gpus": args.gpus, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": 1e3 * secs / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": {"workload": WORKLOAD_TEXT[args.workload]},
+        "cpu_baseline": {"value": value, "unit": "frames/s", "cores": 1, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": "frames/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# ---------------------------------------------------------------- our arm
+def run_ours(args, world, rank, local):
+    import torch
+
+    from paper_2605_31598_gb300 import StateKV, make_config
+    from paper_2605_31598_gb300.inputs import WORKLOADS, batch_qkv
+
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py needs a CUDA device (no CPU fallback exists)")
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    base = WORKLOADS[args.workload]
+    T, B = base.tokens_per_frame, base.state_capacity
+    S, L, Hkv = base.num_streams, base.num_layers, base.num_kv_heads
+    fill = math.ceil(B / T) if B > 0 else 0  # frames until the state holds B tokens
+    nframes = fill + args.warmup + args.steps
+    max_frames = args.max_frames or base.max_frames
+    if max_frames < nframes:
+        max_frames = nframes
+    shape = dataclasses.replace(base, max_frames=max_frames)
+    seed = args.seed + 1000 * rank
+    log(f"[bench] rank {rank}: generating {nframes} frames of {args.workload} inputs")
+    frames = [batch_qkv(shape, n, streams=range(S), layers=range(L), seed=seed, device=device)
+              for n in range(1, nframes + 1)]
+    eng = StateKV(make_config(shape))
+    out = torch.empty_like(frames[0][0])
+    imp = torch.empty((S, L, Hkv, B + T), dtype=torch.float32, device=device)
+
+    def step(n):
+        q, k, v = frames[n]
+        rc = eng.prefill_frame(q, k, v, out, imp)
+        if rc != 0:
+            raise RuntimeError(f"statekv_prefill_frame returned {rc}")
+
+    eng.profile(True)  # creates the event pool outside the timed region
+    for n in range(fill + args.warmup):
+        step(n)
+    torch.cuda.synchronize()
+
+    props = torch.cuda.get_device_properties(device)
+    gpu_id = f"GPU-{props.uuid}" if getattr(props, "uuid", None) else str(local)
+    sampler = ClockSampler(gpu_id)
+    time.sleep(0.3)
+    st = torch.cuda.current_stream()
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    barrier(world)
+    torch.cuda.synchronize()
+    eng.profile(True)
+    t_wall0 = time.time()
+    for i in range(args.steps):
+        starts[i].record(st)
+        step(fill + args.warmup + i)
+        ends[i].record(st)
+    torch.cuda.synchronize()
+    t_wall1 = time.time()
+    barrier(world)
+    prof = eng.profile_read()
+    eng.profile(False)
+    time.sleep(0.3)
+    sampler.stop()
+    per_step = [s.elapsed_time(e) for s, e in zip(starts, ends)]
+    total_ms = starts[0].elapsed_time(ends[-1])
+    total_ms_max = max_over_ranks(total_ms, world, device)
+    assert eng.sync() == 0
+
+    hbm, tf_burst, tf_sust, peak_kind = peaks()
+    # dominant kernel: frame attention + importance (kind 1)
+    k1_launches, k1_ms = prof[1]
+    k1_avg_s = k1_ms / max(k1_launches, 1) * 1e-3
+    flops = S * L * attn_flops(shape, B)
+    achieved = flops / k1_avg_s / 1e12
+    traffic = recorded_traffic()
+    a_launches, a_ms = prof[0]
+    s_launches, s_ms = prof[2]
+    d = shape.head_dim
+    append_bytes = 2 * 2 * S * L * Hkv * T * d * 2  # read + write K and V rows
+    kernels = {
+        "frame_attn_lse_importance": {"avg_us": 1e6 * k1_avg_s, "tflops": achieved,
+                                      "share": k1_ms / max(1e-9, k1_ms + a_ms + s_ms)},
+        "decode_cache_append": {"avg_us": 1e3 * a_ms / max(a_launches, 1),
+                                "gbs": append_bytes / (a_ms / max(a_launches, 1) * 1e-3) / 1e9,
+                                "bytes": append_bytes,
+                                "share": a_ms / max(1e-9, k1_ms + a_ms + s_ms)},
+        "state_select_gather": {"avg_us": 1e3 * s_ms / max(s_launches, 1),
+                                "share": s_ms / max(1e-9, k1_ms + a_ms + s_ms)},
+    }
+    value = world * S * args.steps / (total_ms_max * 1e-3)
+    ps = sorted(per_step)
+    line = {
+        "metric": METRIC,
+        "value": value,
+        "unit": "frames/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": total_ms_max / args.steps,
+        "p50_us_per_frame": 1e3 * ps[len(ps) // 2],
+        "p90_us_per_frame": 1e3 * ps[min(len(ps) - 1, int(0.9 * len(ps)))],
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic",
+        "config": {"workload": WORKLOAD_TEXT[args.workload], "streams": S, "layers": L,
+                   "steady_state_frames": f"{fill + args.warmup + 1}..{nframes}",
+                   "l2": "no flush: each step reads fresh Q/K/V and the full state "
+                         f"(~{(2 * S * L * Hkv * B * d * 2 + S * L * T * (shape.num_q_heads + 2 * Hkv) * d * 2) / 1e6:.0f} MB "
+                         "per step) > 129 MB L2",
+                   "parallelism": f"replicas{world}" if world > 1 else "single"},
+        "roofline": {"bound": "tensor", "achieved": achieved,
+                     "peak": tf_burst, "unit": "TFLOP/s", "frac": achieved / tf_burst,
+                     "peak_kind": f"{peak_kind} bf16 dense burst",
+                     "frac_of_sustained": (achieved / tf_sust) if tf_sust else None,
+                     "traffic": traffic,
+                     "kernel": "frame_attn_lse_importance",
+                     "flops_per_launch": flops},
+        "kernels": kernels,
+        "gpu_launches": 3 * args.steps,
+    }
+    clocks = sampler.summary(t_wall0, t_wall1)
+    line["clocks"] = clocks
+
+    # end to end through the host-buffer entry point (copies inside the timed region)
+    if not args.no_e2e:
+        line["e2e"] = run_e2e(args, shape, fill, seed, device, frames)
+    del frames
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import oracle
+
+        oracle.build()
+        n_units = 16
+        secs, frac = oracle_units_timing(shape, n_units, seed=seed)
+        line["cpu_baseline"] = {
+            "value": S * frac / secs, "unit": "frames/s", "cores": 1, "kind": "oracle",
+            "sample": f"{n_units} (layer, KV head) units of one steady-state frame "
+                      f"({frac:.3f} of a frame, {secs:.1f} s single-threaded fp64), "
+                      "scaled to frames/s"}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+
+
+def run_e2e(args, shape, fill, seed, device, frames):
+    """Same step through statekv_prefill_frame_host: every step copies that
+    frame's Q/K/V from pinned host memory and reads the output (and
+    importance) back, inside the timed region."""
+    import torch
+
+    from paper_2605_31598_gb300 import StateKV, make_config
+
+    S, L, Hkv, T, B = (shape.num_streams, shape.num_layers, shape.num_kv_heads,
+                       shape.tokens_per_frame, shape.state_capacity)
+    steps = min(args.steps, 64)
+    n_total = fill + args.warmup + steps
+    host = [tuple(x.cpu().pin_memory() for x in frames[n]) for n in range(n_total)]
+    out_h = torch.empty(host[0][0].shape, dtype=torch.bfloat16).pin_memory()
+    imp_h = torch.empty((S, L, Hkv, B + T), dtype=torch.float32).pin_memory()
+    eng = StateKV(make_config(shape, host_staging=True))
+
+    def step(n):
+        q, k, v = host[n]
+        rc = eng.prefill_frame_host(q, k, v, out_h, imp_h)
+        if rc != 0:
+            raise RuntimeError(f"statekv_prefill_frame_host returned {rc}")
+
+    for n in range(fill + args.warmup):
+        step(n)
+    torch.cuda.synchronize()
+    st = torch.cuda.current_stream()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(st)
+    for i in range(steps):
+        step(fill + args.warmup + i)
+    e1.record(st)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1)
+    assert eng.sync() == 0
+    h2d = sum(x.numel() * x.element_size() for x in host[0])
+    d2h = out_h.numel() * 2 + imp_h.numel() * 4
+    eng.close()
+    return {"value": S * steps / (ms * 1e-3), "unit": "frames/s", "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h, "steps": steps,
+            "api": "statekv_prefill_frame_host (pinned host buffers)"}
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(WORKLOAD_TEXT))
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--max-frames", type=int, default=0,
+                    help="decode-cache capacity in frames (default: the workload's); "
+                         "a small value keeps the arena small for profiler captures")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        raise SystemExit("--warmup must be at least 3")
+    world, rank, local = dist_setup()
+    if args.impl == "reference":
+        run_reference(args, world, rank)
+    else:
+        run_ours(args, world, rank, local)
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()
