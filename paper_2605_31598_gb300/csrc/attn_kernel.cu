@@ -7,26 +7,30 @@
 //
 // Keys are the valid state slots (tiles of 128 from the compressed state)
 // followed by the frame's tokens.  Two passes over the key tiles (App. B.1):
-//   pass A  S = Q K^T          (M = queries)  -> online max / sum -> LSE per row
-//   pass B  S^T = K Q^T        (M = keys)     -> P = exp(S - LSE) in fp32;
-//           thread = key, so the column sum over the tile's queries (Eq. 1's
-//           importance, restricted to these rows) is a register sum;
-//           O += P V           (P bf16, MN-major from shared memory)
-// Both contractions run on tcgen05 with fp32 accumulators in TMEM.  K and V
-// tiles arrive by TMA (128-byte swizzle) in four 32 KB shared-memory slots:
-// pass A streams K through all four; pass B streams K through slots 0-1 and
-// V through slots 2-3, loaded by two independent producer threads so a V
-// slot that is still waiting for its P.V never holds back the next K load.
+//   pass A  S = Q K^T  -> online max / sum per row -> log-sum-exp
+//   pass B  S = Q K^T  -> P = exp(S - LSE) (fp32) -> column sums of P over the
+//           tile's 128 rows (Eq. 1's importance, restricted to these rows) and
+//           O += P V with P in bf16.
+// tcgen05 runs every contraction with the A operand in TMEM (Q for Q K^T, P
+// for P V), so each MMA streams only K or V from shared memory.  TMEM
+// (512 columns): Q | score/P buffer of softmax warpgroup 0 | of warpgroup 1 |
+// O.  K and V tiles arrive by TMA (128-byte swizzle) in six 32 KB slots:
+// pass A streams K through all six; pass B streams K through slots 0-2 and V
+// through 3-5, each ring fed by its own producer thread.
 //
 // 384 threads, three warpgroups:
-//   WG0  warp 0 K producer, warp 1 TMEM owner + MMA issuer, warp 2 V
-//        producer (warp 3 idle)
-//   WG1, WG2  softmax / importance warpgroups; they take alternate key tiles,
-//        so while one works on tile j the other works on j+1 and the tensor
-//        core computes j+2 (three TMEM score buffers + the O accumulator fill
-//        the 512 TMEM columns).
-// The per-element work uses packed f32x2 FMA/ADD, three-input max and
-// independent accumulators so no dependency chain runs the length of a tile.
+//   WG0  warp 0 K producer, warp 2 V producer, warps 1 and 3 MMA issuers
+//        (warp 1 also owns TMEM).  A tcgen05.mma issues at the tensor core's
+//        pace, so every barrier wait of an issuing thread idles the tensor
+//        core; with two issuers one waits while the other's MMAs run.  Issuer
+//        X (warp 1) issues the pass-A Q K^T of even tiles and every pass-B
+//        Q K^T; issuer Y (warp 3) the pass-A Q K^T of odd tiles and every P V
+//        (in order, so O accumulates deterministically).
+//   WG1, WG2  softmax warpgroups: thread = query row; they take alternate key
+//        tiles, each with its own TMEM score buffer, so the tensor core works
+//        on one warpgroup's tile while the other computes exponentials.
+// The column sums over a warp's 32 rows are a shuffle reduce-scatter (each
+// lane ends with one column); the four warps add through shared memory.
 // Every mbarrier wait is bounded by the watchdog; on expiry the CTA records
 // DEV_TIMEOUT_ATTN, drains its in-flight copies and MMAs, frees TMEM and exits.
 #include "sm103_ptx.cuh"
@@ -38,26 +42,26 @@ namespace {
 using namespace ptx;
 
 constexpr int kThreads = 384;
-constexpr int kSBuf = 3;  // TMEM score buffers
+constexpr int kSlots = 6;        // 32 KB K/V tile slots (D = 128)
+constexpr int kKSlotsB = 3;      // pass B: K slots 0..2, V slots 3..5
+constexpr uint32_t kColS0 = 128; // TMEM columns: Q [0, D/2), S0, S1, O
+constexpr uint32_t kColS1 = 256;
+constexpr uint32_t kColO = 384;
 
 template <int D>
 struct AttnLayout {
-    static constexpr int kQBytes = kBM * D * 2;
     static constexpr int kTileBytes = kBN * D * 2;  // one K or V tile
-    static constexpr int kPBytes = kBM * kBN * 2;
-    static constexpr int kOffQ = 0;
-    static constexpr int kOffSlots = kOffQ + kQBytes;          // 4 K/V tile slots
-    static constexpr int kOffP = kOffSlots + 4 * kTileBytes;
-    static constexpr int kOffNLse = kOffP + 2 * kPBytes;   // float[128]: -LSE*log2e per row
-    static constexpr int kOffTq = kOffNLse + kBM * 4;      // int[128]: token of each row
-    static constexpr int kOffBar = kOffTq + kBM * 4;
-    // slot_full[4] slot_empty[4] s_full[3] s_empty[3] p_full[2] p_empty[2]
+    static constexpr int kOffSlots = 0;
+    static constexpr int kOffRed = kOffSlots + kSlots * kTileBytes;  // float[2 wg][2][4][128]
+    static constexpr int kOffStat = kOffRed + 2 * 2 * 4 * kBM * 4;   // float[2][2][128]
+    static constexpr int kOffBar = kOffStat + 4 * kBM * 4;
+    // slot_full[6] slot_empty[6] s_full[2] s_read[2] p_full[2] pv_done[2]
     // q_full o_full drain a_done
-    static constexpr int kNumBars = 22;
+    static constexpr int kNumBars = 24;
     static constexpr int kOffMisc = kOffBar + kNumBars * 8;
     static constexpr int kBytes = kOffMisc + 16;
     static constexpr int kAlloc = kBytes + 1024;  // room to align the base to 1 KB
-    static_assert(kOffSlots % 1024 == 0 && kOffP % 1024 == 0, "align");
+    static_assert(kOffSlots % 1024 == 0 && kTileBytes % 1024 == 0, "align");
     static_assert(kAlloc <= 232448, "shared memory budget");
 };
 
@@ -130,6 +134,35 @@ __device__ __forceinline__ void named_bar_sync(int id, int nthreads)
     asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
 }
 
+// D[tmem] (+)= A[tmem] * B[smem], bf16 inputs, fp32 accumulator.
+__device__ __forceinline__ void umma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc,
+                                        uint32_t idesc, uint32_t accumulate)
+{
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
+// 16 consecutive 32-bit TMEM columns of this thread's lane <- registers.
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16])
+{
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0],"
+        " {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16};" ::"r"(taddr),
+        "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+        "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),
+        "r"(r[15])
+        : "memory");
+}
+
+__device__ __forceinline__ void tmem_st_wait()
+{
+    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
 // K-major SW128 operand with `rows` rows: k-step ks (16 elements) of the tile.
 __device__ __forceinline__ uint64_t kmajor_desc(uint32_t base, int ks, int rows)
 {
@@ -143,32 +176,29 @@ __device__ __forceinline__ uint64_t mnmajor_desc(uint32_t base, int ks, uint32_t
     return sdesc_sw128(base + ks * 2048, block_bytes, 1024);
 }
 
-__device__ __forceinline__ float4 lds_f4(const void* p)
-{
-    // volatile: re-read per tile instead of being hoisted out of the tile
-    // loop (keeping 128 per-column values live would exhaust registers)
-    float4 v;
-    asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];"
-                 : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
-                 : "r"(smem_addr(p)));
-    return v;
-}
-
-__device__ __forceinline__ int4 lds_i4(const void* p)
-{
-    int4 v;
-    asm volatile("ld.shared.v4.s32 {%0, %1, %2, %3}, [%4];"
-                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
-                 : "r"(smem_addr(p)));
-    return v;
-}
-
-// Pass A tile `it` occupies slot it % 4; pass B K tile j occupies slot j % 2
-// and V tile j slot 2 + j % 2.  The use count of a slot before pass B is the
-// number of pass-A tiles it held.
+// Pass A tile `it` occupies slot it % 6; pass B K tile j slot j % 3 and V
+// tile j slot 3 + j % 3.  The use count of a slot before pass B is the number
+// of pass-A tiles it held.
 __device__ __forceinline__ int pass_a_uses(int nt, int slot)
 {
-    return nt > slot ? (nt - slot + 3) / 4 : 0;
+    return nt > slot ? (nt - slot + kSlots - 1) / kSlots : 0;
+}
+
+// Column sums over the warp's 32 rows of a 32-column chunk held one row per
+// lane: a butterfly reduce-scatter; lane l returns the sum of column l.
+__device__ __forceinline__ float warp_colsum32(float (&x)[32], int lane)
+{
+#pragma unroll
+    for (int m = 16, n = 32; m >= 1; m >>= 1, n >>= 1) {
+        const bool up = (lane & m) != 0;
+#pragma unroll
+        for (int i = 0; i < n / 2; ++i) {
+            const float send = up ? x[i] : x[i + n / 2];
+            const float keep = up ? x[i + n / 2] : x[i];
+            x[i] = keep + __shfl_xor_sync(0xffffffffu, send, m);
+        }
+    }
+    return x[0];
 }
 
 template <int D>
@@ -182,25 +212,20 @@ __global__ void __launch_bounds__(kThreads, 1)
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-    uint8_t* sQ = sm + L::kOffQ;
     uint8_t* sSlot = sm + L::kOffSlots;
-    uint8_t* sP = sm + L::kOffP;
-    float* nlse2 = reinterpret_cast<float*>(sm + L::kOffNLse);
-    int* tq = reinterpret_cast<int*>(sm + L::kOffTq);
-    // (m, l) of both softmax warpgroups at the end of pass A: float[2][2][128].
-    // It borrows the P buffers, which are first written after the merge.
-    float* stat = reinterpret_cast<float*>(sm + L::kOffP);
+    float* red = reinterpret_cast<float*>(sm + L::kOffRed);
+    float* stat = reinterpret_cast<float*>(sm + L::kOffStat);
     uint64_t* bars = reinterpret_cast<uint64_t*>(sm + L::kOffBar);
     uint64_t* slot_full = bars + 0;
-    uint64_t* slot_empty = bars + 4;
-    uint64_t* s_full = bars + 8;
-    uint64_t* s_empty = bars + 11;
-    uint64_t* p_full = bars + 14;
-    uint64_t* p_empty = bars + 16;
-    uint64_t* q_full = bars + 18;
-    uint64_t* o_full = bars + 19;
-    uint64_t* drain = bars + 20;
-    uint64_t* a_done = bars + 21;  // every pass-A MMA has completed
+    uint64_t* slot_empty = bars + 6;
+    uint64_t* s_full = bars + 12;   // QK^T result in score buffer w
+    uint64_t* s_read = bars + 14;   // pass A: warpgroup w has read score buffer w
+    uint64_t* p_full = bars + 16;   // pass B: warpgroup w has written P into buffer w
+    uint64_t* pv_done = bars + 18;  // pass B: the P V that read buffer w has completed
+    uint64_t* q_full = bars + 20;
+    uint64_t* o_full = bars + 21;
+    uint64_t* drain = bars + 22;
+    uint64_t* a_done = bars + 23;   // every pass-A MMA has completed
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + L::kOffMisc);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(sm + L::kOffMisc + 4);
 
@@ -220,22 +245,20 @@ __global__ void __launch_bounds__(kThreads, 1)
     const unsigned long long deadline = globaltimer() + p.watchdog_ns;
 
     if (threadIdx.x == 0) {
-        for (int i = 0; i < 4; ++i) {
+        for (int i = 0; i < kSlots; ++i) {
             mbar_init(&slot_full[i], 1);
             mbar_init(&slot_empty[i], 1);
         }
         for (int i = 0; i < 2; ++i) {
-            mbar_init(&p_full[i], 128);
-            mbar_init(&p_empty[i], 1);
-        }
-        for (int i = 0; i < kSBuf; ++i) {
             mbar_init(&s_full[i], 1);
-            mbar_init(&s_empty[i], 128);
+            mbar_init(&s_read[i], 128);
+            mbar_init(&p_full[i], 128);
+            mbar_init(&pv_done[i], 1);
         }
         mbar_init(q_full, 256);
         mbar_init(o_full, 1);
-        mbar_init(drain, 1);
-        mbar_init(a_done, 1);
+        mbar_init(drain, 2);   // one commit per MMA issuer
+        mbar_init(a_done, 2);
         *abort_flag = 0;
         fence_mbar_init();
     }
@@ -268,25 +291,24 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 const CUtensorMap* smap = kprod ? &tm_sk : &tm_sv;
                 const CUtensorMap* fmap = kprod ? &tm_fk : &tm_fv;
-                int last_use[4] = {-1, -1, -1, -1};
-                // Slots 2-3 also carry pass-A K tiles: the V producer starts only
+                int last_use[kSlots] = {-1, -1, -1, -1, -1, -1};
+                // V slots also carry pass-A K tiles: the V producer starts only
                 // once every pass-A MMA has released them (before that, a wait on
                 // their empty barriers could match an earlier phase of the same
                 // parity).
                 if (!kprod && !wait_until(a_done, 0, deadline)) fail();
-                // loads: pass A (K producer only) then pass B
                 const int nload = kprod ? 2 * nt : nt;
                 for (int n = 0; n < nload; ++n) {
                     if (*abort_flag) break;
                     int slot, use, tile;
                     if (kprod && n < nt) {
                         tile = n;
-                        slot = n & 3;
-                        use = n >> 2;
+                        slot = n % kSlots;
+                        use = n / kSlots;
                     } else {
                         tile = kprod ? n - nt : n;
-                        slot = (kprod ? 0 : 2) + (tile & 1);
-                        use = pass_a_uses(nt, slot) + (tile >> 1);
+                        slot = (kprod ? 0 : kKSlotsB) + tile % kKSlotsB;
+                        use = pass_a_uses(nt, slot) + tile / kKSlotsB;
                     }
                     if (use >= 1 && !wait_until(&slot_empty[slot], (use - 1) & 1, deadline)) {
                         fail();
@@ -308,68 +330,75 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (*abort_flag) {
                     // Let copies already in flight land before the CTA's memory goes away.
                     const unsigned long long dl = globaltimer() + p.watchdog_ns;
-                    for (int sl = 0; sl < 4; ++sl)
+                    for (int sl = 0; sl < kSlots; ++sl)
                         if (last_use[sl] >= 0) wait_until(&slot_full[sl], last_use[sl] & 1, dl);
                 }
             }
             __syncwarp();
-        } else if (warp == 1) {
-            // ------------------------------------------------------------ MMA issuer
+        } else {
+            // ------------------------------------------------------------ MMA issuers
             if (lane == 0) {
-                const uint32_t aQ = smem_addr(sQ), aSlot = smem_addr(sSlot), aP = smem_addr(sP);
-                const uint32_t tO = tbase + kSBuf * 128;
+                const bool isx = warp == 1;
+                const uint32_t aSlot = smem_addr(sSlot);
+                const uint32_t tQ = tbase, tO = tbase + kColO;
                 constexpr uint32_t kIdQK = idesc_bf16_f32(kBM, kBN, false, false);
-                constexpr uint32_t kIdKQ = idesc_bf16_f32(kBN, kBM, false, false);
-                constexpr uint32_t kIdPV = idesc_bf16_f32(kBM, D, true, true);
+                constexpr uint32_t kIdPV = idesc_bf16_f32(kBM, D, false, true);
                 bool ok = wait_until(q_full, 0, deadline);
-                // score MMA of sequence index it (pass A: it < nt; pass B: nt + j)
-                auto issue_s = [&](int it, bool transposed) -> bool {
-                    const int b = it % kSBuf;
+                // QK^T of global sequence index it (pass A: it < nt; pass B: nt + j)
+                // into score buffer it & 1.
+                auto issue_qk = [&](int it) -> bool {
+                    const int w = it & 1;
+                    const bool pass_b = it >= nt;
                     const int j = it - nt;
-                    const int slot = transposed ? (j & 1) : (it & 3);
-                    const int use = transposed ? pass_a_uses(nt, slot) + (j >> 1) : (it >> 2);
+                    const int slot = pass_b ? j % kKSlotsB : it % kSlots;
+                    const int use = pass_b ? pass_a_uses(nt, slot) + j / kKSlotsB : it / kSlots;
                     if (!wait_until(&slot_full[slot], use & 1, deadline)) return false;
-                    if (it >= kSBuf && !wait_until(&s_empty[b], ((it / kSBuf) - 1) & 1, deadline))
-                        return false;
+                    // the buffer's previous tile (it - 2) must be consumed: read by
+                    // its warpgroup in pass A, or read by its P V in pass B
+                    if (it >= 2) {
+                        const int prev = it - 2;
+                        const bool ok2 =
+                            prev < nt
+                                ? wait_until(&s_read[w], (prev >> 1) & 1, deadline)
+                                : wait_until(&pv_done[w], ((prev - nt) >> 1) & 1, deadline);
+                        if (!ok2) return false;
+                    }
                     tc_fence_after();
                     const uint32_t kb = aSlot + slot * L::kTileBytes;
-                    const uint32_t tS = tbase + b * 128;
+                    const uint32_t tS = tbase + (w ? kColS1 : kColS0);
 #pragma unroll
-                    for (int k = 0; k < D / 16; ++k) {
-                        if (transposed)
-                            umma_bf16(tS, kmajor_desc(kb, k, kBN), kmajor_desc(aQ, k, kBM), kIdKQ, k > 0);
-                        else
-                            umma_bf16(tS, kmajor_desc(aQ, k, kBM), kmajor_desc(kb, k, kBN), kIdQK, k > 0);
-                    }
-                    umma_commit(&s_full[b]);
+                    for (int k = 0; k < D / 16; ++k)
+                        umma_ts(tS, tQ + k * 8, kmajor_desc(kb, k, kBN), kIdQK, k > 0);
+                    umma_commit(&s_full[w]);
                     umma_commit(&slot_empty[slot]);
                     return true;
                 };
                 auto issue_pv = [&](int j) -> bool {
-                    const int w = (nt + j) & 1, slot = 2 + (j & 1);
-                    const int use = pass_a_uses(nt, slot) + (j >> 1);
+                    const int w = (nt + j) & 1;
+                    const int slot = kKSlotsB + j % kKSlotsB;
+                    const int use = pass_a_uses(nt, slot) + j / kKSlotsB;
                     if (!wait_until(&p_full[w], (j >> 1) & 1, deadline)) return false;
                     if (!wait_until(&slot_full[slot], use & 1, deadline)) return false;
                     tc_fence_after();
-                    const uint32_t pbase = aP + w * L::kPBytes;
-                    const uint32_t vbase = aSlot + slot * L::kTileBytes;
+                    const uint32_t vb = aSlot + slot * L::kTileBytes;
+                    const uint32_t tP = tbase + (w ? kColS1 : kColS0);
 #pragma unroll
                     for (int k = 0; k < kBN / 16; ++k)
-                        umma_bf16(tO, mnmajor_desc(pbase, k, kBN * 128),
-                                  mnmajor_desc(vbase, k, kBN * 128), kIdPV, (j > 0 || k > 0));
-                    umma_commit(&p_empty[w]);
+                        umma_ts(tO, tP + k * 8, mnmajor_desc(vb, k, kBN * 128), kIdPV,
+                                (j > 0 || k > 0));
+                    umma_commit(&pv_done[w]);
                     umma_commit(&slot_empty[slot]);
                     return true;
                 };
-                for (int it = 0; ok && it < nt; ++it) ok = issue_s(it, false);  // pass A
+                // pass A: X takes even tiles, Y odd tiles
+                for (int it = isx ? 0 : 1; ok && it < nt; it += 2) ok = issue_qk(it);
                 if (ok) umma_commit(a_done);
-                for (int j = 0; ok && j < nt; ++j) {                             // pass B
-                    ok = issue_s(nt + j, true);
-                    if (ok && j >= 2) ok = issue_pv(j - 2);
+                if (isx) {  // pass B Q K^T, in tile order
+                    for (int j = 0; ok && j < nt; ++j) ok = issue_qk(nt + j);
+                } else {    // pass B P V, in tile order
+                    for (int j = 0; ok && j < nt; ++j) ok = issue_pv(j);
+                    if (ok) umma_commit(o_full);
                 }
-                if (ok && nt >= 2) ok = issue_pv(nt - 2);
-                if (ok) ok = issue_pv(nt - 1);
-                if (ok) umma_commit(o_full);
                 if (!ok) fail();
                 // Every MMA issued so far must finish before TMEM is released.
                 umma_commit(drain);
@@ -384,43 +413,49 @@ __global__ void __launch_bounds__(kThreads, 1)
         asm volatile("setmaxnreg.inc.sync.aligned.u32 208;" ::: "memory");
         // ------------------------------------------------------------ softmax warpgroups
         const int wg = (warp >> 2) - 1;          // 0 or 1
-        const int ct = threadIdx.x - 128;        // 0..255 across both warpgroups
         const int quad = warp & 3;               // TMEM lane quadrant of this warp
-        const int row = quad * 32 + lane;        // TMEM lane = tile row
-        const uint32_t tlane = tbase + (static_cast<uint32_t>(quad * 32) << 16);
+        const int row = quad * 32 + lane;        // TMEM lane = query row of the tile
+        const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
+        const uint32_t tS = tbase + lane_off + (wg ? kColS1 : kColS0);
         const float c = p.scale_log2;
+        const int my_r = mt * kBM + row;
+        const bool row_valid = my_r < rows;
+        const int my_tq = row_valid ? my_r / G : T;  // padding rows see every frame key
 
-        for (int i = ct; i < kBM; i += 256) {
-            const int r = mt * kBM + i;
-            tq[i] = r < rows ? r / G : -1;
-        }
-        {   // Q tile -> K-major SW128 shared memory, zero rows past the group
-            constexpr int kChunks = D / 8;  // 16-byte chunks per row
-            const __nv_bfloat16* qu = p.q + static_cast<size_t>(u) * T * p.Hq * D;
-            for (int idx = ct; idx < kBM * kChunks; idx += 256) {
-                const int ri = idx / kChunks, ch = idx % kChunks;
-                const int r = mt * kBM + ri;
-                uint4 val = make_uint4(0, 0, 0, 0);
-                if (r < rows) {
-                    const int t = r / G, g = r - t * G;
-                    val = *reinterpret_cast<const uint4*>(
-                        qu + (static_cast<size_t>(t) * p.Hq + hkv * G + g) * D + ch * 8);
+        {   // Q row -> TMEM columns [0, D/2) (bf16 pairs); warpgroup wg stores
+            // d in [64 wg, 64 wg + 64) when D = 128, warpgroup 0 all of D = 64.
+            if (wg * 64 < D) {
+                uint32_t w32[32];
+                if (row_valid) {
+                    const int t = my_r / G, g = my_r - t * G;
+                    const uint4* src = reinterpret_cast<const uint4*>(
+                        p.q + ((static_cast<size_t>(u) * T + t) * p.Hq + hkv * G + g) * D + wg * 64);
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) {
+                        const uint4 x = src[i];
+                        w32[4 * i] = x.x;
+                        w32[4 * i + 1] = x.y;
+                        w32[4 * i + 2] = x.z;
+                        w32[4 * i + 3] = x.w;
+                    }
+                } else {
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) w32[i] = 0u;
                 }
-                *reinterpret_cast<uint4*>(sQ + (ch >> 3) * (kBM * 128) + sw128_offset(ri, ch & 7)) =
-                    val;
+                tmem_st16(tbase + lane_off + wg * 32, *reinterpret_cast<uint32_t(*)[16]>(&w32[0]));
+                tmem_st16(tbase + lane_off + wg * 32 + 16,
+                          *reinterpret_cast<uint32_t(*)[16]>(&w32[16]));
+                tmem_st_wait();
             }
+            tc_fence_before();
+            mbar_arrive(q_full);
         }
-        fence_proxy_async_smem();
-        mbar_arrive(q_full);
 
         bool ok = true;
-        // ---------------- pass A: thread = query row; online max / sum of exp2
-        const int my_r = mt * kBM + row;
-        const int my_tq = my_r < rows ? my_r / G : T;  // padding rows see every frame key
-        float m = -INFINITY, l = 0.f;                   // in log2 units, scaled
+        // ---------------- pass A: online max / sum of exp2 over this warpgroup's tiles
+        float m = -INFINITY, l = 0.f;  // log2 units, scaled
         for (int it = wg; it < nt; it += 2) {
-            const int b = it % kSBuf;
-            ok = __all_sync(0xffffffffu, wait_until(&s_full[b], (it / kSBuf) & 1, deadline));
+            ok = __all_sync(0xffffffffu, wait_until(&s_full[wg], (it >> 1) & 1, deadline));
             if (!ok) break;
             tc_fence_after();
             int lim;  // keys [0, lim) of this tile are visible to this row
@@ -430,158 +465,142 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const int f0 = (it - nst) * kBN;
                 lim = min(kBN, (p.causal ? min(T, my_tq + 1) : T) - f0);
             }
-            // four 32-column chunks; the next chunk's TMEM load overlaps this
-            // chunk's math (tcgen05.wait::ld waits for every load issued so far)
-            float v[2][32];
-            tmem_ld32(tlane + b * 128, v[0]);
+            // the whole tile into registers, then release the buffer at once so
+            // the next Q K^T into it can start while this one is reduced
+            float v[4][32];
+#pragma unroll
+            for (int ch = 0; ch < 4; ++ch) tmem_ld32(tS + ch * 32, v[ch]);
             tmem_ld_wait();
-#pragma unroll
-            for (int ch = 0; ch < 4; ++ch) {
-                float (&x)[32] = v[ch & 1];
-                if (ch < 3) tmem_ld32(tlane + b * 128 + (ch + 1) * 32, v[(ch + 1) & 1]);
-                if (lim < kBN) {
-#pragma unroll
-                    for (int j = 0; j < 32; ++j) x[j] = (ch * 32 + j < lim) ? x[j] : -INFINITY;
-                }
-                float mx[4];
-#pragma unroll
-                for (int q4 = 0; q4 < 4; ++q4) mx[q4] = fmaxf(x[q4 * 2], x[q4 * 2 + 1]);
-#pragma unroll
-                for (int j = 8; j < 32; j += 8)
-#pragma unroll
-                    for (int q4 = 0; q4 < 4; ++q4)
-                        mx[q4] = max3(mx[q4], x[j + q4 * 2], x[j + q4 * 2 + 1]);
-                const float m_new =
-                    fmaxf(m, fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])) * c);  // c > 0
-                if (m_new != -INFINITY) {
-                    const f2 cc = pk(c, c), nm = pk(-m_new, -m_new);
-                    f2 acc[4] = {pk(0.f, 0.f), pk(0.f, 0.f), pk(0.f, 0.f), pk(0.f, 0.f)};
-#pragma unroll
-                    for (int j = 0; j < 32; j += 2) {
-                        float x0, x1;
-                        upk(fma2(pk(x[j], x[j + 1]), cc, nm), x0, x1);
-                        acc[(j >> 1) & 3] = add2(acc[(j >> 1) & 3], pk(ex2(x0), ex2(x1)));
-                    }
-                    float s0, s1;
-                    upk(add2(add2(acc[0], acc[1]), add2(acc[2], acc[3])), s0, s1);
-                    l = l * ex2(m - m_new) + (s0 + s1);
-                    m = m_new;
-                }
-                if (ch < 3) tmem_ld_wait();
-            }
             tc_fence_before();
-            mbar_arrive(&s_empty[b]);
+            mbar_arrive(&s_read[wg]);
+            if (lim < kBN) {
+#pragma unroll
+                for (int ch = 0; ch < 4; ++ch)
+#pragma unroll
+                    for (int e = 0; e < 32; ++e)
+                        v[ch][e] = (ch * 32 + e < lim) ? v[ch][e] : -INFINITY;
+            }
+            float mx[4];
+#pragma unroll
+            for (int q4 = 0; q4 < 4; ++q4) mx[q4] = fmaxf(v[q4][0], v[q4][1]);
+#pragma unroll
+            for (int ch = 0; ch < 4; ++ch)
+#pragma unroll
+                for (int e = 2; e < 32; e += 2)
+                    mx[ch] = max3(mx[ch], v[ch][e], v[ch][e + 1]);
+            const float m_new =
+                fmaxf(m, fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])) * c);  // c > 0
+            if (m_new != -INFINITY) {
+                const f2 cc = pk(c, c), nm = pk(-m_new, -m_new);
+                f2 acc[4] = {pk(0.f, 0.f), pk(0.f, 0.f), pk(0.f, 0.f), pk(0.f, 0.f)};
+#pragma unroll
+                for (int ch = 0; ch < 4; ++ch)
+#pragma unroll
+                    for (int e = 0; e < 32; e += 2) {
+                        float x0, x1;
+                        upk(fma2(pk(v[ch][e], v[ch][e + 1]), cc, nm), x0, x1);
+                        acc[(e >> 1) & 3] = add2(acc[(e >> 1) & 3], pk(ex2(x0), ex2(x1)));
+                    }
+                float s0, s1;
+                upk(add2(add2(acc[0], acc[1]), add2(acc[2], acc[3])), s0, s1);
+                l = l * ex2(m - m_new) + (s0 + s1);
+                m = m_new;
+            }
         }
         stat[(wg * 2 + 0) * kBM + row] = m;
         stat[(wg * 2 + 1) * kBM + row] = l;
         named_bar_sync(1, 256);
-        if (wg == 0) {
+        float nlse;  // -log2-sum-exp of this row (scaled); -inf for padding rows
+        {
             const float m0 = stat[0 * kBM + row], l0 = stat[1 * kBM + row];
             const float m1 = stat[2 * kBM + row], l1 = stat[3 * kBM + row];
             const float mm = fmaxf(m0, m1);
             const float ll = l0 * ex2(m0 - mm) + l1 * ex2(m1 - mm);
-            nlse2[row] = (my_r < rows) ? -(mm + __log2f(ll)) : -INFINITY;
+            nlse = row_valid ? -(mm + __log2f(ll)) : -INFINITY;
         }
-        named_bar_sync(1, 256);
 
-        // ---------------- pass B: thread = key; columns = the tile's query rows
+        // ---------------- pass B: P = exp2(S c - lse) -> TMEM (bf16) and column sums
         float* part = p.partials + ((static_cast<size_t>(u) * p.Hkv + hkv) * p.MT + mt) * p.P;
-        const int t_lo = (mt * kBM) / G;  // first query token of the tile
-        uint8_t* Pb = sP + wg * L::kPBytes;
-        for (int j = (wg - nt) & 1; ok && j < nt; j += 2) {
-            const int it = nt + j, b = it % kSBuf;
-            ok = __all_sync(0xffffffffu, wait_until(&s_full[b], (it / kSBuf) & 1, deadline));
-            if (!ok) break;
-            tc_fence_after();
-            float v[2][32];
-            tmem_ld32(tlane + b * 128, v[0]);
+        float* myred = red + wg * (2 * 4 * kBM);
+        const int ct = threadIdx.x - 128 - 128 * wg;  // 0..127 within the warpgroup
+        // Every warp runs every iteration and arrives at the per-tile barrier;
+        // after a timeout it only skips the work (a bar.sync cannot time out).
+        for (int j = (wg - nt) & 1, k2 = 0; j < nt; j += 2, ++k2) {
+            const int it = nt + j;
+            if (ok) ok = __all_sync(0xffffffffu, wait_until(&s_full[wg], (it >> 1) & 1, deadline));
             const bool is_state = j < nst;
-            const int key = is_state ? j * kBN + row : (j - nst) * kBN + row;
-            const bool kvalid = is_state ? key < count : key < T;
-            // the tile needs a per-element causal test unless all of its keys
-            // precede the tile's first query token
-            const bool diag = !is_state && p.causal && ((j - nst) * kBN + kBN - 1 > t_lo);
-            const f2 cc = pk(c, c);
-            f2 acc[4] = {pk(0.f, 0.f), pk(0.f, 0.f), pk(0.f, 0.f), pk(0.f, 0.f)};
-            uint32_t pp[kBM / 2];  // the tile's P row, bf16 pairs
-            tmem_ld_wait();
-#pragma unroll
-            for (int ch = 0; ch < 4; ++ch) {
-                float (&x)[32] = v[ch & 1];
-                if (ch < 3) tmem_ld32(tlane + b * 128 + (ch + 1) * 32, v[(ch + 1) & 1]);
-#pragma unroll
-                for (int g8 = 0; g8 < 4; ++g8) {
-                    const int c8 = ch * 4 + g8;  // columns 8*c8 .. 8*c8+7
-                    const float4 la = lds_f4(&nlse2[c8 * 8]);
-                    const float4 lb = lds_f4(&nlse2[c8 * 8 + 4]);
-                    const f2 nl[4] = {pk(la.x, la.y), pk(la.z, la.w), pk(lb.x, lb.y),
-                                      pk(lb.z, lb.w)};
-                    float pr[8];
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        float x0, x1;
-                        upk(fma2(pk(x[g8 * 8 + 2 * e], x[g8 * 8 + 2 * e + 1]), cc, nl[e]), x0, x1);
-                        pr[2 * e] = ex2(x0);
-                        pr[2 * e + 1] = ex2(x1);
-                    }
-                    if (diag) {
-                        const int4 qa = lds_i4(&tq[c8 * 8]);
-                        const int4 qb = lds_i4(&tq[c8 * 8 + 4]);
-                        const int qs[8] = {qa.x, qa.y, qa.z, qa.w, qb.x, qb.y, qb.z, qb.w};
-#pragma unroll
-                        for (int e = 0; e < 8; ++e) pr[e] = (qs[e] >= key) ? pr[e] : 0.f;
-                    }
-                    if (!kvalid) {
-#pragma unroll
-                        for (int e = 0; e < 8; ++e) pr[e] = 0.f;
-                    }
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        acc[e] = add2(acc[e], pk(pr[2 * e], pr[2 * e + 1]));
-                        pp[c8 * 4 + e] = pack_bf16x2(pr[2 * e], pr[2 * e + 1]);
-                    }
+            float* rb = myred + (k2 & 1) * (4 * kBM);  // [4 warps][128 columns]
+            if (ok) {
+                tc_fence_after();
+                int lim;
+                if (is_state) {
+                    lim = min(kBN, count - j * kBN);
+                } else {
+                    const int f0 = (j - nst) * kBN;
+                    lim = min(kBN, (p.causal ? min(T, my_tq + 1) : T) - f0);
                 }
-                if (ch < 3) tmem_ld_wait();
-            }
-            // the score buffer is free as soon as it is in registers
-            tc_fence_before();
-            mbar_arrive(&s_empty[b]);
-            if (j >= 2) {
-                ok = __all_sync(0xffffffffu,
-                                wait_until(&p_empty[wg], ((j >> 1) - 1) & 1, deadline));
-                if (!ok) break;
-            }
+                const f2 cc = pk(c, c), nl = pk(nlse, nlse);
+                float v[4][32];
 #pragma unroll
-            for (int c8 = 0; c8 < kBM / 8; ++c8)
-                *reinterpret_cast<uint4*>(Pb + (c8 >> 3) * (kBN * 128) + sw128_offset(row, c8 & 7)) =
-                    make_uint4(pp[c8 * 4], pp[c8 * 4 + 1], pp[c8 * 4 + 2], pp[c8 * 4 + 3]);
-            fence_proxy_async_smem();
-            mbar_arrive(&p_full[wg]);
-            float s0, s1;
-            upk(add2(add2(acc[0], acc[1]), add2(acc[2], acc[3])), s0, s1);
-            if (kvalid) part[is_state ? key : B + key] = s0 + s1;
+                for (int ch = 0; ch < 4; ++ch) tmem_ld32(tS + ch * 32, v[ch]);
+                tmem_ld_wait();
+#pragma unroll
+                for (int ch = 0; ch < 4; ++ch) {
+                    float (&x)[32] = v[ch];
+#pragma unroll
+                    for (int e = 0; e < 32; e += 2) {
+                        float x0, x1;
+                        upk(fma2(pk(x[e], x[e + 1]), cc, nl), x0, x1);
+                        x[e] = ex2(x0);
+                        x[e + 1] = ex2(x1);
+                    }
+                    if (lim < kBN) {
+#pragma unroll
+                        for (int e = 0; e < 32; ++e) x[e] = (ch * 32 + e < lim) ? x[e] : 0.f;
+                    }
+                    uint32_t pw[16];
+#pragma unroll
+                    for (int e = 0; e < 16; ++e) pw[e] = pack_bf16x2(x[2 * e], x[2 * e + 1]);
+                    // P chunk -> buffer columns [16 ch, 16 ch + 16) (scores of
+                    // every chunk are already in registers)
+                    tmem_st16(tS + ch * 16, pw);
+                }
+                tmem_st_wait();
+                tc_fence_before();
+                mbar_arrive(&p_full[wg]);
+                // the column sums run while the tensor core does this tile's P V
+#pragma unroll
+                for (int ch = 0; ch < 4; ++ch)
+                    rb[quad * kBM + ch * 32 + lane] = warp_colsum32(v[ch], lane);
+            }
+            named_bar_sync(2 + wg, 128);
+            if (ok) {
+                const float s = rb[0 * kBM + ct] + rb[1 * kBM + ct] + rb[2 * kBM + ct] +
+                                rb[3 * kBM + ct];
+                const int key = (is_state ? j : j - nst) * kBN + ct;
+                if (is_state ? key < count : key < T) part[is_state ? key : B + key] = s;
+            }
         }
         // Frame keys no row of this tile can see receive zero importance here.
-        for (int t = nft * kBN + ct; t < T; t += 256) part[B + t] = 0.f;
+        for (int t = nft * kBN + (threadIdx.x - 128); t < T; t += 256) part[B + t] = 0.f;
 
-        // ---------------- epilogue: O rows (thread = query row) -> bf16 out;
-        // warpgroup wg stores columns [wg*D/2, (wg+1)*D/2)
+        // ---------------- epilogue: O rows -> bf16 out; warpgroup wg stores
+        // columns [wg*D/2, (wg+1)*D/2)
         if (ok) ok = __all_sync(0xffffffffu, wait_until(o_full, 0, deadline));
         if (ok) {
             tc_fence_after();
-            const bool valid = my_r < rows;
             __nv_bfloat16* dst = p.out;
-            if (valid) {
+            if (row_valid) {
                 const int t = my_r / G, g = my_r - t * G;
                 dst += ((static_cast<size_t>(u) * T + t) * p.Hq + hkv * G + g) * D;
             }
 #pragma unroll
-            for (int cc = 0; cc < D / 64; ++cc) {
-                const int col = wg * (D / 2) + cc * 32;
+            for (int cc2 = 0; cc2 < D / 64; ++cc2) {
+                const int col = wg * (D / 2) + cc2 * 32;
                 float o[32];
-                tmem_ld32(tlane + kSBuf * 128 + col, o);
+                tmem_ld32(tbase + lane_off + kColO + col, o);
                 tmem_ld_wait();
-                if (valid) {
+                if (row_valid) {
 #pragma unroll
                     for (int e = 0; e < 4; ++e) {
                         const uint4 w = make_uint4(
@@ -600,13 +619,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 }
 
-}  // namespace
-
-size_t attn_smem_bytes(int D)
-{
-    return D == 64 ? AttnLayout<64>::kAlloc : AttnLayout<128>::kAlloc;
-}
-
 // The register split (WG0 down to 80, the softmax warpgroups up to 208 per
 // thread) must fit the registers the CTA is launched with, or setmaxnreg.inc
 // would wait forever: 128 * 80 + 256 * 208 = 63488 <= 384 threads * 168.
@@ -623,6 +635,13 @@ cudaError_t prepare_one()
     return cudaFuncSetAttribute(frame_attn_lse_importance<D>,
                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 AttnLayout<D>::kAlloc);
+}
+
+}  // namespace
+
+size_t attn_smem_bytes(int D)
+{
+    return D == 64 ? AttnLayout<64>::kAlloc : AttnLayout<128>::kAlloc;
 }
 
 cudaError_t attn_prepare(int D)
