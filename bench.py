@@ -277,7 +277,8 @@ def run_ours(args, world, rank, local):
         q, k, v = frames[n]
         rc = eng.prefill_frame(q, k, v, out, imp)
         if rc != 0:
-            raise RuntimeError(f"statekv_prefill_frame returned {rc}")
+            raise RuntimeError(f"statekv_prefill_frame returned {rc} "
+                               f"(device word 0x{eng.device_error():x}) at frame {n + 1}")
 
     eng.profile(True)  # creates the event pool outside the timed region
     for n in range(fill + args.warmup):

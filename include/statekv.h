@@ -57,7 +57,8 @@ typedef enum {
     STATEKV_ERR_CACHE_FULL = 3,      /* a stream/layer already holds max_frames frames */
     STATEKV_ERR_CUDA = 4,            /* a CUDA runtime call failed */
     STATEKV_ERR_DEVICE_TIMEOUT = 5,  /* a kernel's bounded wait expired (sticky) */
-    STATEKV_ERR_ARENA_TOO_SMALL = 6  /* arena smaller than statekv_arena_bytes() */
+    STATEKV_ERR_ARENA_TOO_SMALL = 6, /* arena smaller than statekv_arena_bytes() */
+    STATEKV_ERR_DEVICE_FAULT = 7     /* a kernel detected an internal inconsistency (sticky) */
 } statekv_status;
 
 typedef struct statekv_handle statekv_handle;
@@ -153,9 +154,14 @@ typedef struct {
 statekv_status statekv_profile_enable(statekv_handle* h, int32_t enable);
 statekv_status statekv_profile_read(statekv_handle* h, statekv_profile* out);
 
-/* Synchronises the device and reports a device error (DEVICE_TIMEOUT) if a
- * kernel recorded one. */
+/* Synchronises the device and reports a device error (DEVICE_TIMEOUT or
+ * DEVICE_FAULT) if a kernel recorded one. */
 statekv_status statekv_sync(statekv_handle* h);
+
+/* The raw device status word (0 = none): low byte 1 = an attention-kernel
+ * wait expired (bits 8..15 name the waiting site), 2 = the selection kernel
+ * found an inconsistent top-B split.  Read without synchronising. */
+statekv_status statekv_device_error(const statekv_handle* h, int32_t* code);
 
 void statekv_destroy(statekv_handle* h);
 const char* statekv_status_string(statekv_status s);

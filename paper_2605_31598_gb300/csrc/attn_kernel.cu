@@ -242,6 +242,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int row_hi = min(rows, (mt + 1) * kBM) - 1;
     const int nft = p.causal ? (row_hi / G) / kBN + 1 : (T + kBN - 1) / kBN;
     const int nt = nst + nft;
+    // The query tiles of one KV head read the same state tiles; each starts at
+    // a different one (a fixed rotation by mt) so they do not all request the
+    // same L2 lines at the same moment.  Frame tiles keep their order.
+    const int rot = nst > 0 ? (mt * 3) % nst : 0;
+    auto state_tile = [&](int t) { return t + rot < nst ? t + rot : t + rot - nst; };
     const unsigned long long deadline = globaltimer() + p.watchdog_ns;
 
     if (threadIdx.x == 0) {
@@ -270,9 +275,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     const uint32_t tbase = *tmem_slot;
 
-    auto fail = [&]() {
-        *abort_flag = 1;
-        *reinterpret_cast<volatile int32_t*>(p.status) = DEV_TIMEOUT_ATTN;
+    // Records an expired wait: DEV_TIMEOUT_ATTN with the waiting site in bits
+    // 8..15 (see DeviceError), and tells every role to stop.
+    auto fail = [&](int site) {
+        if (atomicExch(const_cast<int*>(abort_flag), 1) == 0)  // first failure in the CTA
+            *reinterpret_cast<volatile int32_t*>(p.status) = DEV_TIMEOUT_ATTN | (site << 8);
     };
 
     if (warp < 4) {
@@ -296,7 +303,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 // once every pass-A MMA has released them (before that, a wait on
                 // their empty barriers could match an earlier phase of the same
                 // parity).
-                if (!kprod && !wait_until(a_done, 0, deadline)) fail();
+                if (!kprod && !wait_until(a_done, 0, deadline)) fail(1);
                 const int nload = kprod ? 2 * nt : nt;
                 for (int n = 0; n < nload; ++n) {
                     if (*abort_flag) break;
@@ -311,7 +318,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         use = pass_a_uses(nt, slot) + tile / kKSlotsB;
                     }
                     if (use >= 1 && !wait_until(&slot_empty[slot], (use - 1) & 1, deadline)) {
-                        fail();
+                        fail(kprod ? 2 : 3);
                         break;
                     }
                     uint8_t* dst = sSlot + slot * L::kTileBytes;
@@ -320,7 +327,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     for (int h = 0; h < D / 64; ++h) {
                         if (tile < nst)
                             tma_load_4d(dst + h * (kBN * 128), smap, &slot_full[slot], h * 64,
-                                        tile * kBN, hkv, ua);
+                                        state_tile(tile) * kBN, hkv, ua);
                         else
                             tma_load_4d(dst + h * (kBN * 128), fmap, &slot_full[slot], h * 64,
                                         hkv, (tile - nst) * kBN, u);
@@ -343,6 +350,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const uint32_t tQ = tbase, tO = tbase + kColO;
                 constexpr uint32_t kIdQK = idesc_bf16_f32(kBM, kBN, false, false);
                 constexpr uint32_t kIdPV = idesc_bf16_f32(kBM, D, false, true);
+                int site = 4;  // first wait that expired, for the status word
                 bool ok = wait_until(q_full, 0, deadline);
                 // QK^T of global sequence index it (pass A: it < nt; pass B: nt + j)
                 // into score buffer it & 1.
@@ -352,7 +360,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const int j = it - nt;
                     const int slot = pass_b ? j % kKSlotsB : it % kSlots;
                     const int use = pass_b ? pass_a_uses(nt, slot) + j / kKSlotsB : it / kSlots;
+                    site = 5;
                     if (!wait_until(&slot_full[slot], use & 1, deadline)) return false;
+                    site = 6;
                     // the buffer's previous tile (it - 2) must be consumed: read by
                     // its warpgroup in pass A, or read by its P V in pass B
                     if (it >= 2) {
@@ -377,7 +387,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const int w = (nt + j) & 1;
                     const int slot = kKSlotsB + j % kKSlotsB;
                     const int use = pass_a_uses(nt, slot) + j / kKSlotsB;
+                    site = 7;
                     if (!wait_until(&p_full[w], (j >> 1) & 1, deadline)) return false;
+                    site = 8;
                     if (!wait_until(&slot_full[slot], use & 1, deadline)) return false;
                     tc_fence_after();
                     const uint32_t vb = aSlot + slot * L::kTileBytes;
@@ -394,12 +406,21 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int it = isx ? 0 : 1; ok && it < nt; it += 2) ok = issue_qk(it);
                 if (ok) umma_commit(a_done);
                 if (isx) {  // pass B Q K^T, in tile order
+                    // A K slot's previous occupant may be one of Y's pass-A tiles,
+                    // possibly still in flight; waiting on the slot before that
+                    // load lands could match an earlier phase of the same parity.
+                    // Once every pass-A MMA has completed, every pass-A load has
+                    // landed.
+                    if (ok) {
+                        site = 9;
+                        ok = wait_until(a_done, 0, deadline);
+                    }
                     for (int j = 0; ok && j < nt; ++j) ok = issue_qk(nt + j);
                 } else {    // pass B P V, in tile order
                     for (int j = 0; ok && j < nt; ++j) ok = issue_pv(j);
                     if (ok) umma_commit(o_full);
                 }
-                if (!ok) fail();
+                if (!ok) fail(site + (isx ? 0 : 16));
                 // Every MMA issued so far must finish before TMEM is released.
                 umma_commit(drain);
                 wait_until(drain, 0, globaltimer() + p.watchdog_ns);
@@ -452,6 +473,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
 
         bool ok = true;
+        int site = 10;  // first wait that expired, for the status word
         // ---------------- pass A: online max / sum of exp2 over this warpgroup's tiles
         float m = -INFINITY, l = 0.f;  // log2 units, scaled
         for (int it = wg; it < nt; it += 2) {
@@ -460,7 +482,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_fence_after();
             int lim;  // keys [0, lim) of this tile are visible to this row
             if (it < nst) {
-                lim = min(kBN, count - it * kBN);
+                lim = min(kBN, count - state_tile(it) * kBN);
             } else {
                 const int f0 = (it - nst) * kBN;
                 lim = min(kBN, (p.causal ? min(T, my_tq + 1) : T) - f0);
@@ -507,6 +529,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 m = m_new;
             }
         }
+        if (ok) site = 11;
         stat[(wg * 2 + 0) * kBM + row] = m;
         stat[(wg * 2 + 1) * kBM + row] = l;
         named_bar_sync(1, 256);
@@ -534,7 +557,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc_fence_after();
                 int lim;
                 if (is_state) {
-                    lim = min(kBN, count - j * kBN);
+                    lim = min(kBN, count - state_tile(j) * kBN);
                 } else {
                     const int f0 = (j - nst) * kBN;
                     lim = min(kBN, (p.causal ? min(T, my_tq + 1) : T) - f0);
@@ -577,10 +600,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (ok) {
                 const float s = rb[0 * kBM + ct] + rb[1 * kBM + ct] + rb[2 * kBM + ct] +
                                 rb[3 * kBM + ct];
-                const int key = (is_state ? j : j - nst) * kBN + ct;
+                const int key = (is_state ? state_tile(j) : j - nst) * kBN + ct;
                 if (is_state ? key < count : key < T) part[is_state ? key : B + key] = s;
             }
         }
+        if (ok) site = 12;
         // Frame keys no row of this tile can see receive zero importance here.
         for (int t = nft * kBN + (threadIdx.x - 128); t < T; t += 256) part[B + t] = 0.f;
 
@@ -613,7 +637,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             }
         }
-        if (!ok) fail();
+        if (!ok) fail(site + 32 * wg);
         tc_fence_before();
         __syncthreads();
     }

@@ -153,6 +153,12 @@ struct statekv_handle {
 
 namespace {
 
+statekv_status device_status(int32_t word)
+{
+    if (word == 0) return STATEKV_OK;
+    return (word & 0xFF) == DEV_TIMEOUT_ATTN ? STATEKV_ERR_DEVICE_TIMEOUT : STATEKV_ERR_DEVICE_FAULT;
+}
+
 statekv_status check_args(const statekv_handle* h, const statekv_frame_args* a, bool host)
 {
     if (!h || !a) return STATEKV_ERR_INVALID_ARG;
@@ -168,7 +174,7 @@ statekv_status check_args(const statekv_handle* h, const statekv_frame_args* a, 
             return STATEKV_ERR_INVALID_ARG;
     }
     if (host && !c.host_staging) return STATEKV_ERR_INVALID_ARG;
-    if (*h->status_host != 0) return STATEKV_ERR_DEVICE_TIMEOUT;
+    if (*h->status_host != 0) return device_status(*h->status_host);
     for (int s = a->stream_begin; s < a->stream_begin + a->stream_count; ++s)
         for (int l = a->layer_begin; l < a->layer_begin + a->layer_count; ++l)
             if (h->frames_host[static_cast<size_t>(s) * c.num_layers + l] >= c.max_frames)
@@ -467,7 +473,14 @@ statekv_status statekv_sync(statekv_handle* h)
 {
     if (!h) return STATEKV_ERR_INVALID_ARG;
     if (cudaDeviceSynchronize() != cudaSuccess) return STATEKV_ERR_CUDA;
-    return *h->status_host != 0 ? STATEKV_ERR_DEVICE_TIMEOUT : STATEKV_OK;
+    return device_status(*h->status_host);
+}
+
+statekv_status statekv_device_error(const statekv_handle* h, int32_t* code)
+{
+    if (!h || !code) return STATEKV_ERR_INVALID_ARG;
+    *code = *h->status_host;
+    return STATEKV_OK;
 }
 
 void statekv_destroy(statekv_handle* h)
@@ -491,6 +504,7 @@ const char* statekv_status_string(statekv_status s)
     case STATEKV_ERR_CUDA: return "CUDA runtime error";
     case STATEKV_ERR_DEVICE_TIMEOUT: return "device wait timed out";
     case STATEKV_ERR_ARENA_TOO_SMALL: return "arena too small";
+    case STATEKV_ERR_DEVICE_FAULT: return "device-side consistency check failed";
     }
     return "unknown status";
 }

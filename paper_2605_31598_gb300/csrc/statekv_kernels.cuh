@@ -15,11 +15,16 @@
 
 namespace statekv {
 
-// Device error codes written to the status word (0 = no error).
+// Device error codes written to the status word (0 = no error).  The low
+// byte is the kind; an attention-kernel timeout carries the waiting site in
+// bits 8..15 (the first expired wait of the CTA): 1 V producer (pass A
+// done), 2/3 K/V producer (free slot), 4..9 MMA issuer X (Q ready, K/V slot,
+// score buffer, P, V slot, pass A done; +16 for issuer Y), 10..12 softmax
+// warpgroup 0 (pass A, pass B, O ready; +32 for warpgroup 1).
 enum DeviceError : int32_t {
     DEV_OK = 0,
     DEV_TIMEOUT_ATTN = 1,
-    DEV_BAD_SELECT = 2,
+    DEV_BAD_SELECT = 2,  // the top-B selection admitted more tokens than free slots
 };
 
 // Tile sizes of the attention kernel: 128 query rows x 128 keys per MMA tile.

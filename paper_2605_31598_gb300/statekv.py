@@ -19,11 +19,12 @@ STATEKV_OK = 0
 STATUS_NAMES = {
     0: "STATEKV_OK", 1: "STATEKV_ERR_INVALID_ARG", 2: "STATEKV_ERR_UNSUPPORTED",
     3: "STATEKV_ERR_CACHE_FULL", 4: "STATEKV_ERR_CUDA", 5: "STATEKV_ERR_DEVICE_TIMEOUT",
-    6: "STATEKV_ERR_ARENA_TOO_SMALL",
+    6: "STATEKV_ERR_ARENA_TOO_SMALL", 7: "STATEKV_ERR_DEVICE_FAULT",
 }
 EXPORTED = ("statekv_arena_bytes", "statekv_init", "statekv_prefill_frame",
             "statekv_prefill_frame_host", "statekv_state_view", "statekv_cache_view",
             "statekv_profile_enable", "statekv_profile_read", "statekv_sync",
+            "statekv_device_error",
             "statekv_destroy", "statekv_status_string")
 
 
@@ -95,6 +96,8 @@ def lib() -> ctypes.CDLL:
             L.statekv_profile_read.restype = st
             L.statekv_sync.argtypes = [ctypes.c_void_p]
             L.statekv_sync.restype = st
+            L.statekv_device_error.argtypes = [ctypes.c_void_p, P(ctypes.c_int32)]
+            L.statekv_device_error.restype = st
             L.statekv_destroy.argtypes = [ctypes.c_void_p]
             L.statekv_destroy.restype = None
             L.statekv_status_string.argtypes = [ctypes.c_int]
@@ -163,6 +166,12 @@ def statekv_profile_read(handle: int) -> statekv_profile:
 
 def statekv_sync(handle: int) -> int:
     return lib().statekv_sync(handle)
+
+
+def statekv_device_error(handle: int) -> int:
+    code = ctypes.c_int32(0)
+    check(lib().statekv_device_error(handle, ctypes.byref(code)), "statekv_device_error")
+    return code.value
 
 
 def statekv_destroy(handle: int):
@@ -277,3 +286,7 @@ class StateKV:
 
     def sync(self) -> int:
         return statekv_sync(self.handle)
+
+    def device_error(self) -> int:
+        """Raw device status word (0 = none); see statekv_device_error."""
+        return statekv_device_error(self.handle)
