@@ -163,6 +163,34 @@ statekv_status statekv_sync(statekv_handle* h);
  * found an inconsistent top-B split.  Read without synchronising. */
 statekv_status statekv_device_error(const statekv_handle* h, int32_t* code);
 
+/* Frame attention with importance (steps a1 and a2) for ONE (stream, layer)
+ * against a caller-given state, for callers that cannot allocate device
+ * memory -- e.g. plugins held to a host application's memory budget, or code
+ * that must not call cudaMalloc while another component captures a stream.
+ * The paper has no counterpart: this is a packaging of the same kernel.
+ * Its scratch (importance partials, per-head counts, a status word) is a
+ * fixed set of file-scope device arrays, resident on every GPU that loads the
+ * library until the process exits: at most 2^20 fp32 partials, i.e.
+ * num_kv_heads * ceil(G * T / 128) * (B + T) <= 1048576 with G = Hq / Hkv, and
+ * num_kv_heads <= 64; larger shapes return STATEKV_ERR_UNSUPPORTED.  The call
+ * allocates nothing.  Its first call on a device looks up the arrays' device
+ * addresses; make that first call before any stream capture.  Calls share the
+ * scratch: calls that overlap on the GPU race.  The call synchronises `stream`
+ * before it returns and reports its own DEVICE_TIMEOUT.
+ *   cfg           num_q_heads, num_kv_heads, head_dim, tokens_per_frame,
+ *                 state_capacity (B), causal_in_frame, softmax_scale,
+ *                 watchdog_ms are used; the rest is ignored
+ *   q, k, v       bf16 [T][Hq][d], [T][Hkv][d], [T][Hkv][d] (device)
+ *   state_k/v     bf16 [Hkv][B][d] (device); rows [0, state_count) are valid
+ *   out           bf16 [T][Hq][d] (device)
+ *   importance    fp32 [Hkv][B + T] (device), columns as in statekv_frame_args
+ * Nothing of the handle-based state is read or written. */
+statekv_status statekv_frame_attention_noalloc(const statekv_config* cfg, const void* q,
+                                               const void* k, const void* v, const void* state_k,
+                                               const void* state_v, int32_t state_count,
+                                               void* out, float* importance,
+                                               statekv_stream stream);
+
 void statekv_destroy(statekv_handle* h);
 const char* statekv_status_string(statekv_status s);
 

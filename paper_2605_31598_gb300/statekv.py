@@ -24,7 +24,7 @@ STATUS_NAMES = {
 EXPORTED = ("statekv_arena_bytes", "statekv_init", "statekv_prefill_frame",
             "statekv_prefill_frame_host", "statekv_state_view", "statekv_cache_view",
             "statekv_profile_enable", "statekv_profile_read", "statekv_sync",
-            "statekv_device_error",
+            "statekv_device_error", "statekv_frame_attention_noalloc",
             "statekv_destroy", "statekv_status_string")
 
 
@@ -98,6 +98,11 @@ def lib() -> ctypes.CDLL:
             L.statekv_sync.restype = st
             L.statekv_device_error.argtypes = [ctypes.c_void_p, P(ctypes.c_int32)]
             L.statekv_device_error.restype = st
+            L.statekv_frame_attention_noalloc.argtypes = [
+                P(statekv_config), ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
+                ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int32, ctypes.c_void_p,
+                ctypes.c_void_p, ctypes.c_void_p]
+            L.statekv_frame_attention_noalloc.restype = st
             L.statekv_destroy.argtypes = [ctypes.c_void_p]
             L.statekv_destroy.restype = None
             L.statekv_status_string.argtypes = [ctypes.c_int]
@@ -172,6 +177,17 @@ def statekv_device_error(handle: int) -> int:
     code = ctypes.c_int32(0)
     check(lib().statekv_device_error(handle, ctypes.byref(code)), "statekv_device_error")
     return code.value
+
+
+def statekv_frame_attention_noalloc(cfg: statekv_config, q: int, k: int, v: int, state_k: int,
+                                    state_v: int, state_count: int, out: int, importance: int,
+                                    stream: int) -> int:
+    """Attention + importance for one (stream, layer) without device allocation
+    (scratch lives in fixed device arrays of the library); returns the status."""
+    return lib().statekv_frame_attention_noalloc(
+        ctypes.byref(cfg), ctypes.c_void_p(q), ctypes.c_void_p(k), ctypes.c_void_p(v),
+        ctypes.c_void_p(state_k), ctypes.c_void_p(state_v), state_count, ctypes.c_void_p(out),
+        ctypes.c_void_p(importance), ctypes.c_void_p(stream))
 
 
 def statekv_destroy(handle: int):
