@@ -335,6 +335,20 @@ def run_ours(args, world, rank, local):
     }
     value = world * S * args.steps / (total_ms_max * 1e-3)
     ps = sorted(per_step)
+    # flat per-frame cost: slope of a linear fit of per-frame time against the
+    # frame index, and the p50 of the first 32 timed frames vs the last half
+    first = fill + args.warmup + 1
+    idx = list(range(first, first + args.steps))
+    n = len(per_step)
+    mx, my = sum(idx) / n, sum(per_step) / n
+    var = sum((x - mx) ** 2 for x in idx)
+    slope = sum((x - mx) * (y - my) for x, y in zip(idx, per_step)) / var if var > 0 else 0.0
+    early = sorted(per_step[:32])
+    late = sorted(per_step[n // 2:])
+    flatness = {"frames": f"{first}..{first + n - 1}",
+                "slope_pct_per_100_frames": 100.0 * 100.0 * slope / my if my > 0 else None,
+                "p50_first32_us": 1e3 * early[len(early) // 2],
+                "p50_last_half_us": 1e3 * late[len(late) // 2]}
     line = {
         "metric": METRIC,
         "value": value,
@@ -364,6 +378,7 @@ def run_ours(args, world, rank, local):
                      "kernel": "frame_attn_lse_importance",
                      "flops_per_launch": flops},
         "kernels": kernels,
+        "flatness": flatness,
         "gpu_launches": 3 * args.steps,
     }
     clocks = sampler.summary(t_wall0, t_wall1)
