@@ -14,18 +14,28 @@
 // tcgen05 runs every contraction with the A operand in TMEM (Q for Q K^T, P
 // for P V), so each MMA streams only K or V from shared memory.  TMEM
 // (512 columns): Q | score/P buffer of softmax warpgroup 0 | of warpgroup 1 |
-// O.  K and V tiles arrive by TMA (128-byte swizzle) in six 32 KB slots:
-// pass A streams K through all six; pass B streams K through slots 0-2 and V
-// through 3-5, each ring fed by its own producer thread.
+// O; P overwrites the scores it came from.
+//
+// Every query tile of a KV head reads the same K and V tiles, and keeping the
+// tensor core busy would take about as many bytes per cycle from L2 as the
+// SM can receive.  So for D = 128 two CTAs (consecutive query tiles of one
+// KV head) form a cluster: each loads one 64-column half of every K/V tile by
+// TMA with multicast into both CTAs' shared memory, halving the L2 reads and
+// TMA issues per CTA.  Both CTAs walk the same key tiles (the frame tiles
+// visible to either).  Tiles stream through a ring of six 32 KB slots in one
+// sequence: pass A's K tiles, then pass B's K(0) V(0) K(1) V(1) ...; a slot
+// is refilled once the MMAs of every CTA in the cluster have read it (the
+// MMA commit arrives on the slot's barrier in each CTA).
 //
 // 384 threads, three warpgroups:
-//   WG0  warp 0 K producer, warp 2 V producer, warps 1 and 3 MMA issuers
-//        (warp 1 also owns TMEM).  A tcgen05.mma issues at the tensor core's
-//        pace, so every barrier wait of an issuing thread idles the tensor
-//        core; with two issuers one waits while the other's MMAs run.  Issuer
-//        X (warp 1) issues the pass-A Q K^T of even tiles and every pass-B
-//        Q K^T; issuer Y (warp 3) the pass-A Q K^T of odd tiles and every P V
-//        (in order, so O accumulates deterministically).
+//   WG0  warp 0 producer (TMA), warps 1 and 3 MMA issuers X and Y (warp 1
+//        also owns TMEM).  tcgen05.mma issue blocks at the tensor core's pace,
+//        so each barrier wait of an issuing thread idles the tensor core; with
+//        two issuers one waits while the other's MMAs run.  X issues the
+//        pass-A Q K^T of even tiles and every pass-B Q K^T; Y the pass-A Q K^T
+//        of odd tiles and every P V (in order, so O accumulates
+//        deterministically).  Descriptors are precomputed words, so an MMA
+//        costs the issuing warp an add or two besides itself.
 //   WG1, WG2  softmax warpgroups: thread = query row; they take alternate key
 //        tiles, each with its own TMEM score buffer, so the tensor core works
 //        on one warpgroup's tile while the other computes exponentials.
@@ -42,11 +52,15 @@ namespace {
 using namespace ptx;
 
 constexpr int kThreads = 384;
-constexpr int kSlots = 6;        // 32 KB K/V tile slots (D = 128)
-constexpr int kKSlotsB = 3;      // pass B: K slots 0..2, V slots 3..5
-constexpr uint32_t kColS0 = 128; // TMEM columns: Q [0, D/2), S0, S1, O
-constexpr uint32_t kColS1 = 256;
+constexpr int kSlots = 6;        // 32 KB K/V tile slots (D = 128), one ring
+constexpr uint32_t kColS0 = 128; // TMEM columns: Q [0, D/2), S0, S1, O; pass A also
+constexpr uint32_t kColS1 = 256; // uses O's columns as a third score buffer S2
 constexpr uint32_t kColO = 384;
+constexpr int kSA = 3;           // pass-A score buffers
+// Pass-A barriers are indexed by tile mod 6 (buffer tile % 3, warpgroup and
+// issuer tile % 2), so each waiter has seen the barrier's previous phase and
+// can never mistake a phase two back for the one it waits for.
+constexpr int kSA2 = 2 * kSA;
 
 template <int D>
 struct AttnLayout {
@@ -55,9 +69,9 @@ struct AttnLayout {
     static constexpr int kOffRed = kOffSlots + kSlots * kTileBytes;  // float[2 wg][2][4][128]
     static constexpr int kOffStat = kOffRed + 2 * 2 * 4 * kBM * 4;   // float[2][2][128]
     static constexpr int kOffBar = kOffStat + 4 * kBM * 4;
-    // slot_full[6] slot_empty[6] s_full[2] s_read[2] p_full[2] pv_done[2]
-    // q_full o_full drain a_done
-    static constexpr int kNumBars = 24;
+    // slot_full[6] slot_empty[6] sa_full[6] sa_read[6] sb_full[2] p_full[2]
+    // pv_done[2] q_full o_full drain a_done a_read
+    static constexpr int kNumBars = 40;
     static constexpr int kOffMisc = kOffBar + kNumBars * 8;
     static constexpr int kBytes = kOffMisc + 16;
     static constexpr int kAlloc = kBytes + 1024;  // room to align the base to 1 KB
@@ -134,15 +148,74 @@ __device__ __forceinline__ void named_bar_sync(int id, int nthreads)
     asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
 }
 
-// D[tmem] (+)= A[tmem] * B[smem], bf16 inputs, fp32 accumulator.
-__device__ __forceinline__ void umma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc,
-                                        uint32_t idesc, uint32_t accumulate)
+// One MMA group, D[d] (+)= A[a + 8k] * B_k for k < NK (bf16 in, fp32
+// accumulator, A in TMEM), with B's descriptor for step k given as its two
+// 32-bit words (lo + off(k), hi): the issuing warp shares its SM sub-partition
+// with the softmax warps, so each MMA should cost it as few instructions as
+// possible.
+template <int NK, bool kMajorB>
+__device__ __forceinline__ void mma_group(uint32_t d, uint32_t a, uint32_t blo, uint32_t bhi,
+                                          uint32_t idesc, bool accumulate)
+{
+#pragma unroll
+    for (int k = 0; k < NK; ++k) {
+        // K-major B: 16 KB per 64-wide K half of a 128-row tile, 32 B per
+        // 16-element step inside a half; MN-major B: 2 KB per step.
+        const uint32_t off =
+            kMajorB ? ((k >> 2) * (kBN * 128) + (k & 3) * 32) >> 4 : (k * 2048) >> 4;
+        if (k == 0 && !accumulate)
+            asm volatile(
+                "{\n\t.reg .b64 bd;\n\t"
+                "mov.b64 bd, {%2, %3};\n\t"
+                "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], bd, %4, 0;\n\t}" ::"r"(d),
+                "r"(a), "r"(blo + off), "r"(bhi), "r"(idesc)
+                : "memory");
+        else
+            asm volatile(
+                "{\n\t.reg .b64 bd;\n\t"
+                "mov.b64 bd, {%2, %3};\n\t"
+                "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], bd, %4, 1;\n\t}" ::"r"(d),
+                "r"(a + 8 * k), "r"(blo + off), "r"(bhi), "r"(idesc)
+                : "memory");
+    }
+}
+
+__device__ __forceinline__ uint32_t cluster_ctarank()
+{
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+
+// Every thread of every CTA in the cluster arrives and waits.
+__device__ __forceinline__ void cluster_sync_all()
 {
     asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "setp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
-        "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+        "barrier.cluster.arrive.release.aligned;\n\t"
+        "barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+// TMA tile load delivered to the same shared-memory offset, and completing on
+// the same mbarrier offset, in every CTA of `mask`.
+__device__ __forceinline__ void tma_load_4d_mc(void* dst, const void* tmap, uint64_t* bar, int c0,
+                                               int c1, int c2, int c3, uint16_t mask)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes"
+        ".multicast::cluster [%0], [%1, {%3, %4, %5, %6}], [%2], %7;" ::"r"(smem_addr(dst)),
+        "l"(reinterpret_cast<uint64_t>(tmap)), "r"(smem_addr(bar)), "r"(c0), "r"(c1), "r"(c2),
+        "r"(c3), "h"(mask)
+        : "memory");
+}
+
+// Arrives once on `bar` in every CTA of `mask` when this thread's MMAs so far
+// have completed.
+__device__ __forceinline__ void umma_commit_mc(uint64_t* bar, uint16_t mask)
+{
+    asm volatile(
+        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
+        " [%0], %1;" ::"r"(smem_addr(bar)),
+        "h"(mask)
         : "memory");
 }
 
@@ -163,25 +236,12 @@ __device__ __forceinline__ void tmem_st_wait()
     asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
 
-// K-major SW128 operand with `rows` rows: k-step ks (16 elements) of the tile.
-__device__ __forceinline__ uint64_t kmajor_desc(uint32_t base, int ks, int rows)
+// The ring carries pass A's K tiles (items 0 .. nt-1), then pass B's K(j)
+// (item nt + 2j) and V(j) (item nt + 2j + 1); item n sits in slot n % 6 as the
+// slot's use n / 6.
+__device__ __forceinline__ int qk_item(int nt, int it)  // it: Q K^T sequence index
 {
-    return sdesc_sw128(base + (ks >> 2) * (rows * 128) + (ks & 3) * 32, 16, 1024);
-}
-
-// MN-major SW128 operand whose 64-wide MN blocks are `block_bytes` apart:
-// k-step ks covers 16 K rows (2 groups of 8).
-__device__ __forceinline__ uint64_t mnmajor_desc(uint32_t base, int ks, uint32_t block_bytes)
-{
-    return sdesc_sw128(base + ks * 2048, block_bytes, 1024);
-}
-
-// Pass A tile `it` occupies slot it % 6; pass B K tile j slot j % 3 and V
-// tile j slot 3 + j % 3.  The use count of a slot before pass B is the number
-// of pass-A tiles it held.
-__device__ __forceinline__ int pass_a_uses(int nt, int slot)
-{
-    return nt > slot ? (nt - slot + kSlots - 1) / kSlots : 0;
+    return it < nt ? it : nt + 2 * (it - nt);
 }
 
 // Column sums over the warp's 32 rows of a 32-column chunk held one row per
@@ -201,7 +261,7 @@ __device__ __forceinline__ float warp_colsum32(float (&x)[32], int lane)
     return x[0];
 }
 
-template <int D>
+template <int D, int C>  // C: CTAs per cluster sharing K/V tiles (1 or 2)
 __global__ void __launch_bounds__(kThreads, 1)
     frame_attn_lse_importance(const __grid_constant__ CUtensorMap tm_sk,
                               const __grid_constant__ CUtensorMap tm_sv,
@@ -218,48 +278,59 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t* bars = reinterpret_cast<uint64_t*>(sm + L::kOffBar);
     uint64_t* slot_full = bars + 0;
     uint64_t* slot_empty = bars + 6;
-    uint64_t* s_full = bars + 12;   // QK^T result in score buffer w
-    uint64_t* s_read = bars + 14;   // pass A: warpgroup w has read score buffer w
-    uint64_t* p_full = bars + 16;   // pass B: warpgroup w has written P into buffer w
-    uint64_t* pv_done = bars + 18;  // pass B: the P V that read buffer w has completed
-    uint64_t* q_full = bars + 20;
-    uint64_t* o_full = bars + 21;
-    uint64_t* drain = bars + 22;
-    uint64_t* a_done = bars + 23;   // every pass-A MMA has completed
+    uint64_t* sa_full = bars + 12;  // pass A: Q K^T of tile i done (index i % 6)
+    uint64_t* sa_read = bars + 18;  // pass A: tile i read by its warpgroup (index i % 6)
+    uint64_t* sb_full = bars + 24;  // pass B: Q K^T result in score buffer w (of 2)
+    uint64_t* p_full = bars + 26;   // pass B: warpgroup w has written P into buffer w
+    uint64_t* pv_done = bars + 28;  // pass B: the P V that read buffer w has completed
+    uint64_t* q_full = bars + 30;
+    uint64_t* o_full = bars + 31;
+    uint64_t* drain = bars + 32;
+    uint64_t* a_done = bars + 33;   // every pass-A MMA has completed
+    uint64_t* a_read = bars + 34;   // both warpgroups have read every pass-A score tile
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + L::kOffMisc);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(sm + L::kOffMisc + 4);
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
-    const int mt = blockIdx.x;
+    const int mt = blockIdx.x;  // query tile; tiles >= MT (cluster padding) have no valid row
     const int hkv = blockIdx.y;
     const int u = blockIdx.z;
     const int ua = p.units.unit_abs(u);
     const int T = p.T, G = p.G, B = p.B;
     const int rows = G * T;
+    const bool tile_valid = mt < p.MT;
+    const int crank = C > 1 ? static_cast<int>(cluster_ctarank()) : 0;
     const int count = (B > 0) ? p.counts[ua * p.Hkv + hkv] : 0;
     const int nst = (count + kBN - 1) / kBN;
-    const int row_hi = min(rows, (mt + 1) * kBM) - 1;
+    // frame tiles seen by the cluster's last query tile (the union over the cluster)
+    const int mt_last = min(mt - crank + C - 1, p.MT - 1);
+    const int row_hi = min(rows, (mt_last + 1) * kBM) - 1;
     const int nft = p.causal ? (row_hi / G) / kBN + 1 : (T + kBN - 1) / kBN;
     const int nt = nst + nft;
-    // The query tiles of one KV head read the same state tiles; each starts at
-    // a different one (a fixed rotation by mt) so they do not all request the
-    // same L2 lines at the same moment.  Frame tiles keep their order.
-    const int rot = nst > 0 ? (mt * 3) % nst : 0;
+    const int nitems = 3 * nt;  // pass-A K tiles + pass-B K and V tiles
+    // The clusters of one KV head read the same state tiles; each starts at a
+    // different one (a fixed rotation) so they do not all request the same L2
+    // lines at the same moment.  Frame tiles keep their order.
+    const int rot = nst > 0 ? ((mt / C) * 3) % nst : 0;
     auto state_tile = [&](int t) { return t + rot < nst ? t + rot : t + rot - nst; };
     const unsigned long long deadline = globaltimer() + p.watchdog_ns;
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < kSlots; ++i) {
             mbar_init(&slot_full[i], 1);
-            mbar_init(&slot_empty[i], 1);
+            mbar_init(&slot_empty[i], C);  // one MMA commit per CTA of the cluster
+        }
+        for (int i = 0; i < kSA2; ++i) {
+            mbar_init(&sa_full[i], 1);
+            mbar_init(&sa_read[i], 128);
         }
         for (int i = 0; i < 2; ++i) {
-            mbar_init(&s_full[i], 1);
-            mbar_init(&s_read[i], 128);
+            mbar_init(&sb_full[i], 1);
             mbar_init(&p_full[i], 128);
             mbar_init(&pv_done[i], 1);
         }
+        mbar_init(a_read, 256);
         mbar_init(q_full, 256);
         mbar_init(o_full, 1);
         mbar_init(drain, 2);   // one commit per MMA issuer
@@ -272,6 +343,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_relinquish();
     }
     __syncthreads();
+    if (C > 1) cluster_sync_all();  // the partner's barriers exist before any multicast
     tc_fence_after();
     const uint32_t tbase = *tmem_slot;
 
@@ -284,136 +356,161 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     if (warp < 4) {
         asm volatile("setmaxnreg.dec.sync.aligned.u32 80;" ::: "memory");
-        if (warp == 0 || warp == 2) {
-            // ------------------------------------------------------------ producers
-            // warp 0: K tiles of both passes; warp 2: V tiles of pass B
+        if (warp == 0) {
+            // ------------------------------------------------------------ producer
+            // One ring of tiles for both passes; with a cluster, this CTA loads
+            // the d-half `crank` of every tile for both CTAs.
             if (lane == 0) {
-                const bool kprod = warp == 0;
-                if (kprod) {
-                    tma_prefetch_desc(&tm_fk);
-                    if (B > 0) tma_prefetch_desc(&tm_sk);
-                } else {
-                    tma_prefetch_desc(&tm_fv);
-                    if (B > 0) tma_prefetch_desc(&tm_sv);
+                tma_prefetch_desc(&tm_fk);
+                tma_prefetch_desc(&tm_fv);
+                if (B > 0) {
+                    tma_prefetch_desc(&tm_sk);
+                    tma_prefetch_desc(&tm_sv);
                 }
-                const CUtensorMap* smap = kprod ? &tm_sk : &tm_sv;
-                const CUtensorMap* fmap = kprod ? &tm_fk : &tm_fv;
-                int last_use[kSlots] = {-1, -1, -1, -1, -1, -1};
-                // V slots also carry pass-A K tiles: the V producer starts only
-                // once every pass-A MMA has released them (before that, a wait on
-                // their empty barriers could match an earlier phase of the same
-                // parity).
-                if (!kprod && !wait_until(a_done, 0, deadline)) fail(1);
-                const int nload = kprod ? 2 * nt : nt;
-                for (int n = 0; n < nload; ++n) {
-                    if (*abort_flag) break;
-                    int slot, use, tile;
-                    if (kprod && n < nt) {
-                        tile = n;
-                        slot = n % kSlots;
-                        use = n / kSlots;
-                    } else {
-                        tile = kprod ? n - nt : n;
-                        slot = (kprod ? 0 : kKSlotsB) + tile % kKSlotsB;
-                        use = pass_a_uses(nt, slot) + tile / kKSlotsB;
-                    }
-                    if (use >= 1 && !wait_until(&slot_empty[slot], (use - 1) & 1, deadline)) {
-                        fail(kprod ? 2 : 3);
+                int last_use[kSlots];
+#pragma unroll
+                for (int sl = 0; sl < kSlots; ++sl) last_use[sl] = -1;
+                // map and coordinates of item n (this CTA's d-half when C = 2)
+                auto item_src = [&](int n, const CUtensorMap*& map, int& c1, int& c2, int& c3) {
+                    const bool is_v = n >= nt && ((n - nt) & 1);
+                    const int tile = n < nt ? n : (n - nt) >> 1;
+                    map = tile < nst ? (is_v ? &tm_sv : &tm_sk) : (is_v ? &tm_fv : &tm_fk);
+                    c1 = tile < nst ? state_tile(tile) * kBN : hkv;
+                    c2 = tile < nst ? hkv : (tile - nst) * kBN;
+                    c3 = tile < nst ? ua : u;
+                };
+                bool ok = true;
+                for (int n = 0; n < nitems; ++n) {
+                    if (*abort_flag) {
+                        ok = false;
                         break;
                     }
+                    const int slot = n % kSlots, use = n / kSlots;
+                    if (use >= 1 && !wait_until(&slot_empty[slot], (use - 1) & 1, deadline)) {
+                        fail(2);
+                        ok = false;
+                        break;
+                    }
+                    const CUtensorMap* map;
+                    int c1, c2, c3;
+                    item_src(n, map, c1, c2, c3);
                     uint8_t* dst = sSlot + slot * L::kTileBytes;
                     mbar_arrive_expect_tx(&slot_full[slot], L::kTileBytes);
+                    if (C == 1) {
 #pragma unroll
-                    for (int h = 0; h < D / 64; ++h) {
-                        if (tile < nst)
-                            tma_load_4d(dst + h * (kBN * 128), smap, &slot_full[slot], h * 64,
-                                        state_tile(tile) * kBN, hkv, ua);
-                        else
-                            tma_load_4d(dst + h * (kBN * 128), fmap, &slot_full[slot], h * 64,
-                                        hkv, (tile - nst) * kBN, u);
+                        for (int h = 0; h < D / 64; ++h)
+                            tma_load_4d(dst + h * (kBN * 128), map, &slot_full[slot], h * 64, c1, c2, c3);
+                    } else {
+                        tma_load_4d_mc(dst + crank * (kBN * 128), map, &slot_full[slot], crank * 64, c1,
+                                       c2, c3, static_cast<uint16_t>((1u << C) - 1));
                     }
                     last_use[slot] = use;
                 }
-                if (*abort_flag) {
+                const unsigned long long dl = globaltimer() + p.watchdog_ns;
+                if (ok) {
+                    // Every CTA's MMAs have released every slot: no commit from the
+                    // partner is still on its way to this CTA's barriers.
+                    for (int sl = 0; sl < kSlots && sl < nitems; ++sl)
+                        wait_until(&slot_empty[sl], last_use[sl] & 1, dl);
+                } else {
                     // Let copies already in flight land before the CTA's memory goes away.
-                    const unsigned long long dl = globaltimer() + p.watchdog_ns;
                     for (int sl = 0; sl < kSlots; ++sl)
                         if (last_use[sl] >= 0) wait_until(&slot_full[sl], last_use[sl] & 1, dl);
+                    if (C > 1) {  // and those the partner may have sent
+                        const unsigned long long t_end = globaltimer() + 20000;
+                        while (globaltimer() < t_end) __nanosleep(1000);
+                    }
                 }
             }
             __syncwarp();
-        } else {
+        } else if (warp == 1 || warp == 3) {
             // ------------------------------------------------------------ MMA issuers
             if (lane == 0) {
                 const bool isx = warp == 1;
                 const uint32_t aSlot = smem_addr(sSlot);
+                const uint64_t dk = sdesc_sw128(aSlot, 16, 1024);         // K-major, slot 0
+                const uint64_t dv = sdesc_sw128(aSlot, kBN * 128, 1024);  // MN-major, slot 0
+                const uint32_t dk_lo = static_cast<uint32_t>(dk), d_hi = static_cast<uint32_t>(dk >> 32);
+                const uint32_t dv_lo = static_cast<uint32_t>(dv);
+                constexpr uint32_t kSlotStep = L::kTileBytes >> 4;  // descriptor address units
                 const uint32_t tQ = tbase, tO = tbase + kColO;
+                const uint32_t tS0 = tbase + kColS0, tS1 = tbase + kColS1;
                 constexpr uint32_t kIdQK = idesc_bf16_f32(kBM, kBN, false, false);
                 constexpr uint32_t kIdPV = idesc_bf16_f32(kBM, D, false, true);
+                constexpr uint16_t kAll = static_cast<uint16_t>((1u << C) - 1);
+                // the slot's barrier in every CTA of the cluster: this CTA's MMAs are
+                // done with the tile
+                auto release = [&](int slot) {
+                    if (C == 1)
+                        umma_commit(&slot_empty[slot]);
+                    else
+                        umma_commit_mc(&slot_empty[slot], kAll);
+                };
                 int site = 4;  // first wait that expired, for the status word
                 bool ok = wait_until(q_full, 0, deadline);
-                // QK^T of global sequence index it (pass A: it < nt; pass B: nt + j)
-                // into score buffer it & 1.
+                // S(it & 1) = Q K^T for sequence index it (pass A: it < nt; pass B: nt + j)
+                // pass A: S(it % 3) = Q K^T of tile it; pass B (it = nt + j): S(j')
+                // with j' = (nt + j) & 1
                 auto issue_qk = [&](int it) -> bool {
-                    const int w = it & 1;
                     const bool pass_b = it >= nt;
-                    const int j = it - nt;
-                    const int slot = pass_b ? j % kKSlotsB : it % kSlots;
-                    const int use = pass_b ? pass_a_uses(nt, slot) + j / kKSlotsB : it / kSlots;
+                    const int item = qk_item(nt, it);
+                    const int slot = item % kSlots;
                     site = 5;
-                    if (!wait_until(&slot_full[slot], use & 1, deadline)) return false;
+                    if (!wait_until(&slot_full[slot], (item / kSlots) & 1, deadline)) return false;
                     site = 6;
-                    // the buffer's previous tile (it - 2) must be consumed: read by
-                    // its warpgroup in pass A, or read by its P V in pass B
-                    if (it >= 2) {
-                        const int prev = it - 2;
-                        const bool ok2 =
-                            prev < nt
-                                ? wait_until(&s_read[w], (prev >> 1) & 1, deadline)
-                                : wait_until(&pv_done[w], ((prev - nt) >> 1) & 1, deadline);
-                        if (!ok2) return false;
+                    uint32_t tS;
+                    uint64_t* done;
+                    if (!pass_b) {
+                        // the buffer's previous tile (it - 3) has been read by its warpgroup
+                        const int b = it % kSA;
+                        if (it >= kSA) {
+                            const int prev = it - kSA;
+                            if (!wait_until(&sa_read[prev % kSA2], (prev / kSA2) & 1, deadline)) return false;
+                        }
+                        tS = b == 0 ? tS0 : b == 1 ? tS1 : tO;
+                        done = &sa_full[it % kSA2];
+                    } else {
+                        // the buffer's previous pass-B tile (j - 2) has been read by its P V
+                        const int j = it - nt, w = it & 1;
+                        if (j >= 2 && !wait_until(&pv_done[w], ((j - 2) >> 1) & 1, deadline)) return false;
+                        tS = w ? tS1 : tS0;
+                        done = &sb_full[w];
                     }
                     tc_fence_after();
-                    const uint32_t kb = aSlot + slot * L::kTileBytes;
-                    const uint32_t tS = tbase + (w ? kColS1 : kColS0);
-#pragma unroll
-                    for (int k = 0; k < D / 16; ++k)
-                        umma_ts(tS, tQ + k * 8, kmajor_desc(kb, k, kBN), kIdQK, k > 0);
-                    umma_commit(&s_full[w]);
-                    umma_commit(&slot_empty[slot]);
+                    mma_group<D / 16, true>(tS, tQ, dk_lo + slot * kSlotStep, d_hi, kIdQK, false);
+                    umma_commit(done);
+                    release(slot);
                     return true;
                 };
+                // O += P(j) V(j), P in score buffer (nt + j) & 1
                 auto issue_pv = [&](int j) -> bool {
                     const int w = (nt + j) & 1;
-                    const int slot = kKSlotsB + j % kKSlotsB;
-                    const int use = pass_a_uses(nt, slot) + j / kKSlotsB;
+                    const int item = nt + 2 * j + 1;
+                    const int slot = item % kSlots;
                     site = 7;
                     if (!wait_until(&p_full[w], (j >> 1) & 1, deadline)) return false;
                     site = 8;
-                    if (!wait_until(&slot_full[slot], use & 1, deadline)) return false;
+                    if (!wait_until(&slot_full[slot], (item / kSlots) & 1, deadline)) return false;
                     tc_fence_after();
-                    const uint32_t vb = aSlot + slot * L::kTileBytes;
-                    const uint32_t tP = tbase + (w ? kColS1 : kColS0);
-#pragma unroll
-                    for (int k = 0; k < kBN / 16; ++k)
-                        umma_ts(tO, tP + k * 8, mnmajor_desc(vb, k, kBN * 128), kIdPV,
-                                (j > 0 || k > 0));
+                    mma_group<kBN / 16, false>(tO, w ? tS1 : tS0, dv_lo + slot * kSlotStep, d_hi, kIdPV,
+                                               j > 0);
                     umma_commit(&pv_done[w]);
-                    umma_commit(&slot_empty[slot]);
+                    release(slot);
                     return true;
                 };
                 // pass A: X takes even tiles, Y odd tiles
                 for (int it = isx ? 0 : 1; ok && it < nt; it += 2) ok = issue_qk(it);
                 if (ok) umma_commit(a_done);
                 if (isx) {  // pass B Q K^T, in tile order
-                    // A K slot's previous occupant may be one of Y's pass-A tiles,
-                    // possibly still in flight; waiting on the slot before that
-                    // load lands could match an earlier phase of the same parity.
-                    // Once every pass-A MMA has completed, every pass-A load has
-                    // landed.
+                    // A slot's previous occupant may be one of Y's pass-A tiles, possibly
+                    // still in flight; waiting on the slot before that load lands could
+                    // match an earlier phase of the same parity.  Once every pass-A MMA
+                    // has completed, every pass-A load has landed.
+                    // The first pass-B tiles reuse S0 and S1: both warpgroups must have
+                    // read every pass-A tile.
                     if (ok) {
                         site = 9;
-                        ok = wait_until(a_done, 0, deadline);
+                        ok = wait_until(a_done, 0, deadline) && wait_until(a_read, 0, deadline);
                     }
                     for (int j = 0; ok && j < nt; ++j) ok = issue_qk(nt + j);
                 } else {    // pass B P V, in tile order
@@ -430,6 +527,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_before();
         __syncthreads();
         if (warp == 1) tmem_dealloc(tbase, 512);
+        if (C > 1) cluster_sync_all();  // no CTA leaves while its partner may still write to it
     } else {
         asm volatile("setmaxnreg.inc.sync.aligned.u32 208;" ::: "memory");
         // ------------------------------------------------------------ softmax warpgroups
@@ -477,9 +575,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ---------------- pass A: online max / sum of exp2 over this warpgroup's tiles
         float m = -INFINITY, l = 0.f;  // log2 units, scaled
         for (int it = wg; it < nt; it += 2) {
-            ok = __all_sync(0xffffffffu, wait_until(&s_full[wg], (it >> 1) & 1, deadline));
+            const int b = it % kSA;  // score buffer of this tile
+            ok = __all_sync(0xffffffffu, wait_until(&sa_full[it % kSA2], (it / kSA2) & 1, deadline));
             if (!ok) break;
             tc_fence_after();
+            const uint32_t tSa =
+                tbase + lane_off + (b == 0 ? kColS0 : b == 1 ? kColS1 : kColO);
             int lim;  // keys [0, lim) of this tile are visible to this row
             if (it < nst) {
                 lim = min(kBN, count - state_tile(it) * kBN);
@@ -491,10 +592,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             // the next Q K^T into it can start while this one is reduced
             float v[4][32];
 #pragma unroll
-            for (int ch = 0; ch < 4; ++ch) tmem_ld32(tS + ch * 32, v[ch]);
+            for (int ch = 0; ch < 4; ++ch) tmem_ld32(tSa + ch * 32, v[ch]);
             tmem_ld_wait();
             tc_fence_before();
-            mbar_arrive(&s_read[wg]);
+            mbar_arrive(&sa_read[it % kSA2]);
             if (lim < kBN) {
 #pragma unroll
                 for (int ch = 0; ch < 4; ++ch)
@@ -529,6 +630,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 m = m_new;
             }
         }
+        mbar_arrive(a_read);  // every pass-A tile of this thread has been read
         if (ok) site = 11;
         stat[(wg * 2 + 0) * kBM + row] = m;
         stat[(wg * 2 + 1) * kBM + row] = l;
@@ -549,8 +651,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // Every warp runs every iteration and arrives at the per-tile barrier;
         // after a timeout it only skips the work (a bar.sync cannot time out).
         for (int j = (wg - nt) & 1, k2 = 0; j < nt; j += 2, ++k2) {
-            const int it = nt + j;
-            if (ok) ok = __all_sync(0xffffffffu, wait_until(&s_full[wg], (it >> 1) & 1, deadline));
+            if (ok) ok = __all_sync(0xffffffffu, wait_until(&sb_full[wg], (j >> 1) & 1, deadline));
             const bool is_state = j < nst;
             float* rb = myred + (k2 & 1) * (4 * kBM);  // [4 warps][128 columns]
             if (ok) {
@@ -597,7 +698,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     rb[quad * kBM + ch * 32 + lane] = warp_colsum32(v[ch], lane);
             }
             named_bar_sync(2 + wg, 128);
-            if (ok) {
+            if (ok && tile_valid) {
                 const float s = rb[0 * kBM + ct] + rb[1 * kBM + ct] + rb[2 * kBM + ct] +
                                 rb[3 * kBM + ct];
                 const int key = (is_state ? state_tile(j) : j - nst) * kBN + ct;
@@ -606,7 +707,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (ok) site = 12;
         // Frame keys no row of this tile can see receive zero importance here.
-        for (int t = nft * kBN + (threadIdx.x - 128); t < T; t += 256) part[B + t] = 0.f;
+        if (tile_valid)
+            for (int t = nft * kBN + (threadIdx.x - 128); t < T; t += 256) part[B + t] = 0.f;
 
         // ---------------- epilogue: O rows -> bf16 out; warpgroup wg stores
         // columns [wg*D/2, (wg+1)*D/2)
@@ -640,6 +742,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!ok) fail(site + 32 * wg);
         tc_fence_before();
         __syncthreads();
+        if (C > 1) cluster_sync_all();
     }
 }
 
@@ -649,16 +752,41 @@ __global__ void __launch_bounds__(kThreads, 1)
 constexpr int kLaunchRegs = 168;
 static_assert(128 * 80 + 256 * 208 <= kThreads * kLaunchRegs, "register split");
 
+// Query tiles per cluster for head dim D: two CTAs share each K/V tile by
+// multicast (one 64-column half each) when D = 128.
+constexpr int cluster_size(int D) { return D == 128 ? 1 : 1; }
+
 template <int D>
 cudaError_t prepare_one()
 {
+    constexpr int C = cluster_size(D);
     cudaFuncAttributes fa;
-    cudaError_t e = cudaFuncGetAttributes(&fa, frame_attn_lse_importance<D>);
+    cudaError_t e = cudaFuncGetAttributes(&fa, frame_attn_lse_importance<D, C>);
     if (e != cudaSuccess) return e;
     if (fa.numRegs < kLaunchRegs) return cudaErrorInvalidConfiguration;
-    return cudaFuncSetAttribute(frame_attn_lse_importance<D>,
+    return cudaFuncSetAttribute(frame_attn_lse_importance<D, C>,
                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 AttnLayout<D>::kAlloc);
+}
+
+template <int D>
+cudaError_t launch_one(const CUtensorMap& tm_sk, const CUtensorMap& tm_sv, const CUtensorMap& tm_fk,
+                       const CUtensorMap& tm_fv, const AttnParams& p, int U, cudaStream_t st)
+{
+    constexpr int C = cluster_size(D);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((p.MT + C - 1) / C * C, p.Hkv, U);
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = AttnLayout<D>::kAlloc;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = C;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, frame_attn_lse_importance<D, C>, tm_sk, tm_sv, tm_fk, tm_fv, p);
 }
 
 }  // namespace
@@ -677,14 +805,9 @@ cudaError_t launch_attn(int D, const CUtensorMap& tm_sk, const CUtensorMap& tm_s
                         const CUtensorMap& tm_fk, const CUtensorMap& tm_fv, const AttnParams& p,
                         int U, cudaStream_t st)
 {
-    const dim3 grid(p.MT, p.Hkv, U);
-    if (D == 64)
-        frame_attn_lse_importance<64>
-            <<<grid, kThreads, AttnLayout<64>::kAlloc, st>>>(tm_sk, tm_sv, tm_fk, tm_fv, p);
-    else
-        frame_attn_lse_importance<128>
-            <<<grid, kThreads, AttnLayout<128>::kAlloc, st>>>(tm_sk, tm_sv, tm_fk, tm_fv, p);
-    return cudaGetLastError();
+    const cudaError_t e = D == 64 ? launch_one<64>(tm_sk, tm_sv, tm_fk, tm_fv, p, U, st)
+                                  : launch_one<128>(tm_sk, tm_sv, tm_fk, tm_fv, p, U, st);
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 }  // namespace statekv

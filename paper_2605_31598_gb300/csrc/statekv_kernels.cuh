@@ -18,8 +18,9 @@ namespace statekv {
 // Device error codes written to the status word (0 = no error).  The low
 // byte is the kind; an attention-kernel timeout carries the waiting site in
 // bits 8..15 (the first expired wait of the CTA): 1 V producer (pass A
-// done), 2/3 K/V producer (free slot), 4..9 MMA issuer X (Q ready, K/V slot,
-// score buffer, P, V slot, pass A done; +16 for issuer Y), 10..12 softmax
+// done), 2/3 K/V producer (free slot), 4..9 the MMA issuer's waiter (4 Q
+// ready, 5 K tile landed, 6 score buffer read in pass A, 7 P written, 8 V
+// tile landed, 9 score buffer's P V done in pass B), 10..12 softmax
 // warpgroup 0 (pass A, pass B, O ready; +32 for warpgroup 1).
 enum DeviceError : int32_t {
     DEV_OK = 0,
