@@ -53,8 +53,12 @@ using namespace ptx;
 
 constexpr int kThreads = 384;
 constexpr int kSlots = 6;        // 32 KB K/V tile slots (D = 128), one ring
-constexpr uint32_t kColS0 = 128; // TMEM columns: Q [0, D/2), S0, S1, O; pass A also
-constexpr uint32_t kColS1 = 256; // uses O's columns as a third score buffer S2
+// TMEM columns: Q [0, 64) | P [64, 128) | S0 | S1 | O; pass A also uses O's
+// columns as a third score buffer S2.  P (bf16 pairs) is one buffer shared by
+// both softmax warpgroups: P(j + 1) is written once P V(j) has read P(j).
+constexpr uint32_t kColP = 64;
+constexpr uint32_t kColS0 = 128;
+constexpr uint32_t kColS1 = 256;
 constexpr uint32_t kColO = 384;
 constexpr int kSA = 3;           // pass-A score buffers
 // Pass-A barriers are indexed by tile mod 6 (buffer tile % 3, warpgroup and
@@ -67,10 +71,10 @@ struct AttnLayout {
     static constexpr int kTileBytes = kBN * D * 2;  // one K or V tile
     static constexpr int kOffSlots = 0;
     static constexpr int kOffRed = kOffSlots + kSlots * kTileBytes;  // float[2 wg][2][4][128]
-    static constexpr int kOffStat = kOffRed + 2 * 2 * 4 * kBM * 4;   // float[2][2][128]
-    static constexpr int kOffBar = kOffStat + 4 * kBM * 4;
-    // slot_full[6] slot_empty[6] sa_full[6] sa_read[6] sb_full[2] p_full[2]
-    // pv_done[2] q_full o_full drain a_done a_read
+    static constexpr int kOffStat = kOffRed + 2 * 2 * 4 * kBM * 4;   // float[5][128]
+    static constexpr int kOffBar = kOffStat + 5 * kBM * 4;
+    // slot_full[6] slot_empty[6] sa_full[6] sa_read[6] sb_full[2] sb_read[2]
+    // p_full[2] pv_done[2] q_full o_full drain a_done a_read
     static constexpr int kNumBars = 40;
     static constexpr int kOffMisc = kOffBar + kNumBars * 8;
     static constexpr int kBytes = kOffMisc + 16;
@@ -244,21 +248,78 @@ __device__ __forceinline__ int qk_item(int nt, int it)  // it: Q K^T sequence in
     return it < nt ? it : nt + 2 * (it - nt);
 }
 
-// Column sums over the warp's 32 rows of a 32-column chunk held one row per
-// lane: a butterfly reduce-scatter; lane l returns the sum of column l.
-__device__ __forceinline__ float warp_colsum32(float (&x)[32], int lane)
+// 16 TMEM lanes x 128 columns -> 64 registers (.16x256b layout): register
+// 4r + 2k + e holds lane (base + t/4 + 8k), column 8r + 2(t%4) + e, for
+// thread t and r < 16.
+__device__ __forceinline__ void tmem_ld_16x256b_x16(uint32_t taddr, float (&v)[64])
+{
+    uint32_t r[64];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.16x256b.x16.b32"
+        " {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15,"
+        " %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31,"
+        " %32, %33, %34, %35, %36, %37, %38, %39, %40, %41, %42, %43, %44, %45, %46, %47,"
+        " %48, %49, %50, %51, %52, %53, %54, %55, %56, %57, %58, %59, %60, %61, %62, %63},"
+        " [%64];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+          "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
+          "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+          "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
+          "=r"(r[31]), "=r"(r[32]), "=r"(r[33]), "=r"(r[34]), "=r"(r[35]), "=r"(r[36]),
+          "=r"(r[37]), "=r"(r[38]), "=r"(r[39]), "=r"(r[40]), "=r"(r[41]), "=r"(r[42]),
+          "=r"(r[43]), "=r"(r[44]), "=r"(r[45]), "=r"(r[46]), "=r"(r[47]), "=r"(r[48]),
+          "=r"(r[49]), "=r"(r[50]), "=r"(r[51]), "=r"(r[52]), "=r"(r[53]), "=r"(r[54]),
+          "=r"(r[55]), "=r"(r[56]), "=r"(r[57]), "=r"(r[58]), "=r"(r[59]), "=r"(r[60]),
+          "=r"(r[61]), "=r"(r[62]), "=r"(r[63])
+        : "r"(taddr)
+        : "memory");
+#pragma unroll
+    for (int i = 0; i < 64; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// 32 registers -> 16 TMEM lanes x 64 columns (.16x128b layout): register
+// 2r + k goes to lane (base + t/4 + 8k), column 4r + t%4.
+__device__ __forceinline__ void tmem_st_16x128b_x16(uint32_t taddr, const uint32_t (&r)[32])
+{
+    asm volatile(
+        "tcgen05.st.sync.aligned.16x128b.x16.b32 [%0],"
+        " {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16,"
+        " %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};" ::"r"(
+            taddr),
+        "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+        "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),
+        "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]),
+        "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]),
+        "r"(r[29]), "r"(r[30]), "r"(r[31])
+        : "memory");
+}
+
+// Sums over the 8 lanes that share lane % 4 (lane bits 2..4) of 32 values,
+// as a reduce-scatter: lane l returns the sums of values 4 (l/4) .. +3.
+__device__ __forceinline__ void lane8_reduce_scatter(float (&x)[32], int lane, float (&out)[4])
 {
 #pragma unroll
-    for (int m = 16, n = 32; m >= 1; m >>= 1, n >>= 1) {
-        const bool up = (lane & m) != 0;
-#pragma unroll
-        for (int i = 0; i < n / 2; ++i) {
-            const float send = up ? x[i] : x[i + n / 2];
-            const float keep = up ? x[i + n / 2] : x[i];
-            x[i] = keep + __shfl_xor_sync(0xffffffffu, send, m);
-        }
+    for (int i = 0; i < 16; ++i) {
+        const bool up = (lane & 16) != 0;
+        const float send = up ? x[i] : x[i + 16];
+        const float keep = up ? x[i + 16] : x[i];
+        x[i] = keep + __shfl_xor_sync(0xffffffffu, send, 16);
     }
-    return x[0];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        const bool up = (lane & 8) != 0;
+        const float send = up ? x[i] : x[i + 8];
+        const float keep = up ? x[i + 8] : x[i];
+        x[i] = keep + __shfl_xor_sync(0xffffffffu, send, 8);
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const bool up = (lane & 4) != 0;
+        const float send = up ? x[i] : x[i + 4];
+        const float keep = up ? x[i + 4] : x[i];
+        out[i] = keep + __shfl_xor_sync(0xffffffffu, send, 4);
+    }
 }
 
 template <int D, int C>  // C: CTAs per cluster sharing K/V tiles (1 or 2)
@@ -281,13 +342,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t* sa_full = bars + 12;  // pass A: Q K^T of tile i done (index i % 6)
     uint64_t* sa_read = bars + 18;  // pass A: tile i read by its warpgroup (index i % 6)
     uint64_t* sb_full = bars + 24;  // pass B: Q K^T result in score buffer w (of 2)
-    uint64_t* p_full = bars + 26;   // pass B: warpgroup w has written P into buffer w
-    uint64_t* pv_done = bars + 28;  // pass B: the P V that read buffer w has completed
-    uint64_t* q_full = bars + 30;
-    uint64_t* o_full = bars + 31;
-    uint64_t* drain = bars + 32;
-    uint64_t* a_done = bars + 33;   // every pass-A MMA has completed
-    uint64_t* a_read = bars + 34;   // both warpgroups have read every pass-A score tile
+    uint64_t* sb_read = bars + 26;  // pass B: warpgroup w has read score buffer w
+    uint64_t* p_full = bars + 28;   // pass B: warpgroup w has written its tile's P
+    uint64_t* pv_done = bars + 30;  // pass B: P V(j) has completed (index j & 1)
+    uint64_t* q_full = bars + 32;
+    uint64_t* o_full = bars + 33;
+    uint64_t* drain = bars + 34;
+    uint64_t* a_done = bars + 35;   // every pass-A MMA has completed
+    uint64_t* a_read = bars + 36;   // both warpgroups have read every pass-A score tile
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + L::kOffMisc);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(sm + L::kOffMisc + 4);
 
@@ -327,6 +389,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(&sb_full[i], 1);
+            mbar_init(&sb_read[i], 128);
             mbar_init(&p_full[i], 128);
             mbar_init(&pv_done[i], 1);
         }
@@ -470,9 +533,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                         tS = b == 0 ? tS0 : b == 1 ? tS1 : tO;
                         done = &sa_full[it % kSA2];
                     } else {
-                        // the buffer's previous pass-B tile (j - 2) has been read by its P V
+                        // the buffer's previous pass-B tile (j - 2) has been read by its
+                        // warpgroup
                         const int j = it - nt, w = it & 1;
-                        if (j >= 2 && !wait_until(&pv_done[w], ((j - 2) >> 1) & 1, deadline)) return false;
+                        if (j >= 2 && !wait_until(&sb_read[w], ((j - 2) >> 1) & 1, deadline)) return false;
                         tS = w ? tS1 : tS0;
                         done = &sb_full[w];
                     }
@@ -492,9 +556,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                     site = 8;
                     if (!wait_until(&slot_full[slot], (item / kSlots) & 1, deadline)) return false;
                     tc_fence_after();
-                    mma_group<kBN / 16, false>(tO, w ? tS1 : tS0, dv_lo + slot * kSlotStep, d_hi, kIdPV,
+                    mma_group<kBN / 16, false>(tO, tbase + kColP, dv_lo + slot * kSlotStep, d_hi, kIdPV,
                                                j > 0);
-                    umma_commit(&pv_done[w]);
+                    umma_commit(&pv_done[j & 1]);
                     release(slot);
                     return true;
                 };
@@ -536,6 +600,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int row = quad * 32 + lane;        // TMEM lane = query row of the tile
         const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
         const uint32_t tS = tbase + lane_off + (wg ? kColS1 : kColS0);
+        const uint32_t tP = tbase + lane_off + kColP;
         const float c = p.scale_log2;
         const int my_r = mt * kBM + row;
         const bool row_valid = my_r < rows;
@@ -645,9 +710,28 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
 
         // ---------------- pass B: P = exp2(S c - lse) -> TMEM (bf16) and column sums
+        // Layout of pass B: TMEM is read in 16-lane x 256-bit groups, so a thread
+        // holds 4 rows (quadrant rows 16h + t/4 + 8k, h, k in {0, 1}) x 32 columns
+        // (8r + 2(t%4) + e); the column sums add 4 rows in registers and the 8
+        // lanes that share t % 4 by a 3-step reduce-scatter.
+        float* nl_row = stat + 4 * kBM;  // -lse of every row of the tile
+        if (wg == 0) nl_row[row] = nlse;
+        named_bar_sync(1, 256);
+        float nl4[4];       // -lse of this thread's 4 rows, index 2h + k
+        int tq4[4];         // token of each row (T for padding rows)
+#pragma unroll
+        for (int h = 0; h < 2; ++h)
+#pragma unroll
+            for (int k = 0; k < 2; ++k) {
+                const int rr = quad * 32 + 16 * h + lane / 4 + 8 * k;
+                nl4[2 * h + k] = nl_row[rr];
+                const int gr = mt * kBM + rr;
+                tq4[2 * h + k] = gr < rows ? gr / G : T;
+            }
         float* part = p.partials + ((static_cast<size_t>(u) * p.Hkv + hkv) * p.MT + mt) * p.P;
         float* myred = red + wg * (2 * 4 * kBM);
         const int ct = threadIdx.x - 128 - 128 * wg;  // 0..127 within the warpgroup
+        const int cq = 2 * (lane & 3);                // this thread's column offset in 8
         // Every warp runs every iteration and arrives at the per-tile barrier;
         // after a timeout it only skips the work (a bar.sync cannot time out).
         for (int j = (wg - nt) & 1, k2 = 0; j < nt; j += 2, ++k2) {
@@ -656,46 +740,79 @@ __global__ void __launch_bounds__(kThreads, 1)
             float* rb = myred + (k2 & 1) * (4 * kBM);  // [4 warps][128 columns]
             if (ok) {
                 tc_fence_after();
-                int lim;
+                int lim4[4];  // keys [0, lim) of this tile are visible to each row
                 if (is_state) {
-                    lim = min(kBN, count - state_tile(j) * kBN);
+                    const int lim = min(kBN, count - state_tile(j) * kBN);
+#pragma unroll
+                    for (int q4 = 0; q4 < 4; ++q4) lim4[q4] = lim;
                 } else {
                     const int f0 = (j - nst) * kBN;
-                    lim = min(kBN, (p.causal ? min(T, my_tq + 1) : T) - f0);
-                }
-                const f2 cc = pk(c, c), nl = pk(nlse, nlse);
-                float v[4][32];
 #pragma unroll
-                for (int ch = 0; ch < 4; ++ch) tmem_ld32(tS + ch * 32, v[ch]);
+                    for (int q4 = 0; q4 < 4; ++q4)
+                        lim4[q4] = min(kBN, (p.causal ? min(T, tq4[q4] + 1) : T) - f0);
+                }
+                const bool full = lim4[0] == kBN && lim4[1] == kBN && lim4[2] == kBN && lim4[3] == kBN;
+                const f2 cc = pk(c, c);
+                float v[2][64];
+#pragma unroll
+                for (int h = 0; h < 2; ++h) tmem_ld_16x256b_x16(tS + ((16u * h) << 16), v[h]);
                 tmem_ld_wait();
-#pragma unroll
-                for (int ch = 0; ch < 4; ++ch) {
-                    float (&x)[32] = v[ch];
-#pragma unroll
-                    for (int e = 0; e < 32; e += 2) {
-                        float x0, x1;
-                        upk(fma2(pk(x[e], x[e + 1]), cc, nl), x0, x1);
-                        x[e] = ex2(x0);
-                        x[e + 1] = ex2(x1);
-                    }
-                    if (lim < kBN) {
-#pragma unroll
-                        for (int e = 0; e < 32; ++e) x[e] = (ch * 32 + e < lim) ? x[e] : 0.f;
-                    }
-                    uint32_t pw[16];
-#pragma unroll
-                    for (int e = 0; e < 16; ++e) pw[e] = pack_bf16x2(x[2 * e], x[2 * e + 1]);
-                    // P chunk -> buffer columns [16 ch, 16 ch + 16) (scores of
-                    // every chunk are already in registers)
-                    tmem_st16(tS + ch * 16, pw);
-                }
-                tmem_st_wait();
                 tc_fence_before();
-                mbar_arrive(&p_full[wg]);
-                // the column sums run while the tensor core does this tile's P V
+                mbar_arrive(&sb_read[wg]);  // Q K^T of tile j + 2 may overwrite the buffer
 #pragma unroll
-                for (int ch = 0; ch < 4; ++ch)
-                    rb[quad * kBM + ch * 32 + lane] = warp_colsum32(v[ch], lane);
+                for (int h = 0; h < 2; ++h)
+#pragma unroll
+                    for (int r = 0; r < 16; ++r)
+#pragma unroll
+                        for (int k = 0; k < 2; ++k) {
+                            const int i = 4 * r + 2 * k;
+                            const float nk = nl4[2 * h + k];
+                            float x0, x1;
+                            upk(fma2(pk(v[h][i], v[h][i + 1]), cc, pk(nk, nk)), x0, x1);
+                            v[h][i] = ex2(x0);
+                            v[h][i + 1] = ex2(x1);
+                            if (!full) {
+                                const int col = 8 * r + cq, lim = lim4[2 * h + k];
+                                v[h][i] = col < lim ? v[h][i] : 0.f;
+                                v[h][i + 1] = col + 1 < lim ? v[h][i + 1] : 0.f;
+                            }
+                        }
+                // the shared P buffer is free once P V(j - 1) has read it
+                if (j >= 1)
+                    ok = __all_sync(0xffffffffu,
+                                    wait_until(&pv_done[(j - 1) & 1], ((j - 1) >> 1) & 1, deadline));
+                if (ok) {
+                    tc_fence_after();
+#pragma unroll
+                    for (int h = 0; h < 2; ++h) {
+                        uint32_t pw[32];  // register 2r + k: row k, P column 4r + t%4
+#pragma unroll
+                        for (int r = 0; r < 16; ++r)
+#pragma unroll
+                            for (int k = 0; k < 2; ++k)
+                                pw[2 * r + k] = pack_bf16x2(v[h][4 * r + 2 * k], v[h][4 * r + 2 * k + 1]);
+                        tmem_st_16x128b_x16(tP + ((16u * h) << 16), pw);
+                    }
+                    tmem_st_wait();
+                    tc_fence_before();
+                    mbar_arrive(&p_full[wg]);
+                    // the column sums run while the tensor core does this tile's P V:
+                    // value 2r + e is column 8r + cq + e summed over the thread's rows
+                    float cs[32];
+#pragma unroll
+                    for (int r = 0; r < 16; ++r) {
+                        const f2 a = add2(pk(v[0][4 * r], v[0][4 * r + 1]), pk(v[0][4 * r + 2], v[0][4 * r + 3]));
+                        const f2 b = add2(pk(v[1][4 * r], v[1][4 * r + 1]), pk(v[1][4 * r + 2], v[1][4 * r + 3]));
+                        upk(add2(a, b), cs[2 * r], cs[2 * r + 1]);
+                    }
+                    float sum4[4];
+                    lane8_reduce_scatter(cs, lane, sum4);
+                    // this lane holds values 4m .. 4m+3 (m = lane / 4): r = 2m + (i >> 1), e = i & 1
+                    const int m4 = lane >> 2;
+#pragma unroll
+                    for (int i = 0; i < 4; ++i)
+                        rb[quad * kBM + 8 * (2 * m4 + (i >> 1)) + cq + (i & 1)] = sum4[i];
+                }
             }
             named_bar_sync(2 + wg, 128);
             if (ok && tile_valid) {
