@@ -446,6 +446,99 @@ def run_e2e(args, shape, fill, seed, device, frames):
             "api": "statekv_prefill_frame_host (pinned host buffers)"}
 
 
+def run_curve(args, local):
+    """Per-frame cost against the frame index, StateKV next to exact full
+    self-attention (Sec. 4.1's comparison, App. B's protocol: given the
+    preceding cache, process one more frame).
+
+    Every frame 1..N runs statekv_prefill_frame (timed with CUDA events; the
+    frame's inputs are generated beforehand, outside the timed region).  At
+    sample frames statekv_full_attention_frame first runs on the same handle,
+    over the decode cache that the earlier frames filled, and is timed the
+    same way.  Prints one JSON line.
+    """
+    import torch
+
+    from paper_2605_31598_gb300 import StateKV, make_config
+    from paper_2605_31598_gb300.inputs import WORKLOADS, batch_qkv
+
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py needs a CUDA device (no CPU fallback exists)")
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    shape = WORKLOADS[args.workload]
+    S, L, T, B = shape.num_streams, shape.num_layers, shape.tokens_per_frame, shape.state_capacity
+    N = args.frames or shape.max_frames
+    shape = dataclasses.replace(shape, max_frames=max(N, shape.max_frames))
+    samples = sorted({n for n in (1, 2, 4, 8, 16, 32, 64, 96, 128, 192, 256, 384, 512, 640, 768,
+                                  896, 1024) if n <= N} | {N})
+    eng = StateKV(make_config(shape))
+    st = torch.cuda.current_stream()
+    out = None
+    step_ms, full_ms = [], {}
+    log(f"[curve] {args.workload}: {N} frames, full attention at {samples}")
+    for n in range(1, N + 1):
+        q, k, v = batch_qkv(shape, n, streams=range(S), layers=range(L), seed=args.seed,
+                            device=device)
+        if out is None:
+            out = torch.empty_like(q)
+        torch.cuda.synchronize()
+        if n in samples:
+            for rep in range(2):  # second run timed: code and TMA descriptors warm
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record(st)
+                rc = eng.full_attention_frame(q, k, v, out)
+                e1.record(st)
+                if rc != 0:
+                    raise RuntimeError(f"statekv_full_attention_frame returned {rc} at frame {n}")
+            torch.cuda.synchronize()
+            full_ms[n] = e0.elapsed_time(e1)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(st)
+        rc = eng.prefill_frame(q, k, v, out)
+        e1.record(st)
+        if rc != 0:
+            raise RuntimeError(f"statekv_prefill_frame returned {rc} at frame {n}")
+        torch.cuda.synchronize()
+        step_ms.append(e0.elapsed_time(e1))
+    assert eng.sync() == 0
+    fill = math.ceil(B / T) if B > 0 else 0
+    post = step_ms[fill + 1:]  # frames whose pool exceeds B
+    first = fill + 2
+    idx = list(range(first, first + len(post)))
+    m = len(post)
+    mx, my = sum(idx) / m, sum(post) / m
+    var = sum((x - mx) ** 2 for x in idx)
+    slope = sum((x - mx) * (y - my) for x, y in zip(idx, post)) / var if var > 0 else 0.0
+    p50 = lambda xs: sorted(xs)[len(xs) // 2]
+
+    def pairs(n):  # visible (query, key) pairs per query head
+        return T * (n - 1) * T + T * (T + 1) / 2
+
+    def pairs_statekv(n):
+        return T * min(B, (n - 1) * T) + T * (T + 1) / 2
+
+    line = {
+        "curve": WORKLOAD_TEXT[args.workload],
+        "frames": N,
+        "streams": S,
+        "layers": L,
+        "statekv_step_us_at": {str(n): 1e3 * step_ms[n - 1] for n in samples},
+        "full_attention_us_at": {str(n): 1e3 * full_ms[n] for n in samples},
+        "full_over_statekv_flops_at": {str(n): pairs(n) / pairs_statekv(n) for n in samples},
+        "statekv_flatness": {
+            "frames": f"{first}..{first + m - 1}",
+            "p50_first32_us": 1e3 * p50(post[:32]),
+            "p50_last_half_us": 1e3 * p50(post[m // 2:]),
+            "slope_pct_per_100_frames": 100.0 * 100.0 * slope / my if my > 0 else None,
+            "p50_all_us": 1e3 * p50(post),
+        },
+        "note": "full attention = the attention call alone (the decode-cache append it also "
+                "needs is the same as StateKV's and not included); StateKV = the whole step",
+    }
+    print(json.dumps(line), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__)
     ap.add_argument("--gpus", type=int, default=1)
@@ -459,7 +552,14 @@ def main():
     ap.add_argument("--max-frames", type=int, default=0,
                     help="decode-cache capacity in frames (default: the workload's); "
                          "a small value keeps the arena small for profiler captures")
+    ap.add_argument("--curve", action="store_true",
+                    help="per-frame cost vs frame index, StateKV next to exact full attention")
+    ap.add_argument("--frames", type=int, default=0, help="--curve: frames to run (default: "
+                    "the workload's video length)")
     args = ap.parse_args()
+    if args.curve:
+        run_curve(args, int(os.environ.get("LOCAL_RANK", 0)))
+        return
     if args.warmup < 3:
         raise SystemExit("--warmup must be at least 3")
     world, rank, local = dist_setup()

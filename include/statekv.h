@@ -111,6 +111,19 @@ typedef struct {
 statekv_status statekv_prefill_frame(statekv_handle* h, const statekv_frame_args* args,
                                      statekv_stream stream);
 
+/* Exact full self-attention of the next frame, the comparison baseline of
+ * Sec. 4.1 / App. B ("full SA"): for every query of the frame, softmax over
+ * all tokens of the frames already processed (read from the decode cache,
+ * every one visible) followed by the frame's own tokens (causal within the
+ * frame as configured), times the matching values.  Writes out only: no
+ * importance (args->importance must be NULL, else INVALID_ARG), and no change
+ * to the states, the decode cache or the frame counters, so it can be timed
+ * next to statekv_prefill_frame on the same handle ("given the preceding
+ * cache, process one more frame").  Its cost grows with the frame index;
+ * statekv_prefill_frame's does not. */
+statekv_status statekv_full_attention_frame(statekv_handle* h, const statekv_frame_args* args,
+                                           statekv_stream stream);
+
 /* Same step with HOST buffers (pinned memory recommended): q/k/v are copied
  * into the arena's staging area, the step runs, and out (and importance if
  * non-null) are copied back, all asynchronously on `stream`.  Host buffers

@@ -14,6 +14,9 @@ only compiles it with gcc and marshals numpy arrays.  What it follows:
   layer and KV head), each weight taken as exp(score - LSE) (App. B.1);
 * Sec. 3.3, Eq. 6 -- keep the top B of the pool (state + frame tokens);
 * Sec. 3.2/3.3 -- append the frame's K, V to the decode cache; L_n += T.
+* Sec. 4.1 / App. B -- the full self-attention baseline: the frame's queries
+  attend to every earlier token and to the frame (causal within it), which
+  is Eq. 5 with nothing ever evicted (``full_attention``, numpy matrix form).
 
 Readings of silent points: score ties keep the older token; a pool of at most
 B tokens is kept whole; the state is stored in ascending position.
@@ -162,3 +165,34 @@ class OracleLayer:
 
     def state_positions(self, h):
         return self.pos[h, : int(self.count[h])].copy()
+
+
+def full_attention(q_bits: np.ndarray, k_bits: np.ndarray, v_bits: np.ndarray, n_prefix: int,
+                   causal: bool = True, scale: float | None = None) -> np.ndarray:
+    """Exact softmax attention of one frame (fp64), the full-SA baseline.
+
+    q: [T][n_q][d]; k, v: [n_prefix + T][n_kv][d] bf16 bits, the earlier
+    tokens in order followed by the frame's own.  Query i of the frame sees
+    every earlier token and frame token j iff j <= i (all frame tokens when
+    not causal); query head h reads KV head h // (n_q / n_kv).  Returns O
+    [T][n_q][d] float64.
+    """
+    q = bf16_bits_to_f64(q_bits)
+    k = bf16_bits_to_f64(k_bits)
+    v = bf16_bits_to_f64(v_bits)
+    T, n_q, d = q.shape
+    n_kv = k.shape[1]
+    G = n_q // n_kv
+    sc = float(scale) if scale else 1.0 / np.sqrt(d)
+    visible = np.ones((T, n_prefix + T), dtype=bool)
+    if causal:
+        visible[:, n_prefix:] = np.tril(np.ones((T, T), dtype=bool))
+    out = np.empty((T, n_q, d))
+    for h in range(n_q):
+        s = (q[:, h, :] @ k[:, h // G, :].T) * sc
+        s = np.where(visible, s, -np.inf)
+        s -= s.max(axis=1, keepdims=True)
+        w = np.exp(s)
+        w /= w.sum(axis=1, keepdims=True)
+        out[:, h, :] = w @ v[:, h // G, :]
+    return out

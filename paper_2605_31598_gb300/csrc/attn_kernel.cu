@@ -363,7 +363,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int rows = G * T;
     const bool tile_valid = mt < p.MT;
     const int crank = C > 1 ? static_cast<int>(cluster_ctarank()) : 0;
-    const int count = (B > 0) ? p.counts[ua * p.Hkv + hkv] : 0;
+    const int count = p.count_mul * ((B > 0 || p.count_mul > 1) ? p.counts[ua * p.Hkv + hkv] : 0);
     const int nst = (count + kBN - 1) / kBN;
     // frame tiles seen by the cluster's last query tile (the union over the cluster)
     const int mt_last = min(mt - crank + C - 1, p.MT - 1);
@@ -728,7 +728,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const int gr = mt * kBM + rr;
                 tq4[2 * h + k] = gr < rows ? gr / G : T;
             }
-        float* part = p.partials + ((static_cast<size_t>(u) * p.Hkv + hkv) * p.MT + mt) * p.P;
+        float* part = p.partials ? p.partials + ((static_cast<size_t>(u) * p.Hkv + hkv) * p.MT + mt) * p.P
+                                 : nullptr;
         float* myred = red + wg * (2 * 4 * kBM);
         const int ct = threadIdx.x - 128 - 128 * wg;  // 0..127 within the warpgroup
         const int cq = 2 * (lane & 3);                // this thread's column offset in 8
@@ -815,7 +816,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             }
             named_bar_sync(2 + wg, 128);
-            if (ok && tile_valid) {
+            if (ok && tile_valid && part != nullptr) {
                 const float s = rb[0 * kBM + ct] + rb[1 * kBM + ct] + rb[2 * kBM + ct] +
                                 rb[3 * kBM + ct];
                 const int key = (is_state ? state_tile(j) : j - nst) * kBN + ct;
@@ -824,7 +825,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (ok) site = 12;
         // Frame keys no row of this tile can see receive zero importance here.
-        if (tile_valid)
+        if (tile_valid && part != nullptr)
             for (int t = nft * kBN + (threadIdx.x - 128); t < T; t += 256) part[B + t] = 0.f;
 
         // ---------------- epilogue: O rows -> bf16 out; warpgroup wg stores

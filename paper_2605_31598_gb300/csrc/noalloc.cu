@@ -191,6 +191,7 @@ extern "C" statekv_status statekv_frame_attention_noalloc(
     p.P = static_cast<int>(P);
     p.MT = MT;
     p.causal = cfg->causal_in_frame;
+    p.count_mul = 1;
     const float scale =
         cfg->softmax_scale > 0.f ? cfg->softmax_scale : 1.0f / std::sqrt(static_cast<float>(D));
     p.scale_log2 = scale * 1.4426950408889634f;

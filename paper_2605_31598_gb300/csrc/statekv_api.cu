@@ -140,7 +140,8 @@ struct statekv_handle {
     Layout lay;
     uint8_t* arena;
     std::vector<int32_t> frames_host;  // [S*L]
-    CUtensorMap tm_sk, tm_sv;
+    CUtensorMap tm_sk, tm_sv;  // state rows, [S*L][Hkv][B][D]
+    CUtensorMap tm_ck, tm_cv;  // decode-cache rows, [S*L][Hkv][cap][D]
     volatile int32_t* status_host;
     int32_t* status_dev;
     bool prof_on;
@@ -250,6 +251,7 @@ statekv_status run_step(statekv_handle* h, const statekv_frame_args& a, cudaStre
     pa.P = d.P;
     pa.MT = d.MT;
     pa.causal = c.causal_in_frame;
+    pa.count_mul = 1;
     pa.scale_log2 = d.scale * 1.4426950408889634f;
     pa.watchdog_ns = 1000000ull * (c.watchdog_ms ? c.watchdog_ms : 2000u);
     if (timed(h, 1, st, [&] { return launch_attn(D, h->tm_sk, h->tm_sv, tm_fk, tm_fv, pa, U, st); }) !=
@@ -280,6 +282,52 @@ statekv_status run_step(statekv_handle* h, const statekv_frame_args& a, cudaStre
     for (int s = a.stream_begin; s < a.stream_begin + a.stream_count; ++s)
         for (int l = a.layer_begin; l < a.layer_begin + a.layer_count; ++l)
             ++h->frames_host[static_cast<size_t>(s) * c.num_layers + l];
+    return STATEKV_OK;
+}
+
+// Exact full self-attention of the frame over every token of the decode cache
+// (the frames processed so far, all visible) followed by the frame's own
+// tokens (causal as configured): the attention kernel with the cache as its
+// key prefix, no importance, no change to any state.
+statekv_status run_full(statekv_handle* h, const statekv_frame_args& a, cudaStream_t st)
+{
+    const statekv_config& c = h->cfg;
+    const Derived& d = h->d;
+    const int U = a.stream_count * a.layer_count;
+    const int D = c.head_dim, T = c.tokens_per_frame, Hkv = c.num_kv_heads;
+    CUtensorMap tm_fk, tm_fv;
+    {
+        const cuuint64_t dims[4] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(Hkv),
+                                    static_cast<cuuint64_t>(T), static_cast<cuuint64_t>(U)};
+        const cuuint64_t strides[3] = {static_cast<cuuint64_t>(D) * 2,
+                                       static_cast<cuuint64_t>(Hkv) * D * 2,
+                                       static_cast<cuuint64_t>(T) * Hkv * D * 2};
+        const cuuint32_t box[4] = {64, 1, static_cast<cuuint32_t>(kBN), 1};
+        if (!encode_4d(&tm_fk, a.k, dims, strides, box) ||
+            !encode_4d(&tm_fv, a.v, dims, strides, box))
+            return STATEKV_ERR_CUDA;
+    }
+    AttnParams pa{};
+    pa.q = static_cast<const __nv_bfloat16*>(a.q);
+    pa.out = static_cast<__nv_bfloat16*>(a.out);
+    pa.partials = nullptr;
+    pa.counts = h->at<int32_t>(h->lay.frames);  // frames so far; keys = frames * T
+    pa.status = h->status_dev;
+    pa.units = UnitRange{a.stream_begin, a.layer_begin, a.layer_count, c.num_layers};
+    pa.T = T;
+    pa.Hq = c.num_q_heads;
+    pa.Hkv = Hkv;
+    pa.G = d.G;
+    pa.B = 1;  // no importance pool
+    pa.P = 0;
+    pa.MT = d.MT;
+    pa.causal = c.causal_in_frame;
+    pa.count_mul = T;
+    pa.scale_log2 = d.scale * 1.4426950408889634f;
+    pa.watchdog_ns = 1000000ull * (c.watchdog_ms ? c.watchdog_ms : 2000u);
+    if (timed(h, 1, st, [&] { return launch_attn(D, h->tm_ck, h->tm_cv, tm_fk, tm_fv, pa, U, st); }) !=
+        cudaSuccess)
+        return STATEKV_ERR_CUDA;
     return STATEKV_OK;
 }
 
@@ -319,6 +367,8 @@ statekv_status statekv_init(const statekv_config* cfg, void* device_arena, size_
     h->prof_used = 0;
     std::memset(&h->tm_sk, 0, sizeof(CUtensorMap));
     std::memset(&h->tm_sv, 0, sizeof(CUtensorMap));
+    std::memset(&h->tm_ck, 0, sizeof(CUtensorMap));
+    std::memset(&h->tm_cv, 0, sizeof(CUtensorMap));
 
     void* st_host = nullptr;
     if (cudaHostAlloc(&st_host, 64, cudaHostAllocMapped) != cudaSuccess) {
@@ -347,6 +397,16 @@ statekv_status statekv_init(const statekv_config* cfg, void* device_arena, size_
         ok = encode_4d(&h->tm_sk, h->arena + lay.state_k, dims, strides, box) &&
              encode_4d(&h->tm_sv, h->arena + lay.state_v, dims, strides, box);
     }
+    if (ok) {
+        const cuuint64_t dims[4] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(d.cap),
+                                    static_cast<cuuint64_t>(Hkv), static_cast<cuuint64_t>(d.SL)};
+        const cuuint64_t strides[3] = {static_cast<cuuint64_t>(D) * 2,
+                                       static_cast<cuuint64_t>(d.cap) * D * 2,
+                                       static_cast<cuuint64_t>(Hkv) * d.cap * D * 2};
+        const cuuint32_t box[4] = {64, static_cast<cuuint32_t>(kBN), 1, 1};
+        ok = encode_4d(&h->tm_ck, h->arena + lay.cache_k, dims, strides, box) &&
+             encode_4d(&h->tm_cv, h->arena + lay.cache_v, dims, strides, box);
+    }
     // Empty states: zero rows (masked keys must still be finite), positions -1.
     ok = ok && cudaMemset(h->arena + lay.state_k, 0, lay.positions - lay.state_k) == cudaSuccess &&
          cudaMemset(h->arena + lay.positions, 0xFF, lay.counts - lay.positions) == cudaSuccess &&
@@ -367,6 +427,15 @@ statekv_status statekv_prefill_frame(statekv_handle* h, const statekv_frame_args
     const statekv_status s = check_args(h, args, false);
     if (s != STATEKV_OK) return s;
     return run_step(h, *args, reinterpret_cast<cudaStream_t>(stream));
+}
+
+statekv_status statekv_full_attention_frame(statekv_handle* h, const statekv_frame_args* args,
+                                           statekv_stream stream)
+{
+    const statekv_status s = check_args(h, args, false);
+    if (s != STATEKV_OK) return s;
+    if (args->importance) return STATEKV_ERR_INVALID_ARG;
+    return run_full(h, *args, reinterpret_cast<cudaStream_t>(stream));
 }
 
 statekv_status statekv_prefill_frame_host(statekv_handle* h, const statekv_frame_args* args,

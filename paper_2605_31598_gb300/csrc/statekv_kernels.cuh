@@ -43,12 +43,13 @@ struct UnitRange {
 struct AttnParams {
     const __nv_bfloat16* q;   // [U][T][Hq][D]
     __nv_bfloat16* out;       // [U][T][Hq][D]
-    float* partials;          // [U][Hkv][MT][P]
-    const int32_t* counts;    // arena [S*L][Hkv]
+    float* partials;          // [U][Hkv][MT][P]; null: no importance (full attention)
+    const int32_t* counts;    // arena [S*L][Hkv]: visible keys before the frame = counts * count_mul
     int32_t* status;          // device-visible status word
     UnitRange units;
     int T, Hq, Hkv, G, B, P, MT;
     int causal;
+    int count_mul;            // 1: counts are state sizes; T: counts are frame counters
     float scale_log2;         // softmax scale * log2(e)
     unsigned long long watchdog_ns;
 };

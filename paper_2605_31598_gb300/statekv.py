@@ -22,7 +22,8 @@ STATUS_NAMES = {
     6: "STATEKV_ERR_ARENA_TOO_SMALL", 7: "STATEKV_ERR_DEVICE_FAULT",
 }
 EXPORTED = ("statekv_arena_bytes", "statekv_init", "statekv_prefill_frame",
-            "statekv_prefill_frame_host", "statekv_state_view", "statekv_cache_view",
+            "statekv_prefill_frame_host", "statekv_full_attention_frame",
+            "statekv_state_view", "statekv_cache_view",
             "statekv_profile_enable", "statekv_profile_read", "statekv_sync",
             "statekv_device_error", "statekv_frame_attention_noalloc",
             "statekv_destroy", "statekv_status_string")
@@ -80,7 +81,8 @@ def lib() -> ctypes.CDLL:
             L.statekv_init.argtypes = [P(statekv_config), ctypes.c_void_p, ctypes.c_size_t,
                                        P(ctypes.c_void_p)]
             L.statekv_init.restype = st
-            for name in ("statekv_prefill_frame", "statekv_prefill_frame_host"):
+            for name in ("statekv_prefill_frame", "statekv_prefill_frame_host",
+                         "statekv_full_attention_frame"):
                 fn = getattr(L, name)
                 fn.argtypes = [ctypes.c_void_p, P(statekv_frame_args), ctypes.c_void_p]
                 fn.restype = st
@@ -143,6 +145,10 @@ def statekv_prefill_frame(handle: int, args: statekv_frame_args, stream: int) ->
 
 def statekv_prefill_frame_host(handle: int, args: statekv_frame_args, stream: int) -> int:
     return lib().statekv_prefill_frame_host(handle, ctypes.byref(args), ctypes.c_void_p(stream))
+
+
+def statekv_full_attention_frame(handle: int, args: statekv_frame_args, stream: int) -> int:
+    return lib().statekv_full_attention_frame(handle, ctypes.byref(args), ctypes.c_void_p(stream))
 
 
 def statekv_state_view(handle: int, stream: int, layer: int) -> statekv_state_info:
@@ -248,6 +254,18 @@ class StateKV:
         st = (stream or torch.cuda.current_stream()).cuda_stream
         args = self._args(q, k, v, out, importance, stream_begin, sc, layer_begin, lc)
         return statekv_prefill_frame(self.handle, args, st)
+
+    def full_attention_frame(self, q, k, v, out, *, stream_begin=0, stream_count=None,
+                             layer_begin=0, layer_count=None, stream=None) -> int:
+        """Exact full self-attention of the next frame over the whole decode
+        cache (the comparison baseline); changes no state.  Returns the C status."""
+        import torch
+
+        sc = self.cfg.num_streams - stream_begin if stream_count is None else stream_count
+        lc = self.cfg.num_layers - layer_begin if layer_count is None else layer_count
+        st = (stream or torch.cuda.current_stream()).cuda_stream
+        args = self._args(q, k, v, out, None, stream_begin, sc, layer_begin, lc)
+        return statekv_full_attention_frame(self.handle, args, st)
 
     def prefill_frame_host(self, q, k, v, out, importance=None, *, stream_begin=0,
                            stream_count=None, layer_begin=0, layer_count=None,

@@ -128,6 +128,21 @@ def test_full_attention_when_capacity_covers_stream(causal):
         assert list(lay.state_positions(h)) == list(range(N * T))
 
 
+@pytest.mark.parametrize("causal", [True, False])
+def test_full_attention_function_matches_uncompressed_stream(causal):
+    """oracle.full_attention (numpy matrix form) against the C loops of the
+    stream whose state never evicts: the same exact attention two ways."""
+    import oracle
+
+    n_q, n_kv, d, T, N = 6, 2, 16, 5, 4
+    lay, frames = _run_stream(n_q, n_kv, d, T, B=N * T, N=N, seed=3, causal=causal)
+    for n, f in enumerate(frames):
+        ks = np.concatenate([fr["k"] for fr in frames[: n + 1]])
+        vs = np.concatenate([fr["v"] for fr in frames[: n + 1]])
+        o = oracle.full_attention(f["q"], ks, vs, n * T, causal=causal)
+        np.testing.assert_allclose(o, f["out"], rtol=1e-11, atol=1e-12)
+
+
 def test_attention_over_selected_state_matches_library():
     """B < N*T: each frame's output is attention over exactly the pre-frame
     state's keys (looked up by position in the full stream) followed by the
