@@ -378,6 +378,21 @@ __global__ void __launch_bounds__(kThreads, 1)
     auto state_tile = [&](int t) { return t + rot < nst ? t + rot : t + rot - nst; };
     const unsigned long long deadline = globaltimer() + p.watchdog_ns;
 
+    // The softmax threads start loading their Q row now, so its global-memory
+    // latency overlaps the barrier and TMEM setup (thread 128 + i: warpgroup
+    // i / 128 - 1, row i % 128; warpgroup wg holds d in [64 wg, 64 wg + 64)).
+    uint4 qreg[8];
+    {
+        const int tq = static_cast<int>(threadIdx.x) - 128;
+        const int qwg = tq >> 7, qrow = tq & 127, qr = mt * kBM + qrow;
+        const bool loads = tq >= 0 && qwg * 64 < D && qr < rows;
+        const int t = loads ? qr / G : 0, g = loads ? qr - t * G : 0;
+        const uint4* src = reinterpret_cast<const uint4*>(
+            p.q + ((static_cast<size_t>(u) * T + t) * p.Hq + hkv * G + g) * D + (loads ? qwg * 64 : 0));
+#pragma unroll
+        for (int i = 0; i < 8; ++i) qreg[i] = loads ? src[i] : make_uint4(0u, 0u, 0u, 0u);
+    }
+
     if (threadIdx.x == 0) {
         for (int i = 0; i < kSlots; ++i) {
             mbar_init(&slot_full[i], 1);
@@ -609,22 +624,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         {   // Q row -> TMEM columns [0, D/2) (bf16 pairs); warpgroup wg stores
             // d in [64 wg, 64 wg + 64) when D = 128, warpgroup 0 all of D = 64.
             if (wg * 64 < D) {
-                uint32_t w32[32];
-                if (row_valid) {
-                    const int t = my_r / G, g = my_r - t * G;
-                    const uint4* src = reinterpret_cast<const uint4*>(
-                        p.q + ((static_cast<size_t>(u) * T + t) * p.Hq + hkv * G + g) * D + wg * 64);
+                uint32_t w32[32];  // the row loaded at kernel entry
 #pragma unroll
-                    for (int i = 0; i < 8; ++i) {
-                        const uint4 x = src[i];
-                        w32[4 * i] = x.x;
-                        w32[4 * i + 1] = x.y;
-                        w32[4 * i + 2] = x.z;
-                        w32[4 * i + 3] = x.w;
-                    }
-                } else {
-#pragma unroll
-                    for (int i = 0; i < 32; ++i) w32[i] = 0u;
+                for (int i = 0; i < 8; ++i) {
+                    w32[4 * i] = qreg[i].x;
+                    w32[4 * i + 1] = qreg[i].y;
+                    w32[4 * i + 2] = qreg[i].z;
+                    w32[4 * i + 3] = qreg[i].w;
                 }
                 tmem_st16(tbase + lane_off + wg * 32, *reinterpret_cast<uint32_t(*)[16]>(&w32[0]));
                 tmem_st16(tbase + lane_off + wg * 32 + 16,
