@@ -54,8 +54,11 @@ using namespace ptx;
 constexpr int kThreads = 384;
 constexpr int kSlots = 6;        // 32 KB K/V tile slots (D = 128), one ring
 // TMEM columns: Q [0, 64) | P [64, 128) | S0 | S1 | O; pass A also uses O's
-// columns as a third score buffer S2.  P (bf16 pairs) is one buffer shared by
-// both softmax warpgroups: P(j + 1) is written once P V(j) has read P(j).
+// columns as a third score buffer S2.  In pass B warpgroup 0 writes its P
+// (bf16 pairs) into the P buffer, so Q K^T can refill S0 as soon as the
+// scores are read; warpgroup 1 writes P over the first 64 columns of S1, so
+// Q K^T into S1 waits for the P V that reads it.  (TMEM has no room for a
+// second P buffer next to Q, two score buffers and O.)
 constexpr uint32_t kColP = 64;
 constexpr uint32_t kColS0 = 128;
 constexpr uint32_t kColS1 = 256;
@@ -548,10 +551,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                         tS = b == 0 ? tS0 : b == 1 ? tS1 : tO;
                         done = &sa_full[it % kSA2];
                     } else {
-                        // the buffer's previous pass-B tile (j - 2) has been read by its
-                        // warpgroup
+                        // the buffer's previous pass-B tile (j - 2) is consumed: read by
+                        // warpgroup 0 (whose P has its own buffer), or, for warpgroup
+                        // 1 (whose P overwrites its scores), read by its P V
                         const int j = it - nt, w = it & 1;
-                        if (j >= 2 && !wait_until(&sb_read[w], ((j - 2) >> 1) & 1, deadline)) return false;
+                        if (j >= 2 && !(w == 0 ? wait_until(&sb_read[0], ((j - 2) >> 1) & 1, deadline)
+                                               : wait_until(&pv_done[j & 1], ((j - 2) >> 1) & 1, deadline)))
+                            return false;
                         tS = w ? tS1 : tS0;
                         done = &sb_full[w];
                     }
@@ -571,7 +577,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     site = 8;
                     if (!wait_until(&slot_full[slot], (item / kSlots) & 1, deadline)) return false;
                     tc_fence_after();
-                    mma_group<kBN / 16, false>(tO, tbase + kColP, dv_lo + slot * kSlotStep, d_hi, kIdPV,
+                    mma_group<kBN / 16, false>(tO, w ? tS1 : tbase + kColP, dv_lo + slot * kSlotStep, d_hi, kIdPV,
                                                j > 0);
                     umma_commit(&pv_done[j & 1]);
                     release(slot);
@@ -784,10 +790,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 v[h][i + 1] = col + 1 < lim ? v[h][i + 1] : 0.f;
                             }
                         }
-                // the shared P buffer is free once P V(j - 1) has read it
-                if (j >= 1)
+                // Warpgroup 0 writes P into the P buffer, free once its previous
+                // tile's P V (j - 2) has read it; warpgroup 1 writes P over the
+                // scores it has just read (the next Q K^T into that buffer waits for
+                // this tile's P V).
+                if (wg == 0 && j >= 2)
                     ok = __all_sync(0xffffffffu,
-                                    wait_until(&pv_done[(j - 1) & 1], ((j - 1) >> 1) & 1, deadline));
+                                    wait_until(&pv_done[j & 1], ((j - 2) >> 1) & 1, deadline));
                 if (ok) {
                     tc_fence_after();
 #pragma unroll
@@ -798,7 +807,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                             for (int k = 0; k < 2; ++k)
                                 pw[2 * r + k] = pack_bf16x2(v[h][4 * r + 2 * k], v[h][4 * r + 2 * k + 1]);
-                        tmem_st_16x128b_x16(tP + ((16u * h) << 16), pw);
+                        tmem_st_16x128b_x16((wg == 0 ? tP : tS) + ((16u * h) << 16), pw);
                     }
                     tmem_st_wait();
                     tc_fence_before();
