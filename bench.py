@@ -566,6 +566,78 @@ def run_curve(args, local):
     print(json.dumps(line), flush=True)
 
 
+def run_decode(args, local):
+    """Decoding over the detailed cache after a prefilled video: one prompt of
+    ``--prompt`` tokens, then single-token steps, each timed with CUDA events.
+    The video's frames run first (untimed).  Prints one JSON line."""
+    import torch
+
+    from paper_2605_31598_gb300 import StateKV, make_config
+    from paper_2605_31598_gb300.inputs import WORKLOADS, batch_qkv
+
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py needs a CUDA device (no CPU fallback exists)")
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    base = WORKLOADS[args.workload]
+    N = args.frames or base.max_frames
+    T, d = base.tokens_per_frame, base.head_dim
+    steps = max(3, args.steps)
+    extra = -(-(args.prompt + steps + 3) // T)
+    shape = dataclasses.replace(base, max_frames=N + extra)
+    S, L, Hq, Hkv = shape.num_streams, shape.num_layers, shape.num_q_heads, shape.num_kv_heads
+    eng = StateKV(make_config(shape))
+    out = None
+    for n in range(1, N + 1):
+        q, k, v = batch_qkv(shape, n, streams=range(S), layers=range(L), seed=args.seed,
+                            device=device)
+        out = out if out is not None else torch.empty_like(q)
+        if eng.prefill_frame(q, k, v, out) != 0:
+            raise RuntimeError(f"prefill failed at frame {n}")
+    gen = torch.Generator(device="cpu").manual_seed(args.seed + 7)
+
+    def tokens(n):
+        mk = lambda h: (torch.randn((S, L, n, h, d), generator=gen) * d ** -0.5).to(
+            torch.bfloat16).to(device)
+        return mk(Hq), mk(Hkv), mk(Hkv)
+
+    st = torch.cuda.current_stream()
+
+    def timed(n):
+        q, k, v = tokens(n)
+        o = torch.empty_like(q)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(st)
+        rc = eng.decode_step(q, k, v, o)
+        e1.record(st)
+        if rc != 0:
+            raise RuntimeError(f"statekv_decode_step returned {rc}")
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1)
+
+    prompt_ms = timed(args.prompt)
+    for _ in range(3):  # warm-up single-token steps
+        timed(1)
+    tok_ms = sorted(timed(1) for _ in range(steps))
+    assert eng.sync() == 0
+    rows = N * T + args.prompt + 3 + steps // 2
+    cache_bytes = S * L * Hkv * rows * d * 2 * 2  # K and V read once per token
+    p50 = tok_ms[len(tok_ms) // 2]
+    line = {
+        "decode": WORKLOAD_TEXT[args.workload],
+        "video_frames": N,
+        "cache_rows_per_head": rows,
+        "prompt_tokens": args.prompt,
+        "prompt_us": 1e3 * prompt_ms,
+        "token_p50_us": 1e3 * p50,
+        "tokens_per_s": 1e3 / p50,
+        "kv_read_gbs_at_p50": cache_bytes / (p50 * 1e-3) / 1e9,
+        "note": "one call = every (stream, layer); the attention kernel reads K twice (two passes)",
+    }
+    print(json.dumps(line), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__)
     ap.add_argument("--gpus", type=int, default=1)
@@ -583,7 +655,13 @@ def main():
                     help="per-frame cost vs frame index, StateKV next to exact full attention")
     ap.add_argument("--frames", type=int, default=0, help="--curve: frames to run (default: "
                     "the workload's video length)")
+    ap.add_argument("--decode", action="store_true",
+                    help="decoding over the detailed cache after --frames video frames")
+    ap.add_argument("--prompt", type=int, default=64, help="--decode: prompt tokens")
     args = ap.parse_args()
+    if args.decode:
+        run_decode(args, int(os.environ.get("LOCAL_RANK", 0)))
+        return
     if args.curve:
         run_curve(args, int(os.environ.get("LOCAL_RANK", 0)))
         return

@@ -124,6 +124,31 @@ statekv_status statekv_prefill_frame(statekv_handle* h, const statekv_frame_args
 statekv_status statekv_full_attention_frame(statekv_handle* h, const statekv_frame_args* args,
                                            statekv_stream stream);
 
+/* Decoding over the detailed cache D_N (Sec. 3.2 / 3.3: decoding reads only
+ * the detailed state; the compressed state is not used).  For every covered
+ * (stream, layer), the num_tokens new tokens (a prompt, or one generated
+ * token per call) attend to every row of the decode cache -- all video
+ * frames processed so far, then the tokens of earlier decode calls -- and
+ * causally to each other; afterwards their K/V rows are appended to the
+ * cache.  q: bf16 [S_cnt][L_cnt][num_tokens][Hq][d]; k, v: bf16
+ * [S_cnt][L_cnt][num_tokens][Hkv][d]; out: bf16 like q (all device, 16-byte
+ * aligned).  Once a (stream, layer) has decoded tokens, statekv_prefill_frame
+ * refuses it (INVALID_ARG): the video part is closed.  Returns CACHE_FULL if
+ * the cache (max_frames * T rows per head) cannot take the new rows.
+ * num_tokens must lie in [1, 4096]. */
+typedef struct {
+    int32_t stream_begin, stream_count;
+    int32_t layer_begin, layer_count;
+    int32_t num_tokens;
+    const void* q;
+    const void* k;
+    const void* v;
+    void* out;
+} statekv_decode_args;
+
+statekv_status statekv_decode_step(statekv_handle* h, const statekv_decode_args* args,
+                                   statekv_stream stream);
+
 /* Same step with HOST buffers (pinned memory recommended): q/k/v are copied
  * into the arena's staging area, the step runs, and out (and importance if
  * non-null) are copied back, all asynchronously on `stream`.  Host buffers
@@ -143,7 +168,7 @@ typedef struct {
 typedef struct {
     const void* k;            /* bf16 [Hkv][capacity][d] (device) */
     const void* v;
-    int64_t length;           /* rows written: frames * T */
+    int64_t length;           /* rows written: frames * T + decoded tokens */
     int64_t capacity;         /* max_frames * T */
 } statekv_cache_info;
 

@@ -366,7 +366,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int rows = G * T;
     const bool tile_valid = mt < p.MT;
     const int crank = C > 1 ? static_cast<int>(cluster_ctarank()) : 0;
-    const int count = p.count_mul * ((B > 0 || p.count_mul > 1) ? p.counts[ua * p.Hkv + hkv] : 0);
+    const int count = p.count_mul * ((B > 0 || p.count_mul > 1) ? p.counts[ua * p.Hkv + hkv] : 0) +
+                      (p.count_add ? p.count_add[ua * p.Hkv + hkv] : 0);
     const int nst = (count + kBN - 1) / kBN;
     // frame tiles seen by the cluster's last query tile (the union over the cluster)
     const int mt_last = min(mt - crank + C - 1, p.MT - 1);

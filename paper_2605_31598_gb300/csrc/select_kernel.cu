@@ -222,7 +222,8 @@ __global__ void __launch_bounds__(256) decode_cache_append(const AppendParams p)
         const int ch = static_cast<int>(rr % chunks);
         const int ua = p.units.unit_abs(u);
         const size_t head = static_cast<size_t>(ua) * p.Hkv + hkv;
-        const long long row = static_cast<long long>(p.frames[head]) * p.T + t;
+        const long long row = static_cast<long long>(p.frames[head]) * p.row_mul +
+                              (p.row_add ? p.row_add[head] : 0) + t;
         const __nv_bfloat16* src = (which ? p.v : p.k) + static_cast<size_t>(u) * per_unit * 8 +
                                    static_cast<size_t>(rr) * 8;
         __nv_bfloat16* dst = (which ? p.cache_v : p.cache_k) +
@@ -248,6 +249,20 @@ cudaError_t launch_select(const SelectParams& p, int U, cudaStream_t st)
 {
     const dim3 grid(p.Hkv, U);
     state_select_gather<<<grid, kSelThreads, select_smem_bytes(p.P, p.T), st>>>(p);
+    return cudaGetLastError();
+}
+
+__global__ void advance_counter(int32_t* counter, UnitRange units, int U, int Hkv, int n)
+{
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= U * Hkv) return;
+    counter[static_cast<size_t>(units.unit_abs(i / Hkv)) * Hkv + i % Hkv] += n;
+}
+
+cudaError_t launch_advance(int32_t* counter, UnitRange units, int U, int Hkv, int n,
+                           cudaStream_t st)
+{
+    advance_counter<<<(U * Hkv + 255) / 256, 256, 0, st>>>(counter, units, U, Hkv, n);
     return cudaGetLastError();
 }
 

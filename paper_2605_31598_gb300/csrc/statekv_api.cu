@@ -27,7 +27,7 @@ constexpr int kProfPairs = 3 * 4096;
 size_t round_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
 struct Layout {
-    size_t state_k, state_v, positions, counts, frames, cache_k, cache_v, partials;
+    size_t state_k, state_v, positions, counts, frames, text, cache_k, cache_v, partials;
     size_t stg_q, stg_k, stg_v, stg_out, stg_imp;
     size_t total;
 };
@@ -82,6 +82,7 @@ Layout make_layout(const statekv_config& c, const Derived& d)
     L.positions = take(heads * B * 4);
     L.counts = take(heads * 4);
     L.frames = take(heads * 4);
+    L.text = take(heads * 4);  // decode-cache rows appended after the video frames
     L.cache_k = take(heads * static_cast<size_t>(d.cap) * D * 2);
     L.cache_v = take(heads * static_cast<size_t>(d.cap) * D * 2);
     L.partials = take(heads * d.MT * static_cast<size_t>(d.P) * 4);
@@ -140,6 +141,7 @@ struct statekv_handle {
     Layout lay;
     uint8_t* arena;
     std::vector<int32_t> frames_host;  // [S*L]
+    std::vector<int32_t> text_host;    // [S*L]: tokens appended by statekv_decode_step
     CUtensorMap tm_sk, tm_sv;  // state rows, [S*L][Hkv][B][D]
     CUtensorMap tm_ck, tm_cv;  // decode-cache rows, [S*L][Hkv][cap][D]
     volatile int32_t* status_host;
@@ -177,9 +179,11 @@ statekv_status check_args(const statekv_handle* h, const statekv_frame_args* a, 
     if (host && !c.host_staging) return STATEKV_ERR_INVALID_ARG;
     if (*h->status_host != 0) return device_status(*h->status_host);
     for (int s = a->stream_begin; s < a->stream_begin + a->stream_count; ++s)
-        for (int l = a->layer_begin; l < a->layer_begin + a->layer_count; ++l)
-            if (h->frames_host[static_cast<size_t>(s) * c.num_layers + l] >= c.max_frames)
-                return STATEKV_ERR_CACHE_FULL;
+        for (int l = a->layer_begin; l < a->layer_begin + a->layer_count; ++l) {
+            const size_t unit = static_cast<size_t>(s) * c.num_layers + l;
+            if (h->text_host[unit] > 0) return STATEKV_ERR_INVALID_ARG;  // video closed
+            if (h->frames_host[unit] >= c.max_frames) return STATEKV_ERR_CACHE_FULL;
+        }
     return STATEKV_OK;
 }
 
@@ -232,6 +236,7 @@ statekv_status run_step(statekv_handle* h, const statekv_frame_args& a, cudaStre
     ap.T = T;
     ap.Hkv = Hkv;
     ap.D = D;
+    ap.row_mul = T;
     ap.cap = d.cap;
     if (timed(h, 0, st, [&] { return launch_append(ap, st); }) != cudaSuccess)
         return STATEKV_ERR_CUDA;
@@ -311,7 +316,8 @@ statekv_status run_full(statekv_handle* h, const statekv_frame_args& a, cudaStre
     pa.q = static_cast<const __nv_bfloat16*>(a.q);
     pa.out = static_cast<__nv_bfloat16*>(a.out);
     pa.partials = nullptr;
-    pa.counts = h->at<int32_t>(h->lay.frames);  // frames so far; keys = frames * T
+    pa.counts = h->at<int32_t>(h->lay.frames);  // keys = frames * T + text rows
+    pa.count_add = h->at<int32_t>(h->lay.text);
     pa.status = h->status_dev;
     pa.units = UnitRange{a.stream_begin, a.layer_begin, a.layer_count, c.num_layers};
     pa.T = T;
@@ -328,6 +334,75 @@ statekv_status run_full(statekv_handle* h, const statekv_frame_args& a, cudaStre
     if (timed(h, 1, st, [&] { return launch_attn(D, h->tm_ck, h->tm_cv, tm_fk, tm_fv, pa, U, st); }) !=
         cudaSuccess)
         return STATEKV_ERR_CUDA;
+    return STATEKV_OK;
+}
+
+// Decoding over the detailed cache: n new tokens per (stream, layer) attend to
+// every row of the decode cache (video frames, then earlier decoded tokens)
+// and causally to each other; their K/V rows are then appended to the cache.
+statekv_status run_decode(statekv_handle* h, const statekv_decode_args& a, cudaStream_t st)
+{
+    const statekv_config& c = h->cfg;
+    const Derived& d = h->d;
+    const int U = a.stream_count * a.layer_count;
+    const int D = c.head_dim, T = c.tokens_per_frame, Hkv = c.num_kv_heads, n = a.num_tokens;
+    const UnitRange ur{a.stream_begin, a.layer_begin, a.layer_count, c.num_layers};
+    CUtensorMap tm_nk, tm_nv;
+    {
+        const cuuint64_t dims[4] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(Hkv),
+                                    static_cast<cuuint64_t>(n), static_cast<cuuint64_t>(U)};
+        const cuuint64_t strides[3] = {static_cast<cuuint64_t>(D) * 2,
+                                       static_cast<cuuint64_t>(Hkv) * D * 2,
+                                       static_cast<cuuint64_t>(n) * Hkv * D * 2};
+        const cuuint32_t box[4] = {64, 1, static_cast<cuuint32_t>(kBN), 1};
+        if (!encode_4d(&tm_nk, a.k, dims, strides, box) ||
+            !encode_4d(&tm_nv, a.v, dims, strides, box))
+            return STATEKV_ERR_CUDA;
+    }
+    int32_t* frames = h->at<int32_t>(h->lay.frames);
+    int32_t* text = h->at<int32_t>(h->lay.text);
+    AttnParams pa{};
+    pa.q = static_cast<const __nv_bfloat16*>(a.q);
+    pa.out = static_cast<__nv_bfloat16*>(a.out);
+    pa.partials = nullptr;
+    pa.counts = frames;
+    pa.count_add = text;
+    pa.status = h->status_dev;
+    pa.units = ur;
+    pa.T = n;
+    pa.Hq = c.num_q_heads;
+    pa.Hkv = Hkv;
+    pa.G = d.G;
+    pa.B = 1;  // no importance pool
+    pa.P = 0;
+    pa.MT = static_cast<int>((static_cast<long long>(d.G) * n + kBM - 1) / kBM);
+    pa.causal = 1;
+    pa.count_mul = T;
+    pa.scale_log2 = d.scale * 1.4426950408889634f;
+    pa.watchdog_ns = 1000000ull * (c.watchdog_ms ? c.watchdog_ms : 2000u);
+    if (timed(h, 1, st, [&] { return launch_attn(D, h->tm_ck, h->tm_cv, tm_nk, tm_nv, pa, U, st); }) !=
+        cudaSuccess)
+        return STATEKV_ERR_CUDA;
+    AppendParams ap{};
+    ap.k = static_cast<const __nv_bfloat16*>(a.k);
+    ap.v = static_cast<const __nv_bfloat16*>(a.v);
+    ap.cache_k = h->at<__nv_bfloat16>(h->lay.cache_k);
+    ap.cache_v = h->at<__nv_bfloat16>(h->lay.cache_v);
+    ap.frames = frames;
+    ap.row_add = text;
+    ap.units = ur;
+    ap.U = U;
+    ap.T = n;
+    ap.Hkv = Hkv;
+    ap.D = D;
+    ap.row_mul = T;
+    ap.cap = d.cap;
+    if (timed(h, 0, st, [&] { return launch_append(ap, st); }) != cudaSuccess ||
+        launch_advance(text, ur, U, Hkv, n, st) != cudaSuccess)
+        return STATEKV_ERR_CUDA;
+    for (int s = a.stream_begin; s < a.stream_begin + a.stream_count; ++s)
+        for (int l = a.layer_begin; l < a.layer_begin + a.layer_count; ++l)
+            h->text_host[static_cast<size_t>(s) * c.num_layers + l] += n;
     return STATEKV_OK;
 }
 
@@ -363,6 +438,7 @@ statekv_status statekv_init(const statekv_config* cfg, void* device_arena, size_
     h->lay = lay;
     h->arena = static_cast<uint8_t*>(device_arena);
     h->frames_host.assign(static_cast<size_t>(d.SL), 0);
+    h->text_host.assign(static_cast<size_t>(d.SL), 0);
     h->prof_on = false;
     h->prof_used = 0;
     std::memset(&h->tm_sk, 0, sizeof(CUtensorMap));
@@ -438,6 +514,30 @@ statekv_status statekv_full_attention_frame(statekv_handle* h, const statekv_fra
     return run_full(h, *args, reinterpret_cast<cudaStream_t>(stream));
 }
 
+statekv_status statekv_decode_step(statekv_handle* h, const statekv_decode_args* a,
+                                  statekv_stream stream)
+{
+    if (!h || !a) return STATEKV_ERR_INVALID_ARG;
+    const statekv_config& c = h->cfg;
+    if (a->stream_count < 1 || a->layer_count < 1 || a->stream_begin < 0 || a->layer_begin < 0 ||
+        a->stream_begin + a->stream_count > c.num_streams ||
+        a->layer_begin + a->layer_count > c.num_layers || a->num_tokens < 1 ||
+        a->num_tokens > kMaxFrameTokens)
+        return STATEKV_ERR_INVALID_ARG;
+    if (!a->q || !a->k || !a->v || !a->out || !aligned(a->q, 16) || !aligned(a->k, 16) ||
+        !aligned(a->v, 16) || !aligned(a->out, 16))
+        return STATEKV_ERR_INVALID_ARG;
+    if (*h->status_host != 0) return device_status(*h->status_host);
+    for (int s = a->stream_begin; s < a->stream_begin + a->stream_count; ++s)
+        for (int l = a->layer_begin; l < a->layer_begin + a->layer_count; ++l) {
+            const size_t unit = static_cast<size_t>(s) * c.num_layers + l;
+            if (static_cast<long long>(h->frames_host[unit]) * c.tokens_per_frame +
+                    h->text_host[unit] + a->num_tokens > h->d.cap)
+                return STATEKV_ERR_CACHE_FULL;
+        }
+    return run_decode(h, *a, reinterpret_cast<cudaStream_t>(stream));
+}
+
 statekv_status statekv_prefill_frame_host(statekv_handle* h, const statekv_frame_args* args,
                                           statekv_stream stream)
 {
@@ -503,7 +603,8 @@ statekv_status statekv_cache_view(const statekv_handle* h, int32_t stream, int32
     const size_t per = static_cast<size_t>(h->cfg.num_kv_heads) * h->d.cap * h->cfg.head_dim * 2;
     out->k = h->arena + h->lay.cache_k + unit * per;
     out->v = h->arena + h->lay.cache_v + unit * per;
-    out->length = static_cast<int64_t>(h->frames_host[unit]) * h->cfg.tokens_per_frame;
+    out->length = static_cast<int64_t>(h->frames_host[unit]) * h->cfg.tokens_per_frame +
+                  h->text_host[unit];
     out->capacity = h->d.cap;
     return STATEKV_OK;
 }

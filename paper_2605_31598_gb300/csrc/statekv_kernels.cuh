@@ -44,7 +44,9 @@ struct AttnParams {
     const __nv_bfloat16* q;   // [U][T][Hq][D]
     __nv_bfloat16* out;       // [U][T][Hq][D]
     float* partials;          // [U][Hkv][MT][P]; null: no importance (full attention)
-    const int32_t* counts;    // arena [S*L][Hkv]: visible keys before the frame = counts * count_mul
+    const int32_t* counts;    // arena [S*L][Hkv]: visible keys before the frame =
+                              //   counts * count_mul + (count_add ? count_add : 0)
+    const int32_t* count_add; // nullable arena [S*L][Hkv]
     int32_t* status;          // device-visible status word
     UnitRange units;
     int T, Hq, Hkv, G, B, P, MT;
@@ -70,15 +72,21 @@ struct SelectParams {
 };
 
 struct AppendParams {
-    const __nv_bfloat16* k;     // [U][T][Hkv][D]
+    const __nv_bfloat16* k;     // [U][T][Hkv][D]: T rows per unit appended
     const __nv_bfloat16* v;
     __nv_bfloat16* cache_k;     // arena [S*L][Hkv][cap][D]
     __nv_bfloat16* cache_v;
     const int32_t* frames;      // arena [S*L][Hkv]
+    const int32_t* row_add;     // nullable arena [S*L][Hkv]: rows already past frames * row_mul
     UnitRange units;
     int U, T, Hkv, D;
+    int row_mul;                // first row = frames * row_mul + row_add
     long long cap;
 };
+
+// Adds `n` to counter[unit_abs(u) * Hkv + h] for every unit u < U and head h.
+cudaError_t launch_advance(int32_t* counter, UnitRange units, int U, int Hkv, int n,
+                           cudaStream_t st);
 
 // Shared-memory bytes the attention kernel needs for head dim D.
 size_t attn_smem_bytes(int D);

@@ -22,7 +22,7 @@ STATUS_NAMES = {
     6: "STATEKV_ERR_ARENA_TOO_SMALL", 7: "STATEKV_ERR_DEVICE_FAULT",
 }
 EXPORTED = ("statekv_arena_bytes", "statekv_init", "statekv_prefill_frame",
-            "statekv_prefill_frame_host", "statekv_full_attention_frame",
+            "statekv_prefill_frame_host", "statekv_full_attention_frame", "statekv_decode_step",
             "statekv_state_view", "statekv_cache_view",
             "statekv_profile_enable", "statekv_profile_read", "statekv_sync",
             "statekv_device_error", "statekv_frame_attention_noalloc",
@@ -36,6 +36,14 @@ class statekv_config(ctypes.Structure):
                 ("state_capacity", ctypes.c_int32), ("max_frames", ctypes.c_int32),
                 ("causal_in_frame", ctypes.c_int32), ("host_staging", ctypes.c_int32),
                 ("softmax_scale", ctypes.c_float), ("watchdog_ms", ctypes.c_uint32)]
+
+
+class statekv_decode_args(ctypes.Structure):
+    _fields_ = [("stream_begin", ctypes.c_int32), ("stream_count", ctypes.c_int32),
+                ("layer_begin", ctypes.c_int32), ("layer_count", ctypes.c_int32),
+                ("num_tokens", ctypes.c_int32),
+                ("q", ctypes.c_void_p), ("k", ctypes.c_void_p), ("v", ctypes.c_void_p),
+                ("out", ctypes.c_void_p)]
 
 
 class statekv_frame_args(ctypes.Structure):
@@ -86,6 +94,9 @@ def lib() -> ctypes.CDLL:
                 fn = getattr(L, name)
                 fn.argtypes = [ctypes.c_void_p, P(statekv_frame_args), ctypes.c_void_p]
                 fn.restype = st
+            L.statekv_decode_step.argtypes = [ctypes.c_void_p, P(statekv_decode_args),
+                                              ctypes.c_void_p]
+            L.statekv_decode_step.restype = st
             L.statekv_state_view.argtypes = [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32,
                                              P(statekv_state_info)]
             L.statekv_state_view.restype = st
@@ -149,6 +160,10 @@ def statekv_prefill_frame_host(handle: int, args: statekv_frame_args, stream: in
 
 def statekv_full_attention_frame(handle: int, args: statekv_frame_args, stream: int) -> int:
     return lib().statekv_full_attention_frame(handle, ctypes.byref(args), ctypes.c_void_p(stream))
+
+
+def statekv_decode_step(handle: int, args: statekv_decode_args, stream: int) -> int:
+    return lib().statekv_decode_step(handle, ctypes.byref(args), ctypes.c_void_p(stream))
 
 
 def statekv_state_view(handle: int, stream: int, layer: int) -> statekv_state_info:
@@ -266,6 +281,20 @@ class StateKV:
         st = (stream or torch.cuda.current_stream()).cuda_stream
         args = self._args(q, k, v, out, None, stream_begin, sc, layer_begin, lc)
         return statekv_full_attention_frame(self.handle, args, st)
+
+    def decode_step(self, q, k, v, out, *, stream_begin=0, stream_count=None, layer_begin=0,
+                    layer_count=None, stream=None) -> int:
+        """Enqueue ``q.shape[2]`` new tokens per (stream, layer) over the decode
+        cache (q: [S][L][n][Hq][d] bf16, k/v: [S][L][n][Hkv][d]); their K/V are
+        appended afterwards.  Returns the C status."""
+        import torch
+
+        sc = self.cfg.num_streams - stream_begin if stream_count is None else stream_count
+        lc = self.cfg.num_layers - layer_begin if layer_count is None else layer_count
+        st = (stream or torch.cuda.current_stream()).cuda_stream
+        args = statekv_decode_args(stream_begin, sc, layer_begin, lc, int(q.shape[2]),
+                                   q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr())
+        return statekv_decode_step(self.handle, args, st)
 
     def prefill_frame_host(self, q, k, v, out, importance=None, *, stream_begin=0,
                            stream_count=None, layer_begin=0, layer_count=None,
