@@ -14,6 +14,8 @@ only compiles it with gcc and marshals numpy arrays.  What it follows:
   layer and KV head), each weight taken as exp(score - LSE) (App. B.1);
 * Sec. 3.3, Eq. 6 -- keep the top B of the pool (state + frame tokens);
 * Sec. 3.2/3.3 -- append the frame's K, V to the decode cache; L_n += T.
+* Sec. 2 / Sec. 4 -- the recency-window baseline the method is compared with
+  (``policy=1``): the state keeps the B most recent tokens instead.
 * Sec. 4.1 / App. B -- the full self-attention baseline: the frame's queries
   attend to every earlier token and to the frame (causal within it), which
   is Eq. 5 with nothing ever evicted (``full_attention``, numpy matrix form).
@@ -66,6 +68,11 @@ def _load():
                 ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
                 ctypes.c_int, ctypes.c_double, ctypes.c_int64,
                 u16p, u16p, u16p, i32p, i64p, u16p, u16p, f64p, f64p, i32p]
+            lib.oracle_prefill_frame_policy.restype = ctypes.c_int
+            lib.oracle_prefill_frame_policy.argtypes = [
+                ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                ctypes.c_int, ctypes.c_double, ctypes.c_int64,
+                u16p, u16p, u16p, i32p, i64p, u16p, u16p, f64p, f64p, i32p, ctypes.c_int]
             lib.oracle_append_cache.restype = ctypes.c_int
             lib.oracle_append_cache.argtypes = [
                 ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int64, ctypes.c_int64,
@@ -102,8 +109,11 @@ class OracleLayer:
     detailed (decode) cache; ``virtual_len`` is L_n.
     """
 
-    def __init__(self, n_q, n_kv, d, T, B, max_frames, causal=True, scale=None):
+    def __init__(self, n_q, n_kv, d, T, B, max_frames, causal=True, scale=None, policy=0):
+        """policy 0: the method's top-B importance selection (Eq. 6); policy 1:
+        the recency window (keep the B most recent tokens), the baseline."""
         self.n_q, self.n_kv, self.d, self.T, self.B = n_q, n_kv, d, T, B
+        self.policy = int(policy)
         self.causal = 1 if causal else 0
         self.scale = float(scale) if scale else 1.0 / np.sqrt(d)
         self.count = np.zeros(n_kv, np.int32)
@@ -151,13 +161,13 @@ class OracleLayer:
                                      _ptr(self.dv, ctypes.c_uint16))
         if rc != 0:
             raise RuntimeError("oracle: decode cache full")
-        rc = lib.oracle_prefill_frame(
+        rc = lib.oracle_prefill_frame_policy(
             n_q, n_kv, d, T, B, self.causal, self.scale, self.virtual_len,
             _ptr(q, ctypes.c_uint16), _ptr(k, ctypes.c_uint16), _ptr(v, ctypes.c_uint16),
             _ptr(self.count, ctypes.c_int32), _ptr(self.pos, ctypes.c_int64),
             _ptr(self.sk, ctypes.c_uint16), _ptr(self.sv, ctypes.c_uint16),
             _ptr(out, ctypes.c_double), _ptr(imp, ctypes.c_double),
-            _ptr(kept, ctypes.c_int32))
+            _ptr(kept, ctypes.c_int32), self.policy)
         if rc != 0:
             raise RuntimeError("oracle: bad arguments")
         self.virtual_len += T

@@ -92,11 +92,34 @@ static int pos_cmp(const void* pa, const void* pb)
  *   kept              optional [n_kv][B+T] 0/1 flags, same columns as imp
  * Returns 0, or -1 on bad arguments or allocation failure.
  */
+int oracle_prefill_frame_policy(int n_q, int n_kv, int d, int T, int B, int causal, double scale,
+                                int64_t virtual_len, const uint16_t* q, const uint16_t* k,
+                                const uint16_t* v, int32_t* count, int64_t* pos, uint16_t* sk,
+                                uint16_t* sv, double* out, double* imp, int32_t* kept, int policy);
+
 int oracle_prefill_frame(int n_q, int n_kv, int d, int T, int B, int causal, double scale,
                          int64_t virtual_len, const uint16_t* q, const uint16_t* k,
                          const uint16_t* v, int32_t* count, int64_t* pos, uint16_t* sk,
                          uint16_t* sv, double* out, double* imp, int32_t* kept)
 {
+    return oracle_prefill_frame_policy(n_q, n_kv, d, T, B, causal, scale, virtual_len, q, k, v,
+                                       count, pos, sk, sv, out, imp, kept, 0);
+}
+
+/*
+ * The same frame step with a choice of which B pool tokens the state keeps:
+ *   policy 0  the method (Eq. 6): the B highest importances, ties to the
+ *             older token;
+ *   policy 1  the recency window of the ReKV-style baseline the paper compares
+ *             with (Sec. 2, Sec. 4): the B most recent positions.
+ * The attention and the importance are computed the same way for both.
+ */
+int oracle_prefill_frame_policy(int n_q, int n_kv, int d, int T, int B, int causal, double scale,
+                                int64_t virtual_len, const uint16_t* q, const uint16_t* k,
+                                const uint16_t* v, int32_t* count, int64_t* pos, uint16_t* sk,
+                                uint16_t* sv, double* out, double* imp, int32_t* kept, int policy)
+{
+    if (policy != 0 && policy != 1) return -1;
     if (n_q <= 0 || n_kv <= 0 || n_q % n_kv != 0 || d <= 0 || T <= 0 || B < 0) return -1;
     const int G = n_q / n_kv;
     const int P = B + T;
@@ -178,6 +201,8 @@ int oracle_prefill_frame(int n_q, int n_kv, int d, int T, int B, int causal, dou
         }
         int nkeep = np;
         if (np > B) {
+            if (policy == 1)  /* most recent first: rank by position */
+                for (int c = 0; c < np; ++c) pool[c].score = (double)pool[c].pos;
             qsort(pool, (size_t)np, sizeof(candidate), candidate_cmp);
             nkeep = B;
         }

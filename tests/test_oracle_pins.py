@@ -143,6 +143,35 @@ def test_full_attention_function_matches_uncompressed_stream(causal):
         np.testing.assert_allclose(o, f["out"], rtol=1e-11, atol=1e-12)
 
 
+@pytest.mark.parametrize("B", [7, 10, 13])
+def test_recency_window_keeps_the_latest_tokens(B):
+    """policy 1 (the recency-window baseline): the state holds the B most
+    recent tokens, so frame n attends exactly to the last min(B, (n-1)T)
+    earlier tokens plus itself (B multiple of T and not)."""
+    import oracle
+
+    n_q, n_kv, d, T, N = 4, 2, 16, 5, 6
+    rng = np.random.default_rng(11)
+    lay = OracleLayer(n_q, n_kv, d, T, B, max_frames=N, policy=1)
+    ks, vs = [], []
+    for n in range(N):
+        q = rand_bits(rng, (T, n_q, d))
+        k = rand_bits(rng, (T, n_kv, d))
+        v = rand_bits(rng, (T, n_kv, d))
+        out, _, _ = lay.prefill_frame(q, k, v)
+        prev_k = np.concatenate(ks) if ks else np.zeros((0, n_kv, d), np.uint16)
+        prev_v = np.concatenate(vs) if vs else np.zeros((0, n_kv, d), np.uint16)
+        w = min(B, n * T)
+        ref = oracle.full_attention(q, np.concatenate([prev_k[len(prev_k) - w:], k]),
+                                    np.concatenate([prev_v[len(prev_v) - w:], v]), w)
+        np.testing.assert_allclose(out, ref, rtol=1e-11, atol=1e-12)
+        ks.append(k)
+        vs.append(v)
+        total = (n + 1) * T
+        for h in range(n_kv):
+            assert list(lay.state_positions(h)) == list(range(max(0, total - B), total))
+
+
 def test_attention_over_selected_state_matches_library():
     """B < N*T: each frame's output is attention over exactly the pre-frame
     state's keys (looked up by position in the full stream) followed by the
