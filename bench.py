@@ -292,9 +292,11 @@ def run_ours(args, world, rank, local):
     log(f"[bench] rank {rank}: generating {nframes} frames of {args.workload} inputs")
     frames = [batch_qkv(shape, n, streams=range(S), layers=range(L), seed=seed, device=device)
               for n in range(1, nframes + 1)]
-    eng = StateKV(make_config(shape))
+    sel = 1 if args.selection == "recency" else 0
+    eng = StateKV(make_config(shape, selection=sel))
     out = torch.empty_like(frames[0][0])
-    imp = torch.empty((S, L, Hkv, B + T), dtype=torch.float32, device=device)
+    imp = (torch.empty((S, L, Hkv, B + T), dtype=torch.float32, device=device)
+           if sel == 0 else None)
 
     def step(n):
         q, k, v = frames[n]
@@ -388,6 +390,8 @@ def run_ours(args, world, rank, local):
         "dtype": "bf16",
         "data": "synthetic",
         "config": {"workload": WORKLOAD_TEXT[args.workload], "streams": S, "layers": L,
+                   "selection": ("top-B importance (the method)" if sel == 0 else
+                                 "recency window (baseline; no importance)"),
                    "steady_state_frames": f"{fill + args.warmup + 1}..{nframes}",
                    "l2": "no flush: each step reads fresh Q/K/V and the full state "
                          f"(~{(2 * S * L * Hkv * B * d * 2 + S * L * T * (shape.num_q_heads + 2 * Hkv) * d * 2) / 1e6:.0f} MB "
@@ -443,9 +447,11 @@ def run_e2e(args, shape, fill, seed, device, frames):
     steps = min(args.steps, 64)
     n_total = fill + args.warmup + steps
     host = [tuple(x.cpu().pin_memory() for x in frames[n]) for n in range(n_total)]
+    sel = 1 if args.selection == "recency" else 0
     out_h = torch.empty(host[0][0].shape, dtype=torch.bfloat16).pin_memory()
-    imp_h = torch.empty((S, L, Hkv, B + T), dtype=torch.float32).pin_memory()
-    eng = StateKV(make_config(shape, host_staging=True))
+    imp_h = (torch.empty((S, L, Hkv, B + T), dtype=torch.float32).pin_memory()
+             if sel == 0 else None)
+    eng = StateKV(make_config(shape, host_staging=True, selection=sel))
 
     def step(n):
         q, k, v = host[n]
@@ -466,7 +472,7 @@ def run_e2e(args, shape, fill, seed, device, frames):
     ms = e0.elapsed_time(e1)
     assert eng.sync() == 0
     h2d = sum(x.numel() * x.element_size() for x in host[0])
-    d2h = out_h.numel() * 2 + imp_h.numel() * 4
+    d2h = out_h.numel() * 2 + (imp_h.numel() * 4 if imp_h is not None else 0)
     eng.close()
     return {"value": S * steps / (ms * 1e-3), "unit": "frames/s", "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "steps": steps,
@@ -651,6 +657,9 @@ def main():
     ap.add_argument("--max-frames", type=int, default=0,
                     help="decode-cache capacity in frames (default: the workload's); "
                          "a small value keeps the arena small for profiler captures")
+    ap.add_argument("--selection", choices=["importance", "recency"], default="importance",
+                    help="state policy: the method's top-B importance, or the recency-window "
+                         "baseline")
     ap.add_argument("--curve", action="store_true",
                     help="per-frame cost vs frame index, StateKV next to exact full attention")
     ap.add_argument("--frames", type=int, default=0, help="--curve: frames to run (default: "

@@ -77,6 +77,12 @@ typedef struct {
     int32_t host_staging;     /* 1: reserve arena space for statekv_prefill_frame_host */
     float softmax_scale;      /* 0 -> 1 / sqrt(head_dim) (Eq. 5) */
     uint32_t watchdog_ms;     /* bound on every device-side wait; 0 -> 2000 ms */
+    int32_t selection;        /* which B tokens the state keeps after each frame:
+                                 0 = the method's top-B importance (Eq. 6);
+                                 1 = recency window, the B most recent tokens (the
+                                     ReKV-style baseline the paper compares with);
+                                     no importance is computed, so the per-call
+                                     importance pointer must be NULL */
 } statekv_config;
 
 /* Bytes of device arena the configuration needs.  Returns INVALID_ARG or

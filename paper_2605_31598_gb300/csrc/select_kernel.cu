@@ -15,6 +15,8 @@
 //      (ascending) as 128-bit row copies, and their positions are updated.
 #include "statekv_kernels.cuh"
 
+#include <algorithm>
+
 namespace statekv {
 namespace {
 
@@ -249,6 +251,62 @@ cudaError_t launch_select(const SelectParams& p, int U, cudaStream_t st)
 {
     const dim3 grid(p.Hkv, U);
     state_select_gather<<<grid, kSelThreads, select_smem_bytes(p.P, p.T), st>>>(p);
+    return cudaGetLastError();
+}
+
+// Recency window (the baseline the method is compared with): the state keeps
+// the B most recent tokens.  Token t of frame n sits at position (n-1) T + t
+// and goes to ring slot position mod B, which holds the token B positions
+// older -- exactly the one leaving the window -- so no search is needed.
+// A flat grid of 16-byte row chunks (like the cache append); a second kernel
+// then advances the per-head counters, after every copy has read them.
+__global__ void __launch_bounds__(256) state_recency_scatter(const RecencyParams p)
+{
+    const int t0 = p.T > p.B ? p.T - p.B : 0;  // older frame tokens leave the window at once
+    const int nt = p.T - t0, chunks = p.D / 8;
+    const long long per_head = static_cast<long long>(nt) * (chunks + 1);  // rows x (chunks + position)
+    const long long total = 2ll * p.U * p.Hkv * per_head;
+    for (long long w = blockIdx.x * 256ll + threadIdx.x; w < total; w += 256ll * gridDim.x) {
+        const int which = static_cast<int>(w / (p.U * p.Hkv * per_head));
+        const long long r = w % (p.U * p.Hkv * per_head);
+        const int uh = static_cast<int>(r / per_head);
+        const int u = uh / p.Hkv, hkv = uh % p.Hkv;
+        const long long rr = r % per_head;
+        const int t = t0 + static_cast<int>(rr / (chunks + 1));
+        const int ch = static_cast<int>(rr % (chunks + 1));
+        const size_t head = static_cast<size_t>(p.units.unit_abs(u)) * p.Hkv + hkv;
+        const long long pos = static_cast<long long>(p.frames[head]) * p.T + t;
+        const long long slot = pos % p.B;
+        if (ch == chunks) {  // one thread per row writes its position
+            if (which == 0) p.positions[head * p.B + slot] = static_cast<int32_t>(pos);
+            continue;
+        }
+        const __nv_bfloat16* src =
+            (which ? p.v : p.k) + ((static_cast<size_t>(u) * p.T + t) * p.Hkv + hkv) * p.D + ch * 8;
+        __nv_bfloat16* dst = (which ? p.state_v : p.state_k) + (head * p.B + slot) * p.D + ch * 8;
+        *reinterpret_cast<uint4*>(dst) = *reinterpret_cast<const uint4*>(src);
+    }
+}
+
+__global__ void recency_advance(const RecencyParams p)
+{
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= p.U * p.Hkv) return;
+    const size_t head = static_cast<size_t>(p.units.unit_abs(i / p.Hkv)) * p.Hkv + i % p.Hkv;
+    const long long seen = static_cast<long long>(p.frames[head] + 1) * p.T;
+    p.counts[head] = static_cast<int32_t>(seen < p.B ? seen : p.B);
+    p.frames[head] += 1;
+}
+
+cudaError_t launch_recency(const RecencyParams& p, cudaStream_t st)
+{
+    if (p.B > 0) {
+        const int t0 = p.T > p.B ? p.T - p.B : 0;
+        const long long work = 2ll * p.U * p.Hkv * (p.T - t0) * (p.D / 8 + 1);
+        const int blocks = static_cast<int>(std::min<long long>((work + 255) / 256, 152ll * 16));
+        state_recency_scatter<<<blocks, 256, 0, st>>>(p);
+    }
+    recency_advance<<<(p.U * p.Hkv + 255) / 256, 256, 0, st>>>(p);
     return cudaGetLastError();
 }
 

@@ -45,7 +45,8 @@ statekv_status check_config(const statekv_config* c, Derived* d)
         c->num_q_heads % c->num_kv_heads != 0 || c->head_dim < 1 || c->tokens_per_frame < 1 ||
         c->state_capacity < 0 || c->max_frames < 1 ||
         (c->causal_in_frame != 0 && c->causal_in_frame != 1) ||
-        (c->host_staging != 0 && c->host_staging != 1) || !(c->softmax_scale >= 0.f) ||
+        (c->host_staging != 0 && c->host_staging != 1) ||
+        (c->selection != 0 && c->selection != 1) || !(c->softmax_scale >= 0.f) ||
         !std::isfinite(c->softmax_scale))
         return STATEKV_ERR_INVALID_ARG;
     if (static_cast<long long>(c->max_frames) * c->tokens_per_frame > 0x7FFFFFFFll)
@@ -177,6 +178,7 @@ statekv_status check_args(const statekv_handle* h, const statekv_frame_args* a, 
             return STATEKV_ERR_INVALID_ARG;
     }
     if (host && !c.host_staging) return STATEKV_ERR_INVALID_ARG;
+    if (c.selection == 1 && a->importance) return STATEKV_ERR_INVALID_ARG;  // none computed
     if (*h->status_host != 0) return device_status(*h->status_host);
     for (int s = a->stream_begin; s < a->stream_begin + a->stream_count; ++s)
         for (int l = a->layer_begin; l < a->layer_begin + a->layer_count; ++l) {
@@ -244,7 +246,7 @@ statekv_status run_step(statekv_handle* h, const statekv_frame_args& a, cudaStre
     AttnParams pa{};
     pa.q = static_cast<const __nv_bfloat16*>(a.q);
     pa.out = static_cast<__nv_bfloat16*>(a.out);
-    pa.partials = partials;
+    pa.partials = c.selection == 0 ? partials : nullptr;  // recency: no importance
     pa.counts = counts;
     pa.status = h->status_dev;
     pa.units = ur;
@@ -263,6 +265,24 @@ statekv_status run_step(statekv_handle* h, const statekv_frame_args& a, cudaStre
         cudaSuccess)
         return STATEKV_ERR_CUDA;
 
+    if (c.selection == 1) {
+        RecencyParams pr{};
+        pr.k = ap.k;
+        pr.v = ap.v;
+        pr.state_k = h->at<__nv_bfloat16>(h->lay.state_k);
+        pr.state_v = h->at<__nv_bfloat16>(h->lay.state_v);
+        pr.positions = h->at<int32_t>(h->lay.positions);
+        pr.counts = counts;
+        pr.frames = frames;
+        pr.units = ur;
+        pr.U = U;
+        pr.T = T;
+        pr.Hkv = Hkv;
+        pr.D = D;
+        pr.B = c.state_capacity;
+        if (timed(h, 2, st, [&] { return launch_recency(pr, st); }) != cudaSuccess)
+            return STATEKV_ERR_CUDA;
+    } else {
     SelectParams ps{};
     ps.partials = partials;
     ps.importance = a.importance;
@@ -283,6 +303,7 @@ statekv_status run_step(statekv_handle* h, const statekv_frame_args& a, cudaStre
     ps.MT = d.MT;
     if (timed(h, 2, st, [&] { return launch_select(ps, U, st); }) != cudaSuccess)
         return STATEKV_ERR_CUDA;
+    }
 
     for (int s = a.stream_begin; s < a.stream_begin + a.stream_count; ++s)
         for (int l = a.layer_begin; l < a.layer_begin + a.layer_count; ++l)

@@ -84,6 +84,22 @@ struct AppendParams {
     long long cap;
 };
 
+struct RecencyParams {
+    const __nv_bfloat16* k;     // [U][T][Hkv][D]
+    const __nv_bfloat16* v;
+    __nv_bfloat16* state_k;     // arena [S*L][Hkv][B][D], slot = position mod B
+    __nv_bfloat16* state_v;
+    int32_t* positions;         // arena [S*L][Hkv][B]
+    int32_t* counts;            // arena [S*L][Hkv]
+    int32_t* frames;            // arena [S*L][Hkv]
+    UnitRange units;
+    int U, T, Hkv, D, B;
+};
+
+// Recency-window state update (the baseline): the frame's tokens enter ring
+// slots position mod B, overwriting the tokens that leave the window.
+cudaError_t launch_recency(const RecencyParams& p, cudaStream_t st);
+
 // Adds `n` to counter[unit_abs(u) * Hkv + h] for every unit u < U and head h.
 cudaError_t launch_advance(int32_t* counter, UnitRange units, int U, int Hkv, int n,
                            cudaStream_t st);

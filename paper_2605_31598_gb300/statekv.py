@@ -35,7 +35,8 @@ class statekv_config(ctypes.Structure):
                 ("head_dim", ctypes.c_int32), ("tokens_per_frame", ctypes.c_int32),
                 ("state_capacity", ctypes.c_int32), ("max_frames", ctypes.c_int32),
                 ("causal_in_frame", ctypes.c_int32), ("host_staging", ctypes.c_int32),
-                ("softmax_scale", ctypes.c_float), ("watchdog_ms", ctypes.c_uint32)]
+                ("softmax_scale", ctypes.c_float), ("watchdog_ms", ctypes.c_uint32),
+                ("selection", ctypes.c_int32)]
 
 
 class statekv_decode_args(ctypes.Structure):
@@ -220,13 +221,17 @@ def statekv_status_string(status: int) -> str:
 
 
 # ---------------------------------------------------------------- owner object
+SELECTION_IMPORTANCE = 0  # the method: top-B by importance (Eq. 6)
+SELECTION_RECENCY = 1     # the baseline: the B most recent tokens
+
+
 def make_config(shape, *, causal=True, host_staging=False, softmax_scale=0.0,
-                watchdog_ms=0) -> statekv_config:
+                watchdog_ms=0, selection=SELECTION_IMPORTANCE) -> statekv_config:
     """statekv_config from an ``inputs.Shape``-like object."""
     return statekv_config(shape.num_streams, shape.num_layers, shape.num_q_heads,
                           shape.num_kv_heads, shape.head_dim, shape.tokens_per_frame,
                           shape.state_capacity, shape.max_frames, 1 if causal else 0,
-                          1 if host_staging else 0, softmax_scale, watchdog_ms)
+                          1 if host_staging else 0, softmax_scale, watchdog_ms, selection)
 
 
 class StateKV:

@@ -64,6 +64,7 @@ def _cfg(**kw):
     (dict(state_capacity=-1), 1),
     (dict(max_frames=0), 1),
     (dict(causal_in_frame=2), 1),
+    (dict(selection=2), 1),               # neither top-B importance nor recency
     (dict(softmax_scale=-1.0), 1),
     (dict(state_capacity=30000), 2),      # pool beyond the select kernel's limit
     (dict(tokens_per_frame=5000), 2),
