@@ -13,19 +13,14 @@
 //           O += P V with P in bf16.
 // tcgen05 runs every contraction with the A operand in TMEM (Q for Q K^T, P
 // for P V), so each MMA streams only K or V from shared memory.  TMEM
-// (512 columns): Q | score/P buffer of softmax warpgroup 0 | of warpgroup 1 |
-// O; P overwrites the scores it came from.
+// (512 columns): Q | P | S0 | S1 | O (layout below).
 //
-// Every query tile of a KV head reads the same K and V tiles, and keeping the
-// tensor core busy would take about as many bytes per cycle from L2 as the
-// SM can receive.  So for D = 128 two CTAs (consecutive query tiles of one
-// KV head) form a cluster: each loads one 64-column half of every K/V tile by
-// TMA with multicast into both CTAs' shared memory, halving the L2 reads and
-// TMA issues per CTA.  Both CTAs walk the same key tiles (the frame tiles
-// visible to either).  Tiles stream through a ring of six 32 KB slots in one
-// sequence: pass A's K tiles, then pass B's K(0) V(0) K(1) V(1) ...; a slot
-// is refilled once the MMAs of every CTA in the cluster have read it (the
-// MMA commit arrives on the slot's barrier in each CTA).
+// K and V tiles stream through a ring of six 32 KB shared-memory slots in one
+// sequence, pass A's K tiles, then pass B's K(0) V(0) K(1) V(1) ...; a slot is
+// refilled once the MMAs that read it have completed (their commit arrives on
+// the slot's barrier).  Optionally (cluster_size() below) two CTAs of
+// consecutive query tiles share each K/V tile by TMA multicast, each loading
+// one 64-column half into both CTAs' shared memory.
 //
 // 384 threads, three warpgroups:
 //   WG0  warp 0 producer (TMA), warps 1 and 3 MMA issuers X and Y (warp 1
@@ -36,11 +31,13 @@
 //        of odd tiles and every P V (in order, so O accumulates
 //        deterministically).  Descriptors are precomputed words, so an MMA
 //        costs the issuing warp an add or two besides itself.
-//   WG1, WG2  softmax warpgroups: thread = query row; they take alternate key
-//        tiles, each with its own TMEM score buffer, so the tensor core works
-//        on one warpgroup's tile while the other computes exponentials.
-// The column sums over a warp's 32 rows are a shuffle reduce-scatter (each
-// lane ends with one column); the four warps add through shared memory.
+//   WG1, WG2  softmax warpgroups.  Pass A: thread = query row; they take
+//        alternate key tiles, so the tensor core works on one warpgroup's
+//        tile while the other computes exponentials.  Pass B: both work on
+//        every tile, warpgroup w on keys [64 w, 64 w + 64), so each tile's P
+//        is ready after half a tile's work.
+// The column sums add a thread's rows in registers, then lanes by a shuffle
+// reduce-scatter, then the four warps of a warpgroup through shared memory.
 // Every mbarrier wait is bounded by the watchdog; on expiry the CTA records
 // DEV_TIMEOUT_ATTN, drains its in-flight copies and MMAs, frees TMEM and exits.
 #include "sm103_ptx.cuh"
@@ -54,11 +51,13 @@ using namespace ptx;
 constexpr int kThreads = 384;
 constexpr int kSlots = 6;        // 32 KB K/V tile slots (D = 128), one ring
 // TMEM columns: Q [0, 64) | P [64, 128) | S0 | S1 | O; pass A also uses O's
-// columns as a third score buffer S2.  In pass B warpgroup 0 writes its P
-// (bf16 pairs) into the P buffer, so Q K^T can refill S0 as soon as the
-// scores are read; warpgroup 1 writes P over the first 64 columns of S1, so
-// Q K^T into S1 waits for the P V that reads it.  (TMEM has no room for a
-// second P buffer next to Q, two score buffers and O.)
+// columns as a third score buffer S2.  Pass B puts even tiles' scores in S0
+// and odd tiles' in S1.  P (bf16 pairs) of even tiles goes to the P buffer,
+// so Q K^T can refill S0 as soon as both warpgroups have read the scores; P
+// of odd tiles overwrites the scores it came from (each warpgroup the first
+// 32 columns of its own 64), so Q K^T into S1 waits for the P V that reads
+// it.  (TMEM has no room for a second P buffer next to Q, two score buffers
+// and O.)
 constexpr uint32_t kColP = 64;
 constexpr uint32_t kColS0 = 128;
 constexpr uint32_t kColS1 = 256;
@@ -155,12 +154,12 @@ __device__ __forceinline__ void named_bar_sync(int id, int nthreads)
     asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
 }
 
-// One MMA group, D[d] (+)= A[a + 8k] * B_k for k < NK (bf16 in, fp32
-// accumulator, A in TMEM), with B's descriptor for step k given as its two
+// One MMA group, D[d] (+)= A[a + 8k (+ kGapA when k >= NK/2)] * B_k for k < NK
+// (bf16 in, fp32 accumulator, A in TMEM), with B's descriptor for step k given as its two
 // 32-bit words (lo + off(k), hi): the issuing warp shares its SM sub-partition
 // with the softmax warps, so each MMA should cost it as few instructions as
 // possible.
-template <int NK, bool kMajorB>
+template <int NK, bool kMajorB, uint32_t kGapA = 0>
 __device__ __forceinline__ void mma_group(uint32_t d, uint32_t a, uint32_t blo, uint32_t bhi,
                                           uint32_t idesc, bool accumulate)
 {
@@ -182,7 +181,7 @@ __device__ __forceinline__ void mma_group(uint32_t d, uint32_t a, uint32_t blo, 
                 "{\n\t.reg .b64 bd;\n\t"
                 "mov.b64 bd, {%2, %3};\n\t"
                 "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], bd, %4, 1;\n\t}" ::"r"(d),
-                "r"(a + 8 * k), "r"(blo + off), "r"(bhi), "r"(idesc)
+                "r"(a + 8 * k + (k >= NK / 2 ? kGapA : 0u)), "r"(blo + off), "r"(bhi), "r"(idesc)
                 : "memory");
     }
 }
@@ -251,76 +250,65 @@ __device__ __forceinline__ int qk_item(int nt, int it)  // it: Q K^T sequence in
     return it < nt ? it : nt + 2 * (it - nt);
 }
 
-// 16 TMEM lanes x 128 columns -> 64 registers (.16x256b layout): register
-// 4r + 2k + e holds lane (base + t/4 + 8k), column 8r + 2(t%4) + e, for
-// thread t and r < 16.
-__device__ __forceinline__ void tmem_ld_16x256b_x16(uint32_t taddr, float (&v)[64])
+// 16 TMEM lanes x 64 columns -> 32 registers (.16x256b layout): register
+// 4r + 2k + e holds lane (base + t/4 + 8k), column 8r + 2(t%4) + e, r < 8.
+__device__ __forceinline__ void tmem_ld_16x256b_x8(uint32_t taddr, float (&v)[32])
 {
-    uint32_t r[64];
+    uint32_t r[32];
     asm volatile(
-        "tcgen05.ld.sync.aligned.16x256b.x16.b32"
+        "tcgen05.ld.sync.aligned.16x256b.x8.b32"
         " {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15,"
-        " %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31,"
-        " %32, %33, %34, %35, %36, %37, %38, %39, %40, %41, %42, %43, %44, %45, %46, %47,"
-        " %48, %49, %50, %51, %52, %53, %54, %55, %56, %57, %58, %59, %60, %61, %62, %63},"
-        " [%64];"
+        " %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31},"
+        " [%32];"
         : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
           "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
           "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
           "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
           "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
-          "=r"(r[31]), "=r"(r[32]), "=r"(r[33]), "=r"(r[34]), "=r"(r[35]), "=r"(r[36]),
-          "=r"(r[37]), "=r"(r[38]), "=r"(r[39]), "=r"(r[40]), "=r"(r[41]), "=r"(r[42]),
-          "=r"(r[43]), "=r"(r[44]), "=r"(r[45]), "=r"(r[46]), "=r"(r[47]), "=r"(r[48]),
-          "=r"(r[49]), "=r"(r[50]), "=r"(r[51]), "=r"(r[52]), "=r"(r[53]), "=r"(r[54]),
-          "=r"(r[55]), "=r"(r[56]), "=r"(r[57]), "=r"(r[58]), "=r"(r[59]), "=r"(r[60]),
-          "=r"(r[61]), "=r"(r[62]), "=r"(r[63])
+          "=r"(r[31])
         : "r"(taddr)
         : "memory");
 #pragma unroll
-    for (int i = 0; i < 64; ++i) v[i] = __uint_as_float(r[i]);
+    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
-// 32 registers -> 16 TMEM lanes x 64 columns (.16x128b layout): register
-// 2r + k goes to lane (base + t/4 + 8k), column 4r + t%4.
-__device__ __forceinline__ void tmem_st_16x128b_x16(uint32_t taddr, const uint32_t (&r)[32])
+// 16 registers -> 16 TMEM lanes x 32 columns (.16x128b layout): register
+// 2r + k goes to lane (base + t/4 + 8k), column 4r + t%4, r < 8.
+__device__ __forceinline__ void tmem_st_16x128b_x8(uint32_t taddr, const uint32_t (&r)[16])
 {
     asm volatile(
-        "tcgen05.st.sync.aligned.16x128b.x16.b32 [%0],"
-        " {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16,"
-        " %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};" ::"r"(
-            taddr),
+        "tcgen05.st.sync.aligned.16x128b.x8.b32 [%0],"
+        " {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16};" ::"r"(taddr),
         "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
         "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),
-        "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]),
-        "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]),
-        "r"(r[29]), "r"(r[30]), "r"(r[31])
+        "r"(r[15])
         : "memory");
 }
 
-// Sums over the 8 lanes that share lane % 4 (lane bits 2..4) of 32 values,
-// as a reduce-scatter: lane l returns the sums of values 4 (l/4) .. +3.
-__device__ __forceinline__ void lane8_reduce_scatter(float (&x)[32], int lane, float (&out)[4])
+// Sums over the 8 lanes that share lane % 4 (lane bits 2..4) of 16 values,
+// as a reduce-scatter: lane l returns the sums of values 2 (l/4) and
+// 2 (l/4) + 1.
+__device__ __forceinline__ void lane8_reduce_scatter16(float (&x)[16], int lane, float (&out)[2])
 {
 #pragma unroll
-    for (int i = 0; i < 16; ++i) {
+    for (int i = 0; i < 8; ++i) {
         const bool up = (lane & 16) != 0;
-        const float send = up ? x[i] : x[i + 16];
-        const float keep = up ? x[i + 16] : x[i];
+        const float send = up ? x[i] : x[i + 8];
+        const float keep = up ? x[i + 8] : x[i];
         x[i] = keep + __shfl_xor_sync(0xffffffffu, send, 16);
     }
 #pragma unroll
-    for (int i = 0; i < 8; ++i) {
+    for (int i = 0; i < 4; ++i) {
         const bool up = (lane & 8) != 0;
-        const float send = up ? x[i] : x[i + 8];
-        const float keep = up ? x[i + 8] : x[i];
+        const float send = up ? x[i] : x[i + 4];
+        const float keep = up ? x[i + 4] : x[i];
         x[i] = keep + __shfl_xor_sync(0xffffffffu, send, 8);
     }
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
+    for (int i = 0; i < 2; ++i) {
         const bool up = (lane & 4) != 0;
-        const float send = up ? x[i] : x[i + 4];
-        const float keep = up ? x[i + 4] : x[i];
+        const float send = up ? x[i] : x[i + 2];
+        const float keep = up ? x[i + 2] : x[i];
         out[i] = keep + __shfl_xor_sync(0xffffffffu, send, 4);
     }
 }
@@ -344,9 +332,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t* slot_empty = bars + 6;
     uint64_t* sa_full = bars + 12;  // pass A: Q K^T of tile i done (index i % 6)
     uint64_t* sa_read = bars + 18;  // pass A: tile i read by its warpgroup (index i % 6)
-    uint64_t* sb_full = bars + 24;  // pass B: Q K^T result in score buffer w (of 2)
-    uint64_t* sb_read = bars + 26;  // pass B: warpgroup w has read score buffer w
-    uint64_t* p_full = bars + 28;   // pass B: warpgroup w has written its tile's P
+    uint64_t* sb_full = bars + 24;  // pass B: Q K^T of tile j in score buffer j & 1
+    uint64_t* sb_read = bars + 26;  // pass B: both warpgroups have read S0 ([1] unused)
+    uint64_t* p_full = bars + 28;   // pass B: both warpgroups have written P of tile j (j & 1)
     uint64_t* pv_done = bars + 30;  // pass B: P V(j) has completed (index j & 1)
     uint64_t* q_full = bars + 32;
     uint64_t* o_full = bars + 33;
@@ -408,8 +396,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(&sb_full[i], 1);
-            mbar_init(&sb_read[i], 128);
-            mbar_init(&p_full[i], 128);
+            mbar_init(&sb_read[i], 256);
+            mbar_init(&p_full[i], 256);
             mbar_init(&pv_done[i], 1);
         }
         mbar_init(a_read, 256);
@@ -553,14 +541,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                         done = &sa_full[it % kSA2];
                     } else {
                         // the buffer's previous pass-B tile (j - 2) is consumed: read by
-                        // warpgroup 0 (whose P has its own buffer), or, for warpgroup
-                        // 1 (whose P overwrites its scores), read by its P V
-                        const int j = it - nt, w = it & 1;
-                        if (j >= 2 && !(w == 0 ? wait_until(&sb_read[0], ((j - 2) >> 1) & 1, deadline)
-                                               : wait_until(&pv_done[j & 1], ((j - 2) >> 1) & 1, deadline)))
+                        // both warpgroups (S0: its P went to the P buffer), or read by
+                        // its P V (S1: its P overwrote the scores)
+                        const int j = it - nt, b = j & 1;
+                        if (j >= 2 && !(b == 0 ? wait_until(&sb_read[0], ((j - 2) >> 1) & 1, deadline)
+                                               : wait_until(&pv_done[1], ((j - 2) >> 1) & 1, deadline)))
                             return false;
-                        tS = w ? tS1 : tS0;
-                        done = &sb_full[w];
+                        tS = b ? tS1 : tS0;
+                        done = &sb_full[b];
                     }
                     tc_fence_after();
                     mma_group<D / 16, true>(tS, tQ, dk_lo + slot * kSlotStep, d_hi, kIdQK, false);
@@ -568,19 +556,27 @@ __global__ void __launch_bounds__(kThreads, 1)
                     release(slot);
                     return true;
                 };
-                // O += P(j) V(j), P in score buffer (nt + j) & 1
+                // O += P(j) V(j): P of even tiles in the P buffer (keys 0..63 then
+                // 64..127), of odd tiles over S1 (keys 0..63 at its columns 0..31,
+                // keys 64..127 at 64..95: each warpgroup over its own scores)
                 auto issue_pv = [&](int j) -> bool {
-                    const int w = (nt + j) & 1;
+                    const int b = j & 1;
                     const int item = nt + 2 * j + 1;
                     const int slot = item % kSlots;
-                    site = 7;
-                    if (!wait_until(&p_full[w], (j >> 1) & 1, deadline)) return false;
+                    // the V tile usually landed long ago: its wait goes first, so the
+                    // wait that P ends is the last before the MMAs
                     site = 8;
                     if (!wait_until(&slot_full[slot], (item / kSlots) & 1, deadline)) return false;
+                    site = 7;
+                    if (!wait_until(&p_full[b], (j >> 1) & 1, deadline)) return false;
                     tc_fence_after();
-                    mma_group<kBN / 16, false>(tO, w ? tS1 : tbase + kColP, dv_lo + slot * kSlotStep, d_hi, kIdPV,
-                                               j > 0);
-                    umma_commit(&pv_done[j & 1]);
+                    if (b == 0)
+                        mma_group<kBN / 16, false>(tO, tbase + kColP, dv_lo + slot * kSlotStep, d_hi,
+                                                   kIdPV, j > 0);
+                    else
+                        mma_group<kBN / 16, false, 32>(tO, tS1, dv_lo + slot * kSlotStep, d_hi, kIdPV,
+                                                       j > 0);
+                    umma_commit(&pv_done[b]);
                     release(slot);
                     return true;
                 };
@@ -621,8 +617,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int quad = warp & 3;               // TMEM lane quadrant of this warp
         const int row = quad * 32 + lane;        // TMEM lane = query row of the tile
         const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
-        const uint32_t tS = tbase + lane_off + (wg ? kColS1 : kColS0);
-        const uint32_t tP = tbase + lane_off + kColP;
         const float c = p.scale_log2;
         const int my_r = mt * kBM + row;
         const bool row_valid = my_r < rows;
@@ -723,10 +717,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
 
         // ---------------- pass B: P = exp2(S c - lse) -> TMEM (bf16) and column sums
-        // Layout of pass B: TMEM is read in 16-lane x 256-bit groups, so a thread
-        // holds 4 rows (quadrant rows 16h + t/4 + 8k, h, k in {0, 1}) x 32 columns
+        // Both warpgroups work on every tile, warpgroup wg on its keys
+        // [64 wg, 64 wg + 64), so a tile's P is ready after half a tile's work.
+        // TMEM is read in 16-lane x 256-bit groups: a thread holds 4 rows
+        // (quadrant rows 16h + t/4 + 8k, h, k in {0, 1}) x 16 columns
         // (8r + 2(t%4) + e); the column sums add 4 rows in registers and the 8
         // lanes that share t % 4 by a 3-step reduce-scatter.
+        // P of even tiles goes to the P buffer (so Q K^T can refill S0 once both
+        // warpgroups have read it); P of odd tiles overwrites the first half of
+        // this warpgroup's own S1 columns (Q K^T into S1 waits for that P V).
         float* nl_row = stat + 4 * kBM;  // -lse of every row of the tile
         if (wg == 0) nl_row[row] = nlse;
         named_bar_sync(1, 256);
@@ -746,12 +745,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         float* myred = red + wg * (2 * 4 * kBM);
         const int ct = threadIdx.x - 128 - 128 * wg;  // 0..127 within the warpgroup
         const int cq = 2 * (lane & 3);                // this thread's column offset in 8
+        const int c0 = 64 * wg;                       // this warpgroup's first key of a tile
+        const uint32_t tSh0 = tbase + lane_off + kColS0 + c0;   // this warpgroup's S0 half
+        const uint32_t tSh1 = tbase + lane_off + kColS1 + c0;   // its S1 half (and odd P)
+        const uint32_t tPh = tbase + lane_off + kColP + c0 / 2;  // its even-tile P
         // Every warp runs every iteration and arrives at the per-tile barrier;
         // after a timeout it only skips the work (a bar.sync cannot time out).
-        for (int j = (wg - nt) & 1, k2 = 0; j < nt; j += 2, ++k2) {
-            if (ok) ok = __all_sync(0xffffffffu, wait_until(&sb_full[wg], (j >> 1) & 1, deadline));
+        for (int j = 0; j < nt; ++j) {
+            const int b = j & 1;
+            if (ok) ok = __all_sync(0xffffffffu, wait_until(&sb_full[b], (j >> 1) & 1, deadline));
             const bool is_state = j < nst;
-            float* rb = myred + (k2 & 1) * (4 * kBM);  // [4 warps][128 columns]
+            float* rb = myred + b * (4 * kBM);  // [4 warps][64 columns]
             if (ok) {
                 tc_fence_after();
                 int lim4[4];  // keys [0, lim) of this tile are visible to each row
@@ -765,18 +769,21 @@ __global__ void __launch_bounds__(kThreads, 1)
                     for (int q4 = 0; q4 < 4; ++q4)
                         lim4[q4] = min(kBN, (p.causal ? min(T, tq4[q4] + 1) : T) - f0);
                 }
-                const bool full = lim4[0] == kBN && lim4[1] == kBN && lim4[2] == kBN && lim4[3] == kBN;
+                const int lmin = min(min(lim4[0], lim4[1]), min(lim4[2], lim4[3]));
+                const bool full = lmin >= c0 + 64;
                 const f2 cc = pk(c, c);
-                float v[2][64];
+                float v[2][32];
 #pragma unroll
-                for (int h = 0; h < 2; ++h) tmem_ld_16x256b_x16(tS + ((16u * h) << 16), v[h]);
+                for (int h = 0; h < 2; ++h) tmem_ld_16x256b_x8((b ? tSh1 : tSh0) + ((16u * h) << 16), v[h]);
                 tmem_ld_wait();
-                tc_fence_before();
-                mbar_arrive(&sb_read[wg]);  // Q K^T of tile j + 2 may overwrite the buffer
+                if (b == 0) {
+                    tc_fence_before();
+                    mbar_arrive(&sb_read[0]);  // Q K^T of tile j + 2 may overwrite S0
+                }
 #pragma unroll
                 for (int h = 0; h < 2; ++h)
 #pragma unroll
-                    for (int r = 0; r < 16; ++r)
+                    for (int r = 0; r < 8; ++r)
 #pragma unroll
                         for (int k = 0; k < 2; ++k) {
                             const int i = 4 * r + 2 * k;
@@ -786,56 +793,51 @@ __global__ void __launch_bounds__(kThreads, 1)
                             v[h][i] = ex2(x0);
                             v[h][i + 1] = ex2(x1);
                             if (!full) {
-                                const int col = 8 * r + cq, lim = lim4[2 * h + k];
+                                const int col = c0 + 8 * r + cq, lim = lim4[2 * h + k];
                                 v[h][i] = col < lim ? v[h][i] : 0.f;
                                 v[h][i + 1] = col + 1 < lim ? v[h][i + 1] : 0.f;
                             }
                         }
-                // Warpgroup 0 writes P into the P buffer, free once its previous
-                // tile's P V (j - 2) has read it; warpgroup 1 writes P over the
-                // scores it has just read (the next Q K^T into that buffer waits for
-                // this tile's P V).
-                if (wg == 0 && j >= 2)
+                // the P buffer is free once the P V of tile j - 2 has read it
+                if (b == 0 && j >= 2)
                     ok = __all_sync(0xffffffffu,
-                                    wait_until(&pv_done[j & 1], ((j - 2) >> 1) & 1, deadline));
+                                    wait_until(&pv_done[0], ((j - 2) >> 1) & 1, deadline));
                 if (ok) {
                     tc_fence_after();
 #pragma unroll
                     for (int h = 0; h < 2; ++h) {
-                        uint32_t pw[32];  // register 2r + k: row k, P column 4r + t%4
+                        uint32_t pw[16];  // register 2r + k: row k, P column 4r + t%4
 #pragma unroll
-                        for (int r = 0; r < 16; ++r)
+                        for (int r = 0; r < 8; ++r)
 #pragma unroll
                             for (int k = 0; k < 2; ++k)
                                 pw[2 * r + k] = pack_bf16x2(v[h][4 * r + 2 * k], v[h][4 * r + 2 * k + 1]);
-                        tmem_st_16x128b_x16((wg == 0 ? tP : tS) + ((16u * h) << 16), pw);
+                        tmem_st_16x128b_x8((b ? tSh1 : tPh) + ((16u * h) << 16), pw);
                     }
                     tmem_st_wait();
                     tc_fence_before();
-                    mbar_arrive(&p_full[wg]);
+                    mbar_arrive(&p_full[b]);
                     // the column sums run while the tensor core does this tile's P V:
                     // value 2r + e is column 8r + cq + e summed over the thread's rows
-                    float cs[32];
+                    float cs[16];
 #pragma unroll
-                    for (int r = 0; r < 16; ++r) {
+                    for (int r = 0; r < 8; ++r) {
                         const f2 a = add2(pk(v[0][4 * r], v[0][4 * r + 1]), pk(v[0][4 * r + 2], v[0][4 * r + 3]));
-                        const f2 b = add2(pk(v[1][4 * r], v[1][4 * r + 1]), pk(v[1][4 * r + 2], v[1][4 * r + 3]));
-                        upk(add2(a, b), cs[2 * r], cs[2 * r + 1]);
+                        const f2 bb = add2(pk(v[1][4 * r], v[1][4 * r + 1]), pk(v[1][4 * r + 2], v[1][4 * r + 3]));
+                        upk(add2(a, bb), cs[2 * r], cs[2 * r + 1]);
                     }
-                    float sum4[4];
-                    lane8_reduce_scatter(cs, lane, sum4);
-                    // this lane holds values 4m .. 4m+3 (m = lane / 4): r = 2m + (i >> 1), e = i & 1
+                    float sum2[2];
+                    lane8_reduce_scatter16(cs, lane, sum2);
+                    // this lane holds values 2m, 2m + 1 (m = lane / 4): columns 8m + cq + e
                     const int m4 = lane >> 2;
-#pragma unroll
-                    for (int i = 0; i < 4; ++i)
-                        rb[quad * kBM + 8 * (2 * m4 + (i >> 1)) + cq + (i & 1)] = sum4[i];
+                    rb[quad * 64 + 8 * m4 + cq] = sum2[0];
+                    rb[quad * 64 + 8 * m4 + cq + 1] = sum2[1];
                 }
             }
             named_bar_sync(2 + wg, 128);
-            if (ok && tile_valid && part != nullptr) {
-                const float s = rb[0 * kBM + ct] + rb[1 * kBM + ct] + rb[2 * kBM + ct] +
-                                rb[3 * kBM + ct];
-                const int key = (is_state ? state_tile(j) : j - nst) * kBN + ct;
+            if (ok && tile_valid && part != nullptr && ct < 64) {
+                const float s = rb[0 * 64 + ct] + rb[1 * 64 + ct] + rb[2 * 64 + ct] + rb[3 * 64 + ct];
+                const int key = (is_state ? state_tile(j) : j - nst) * kBN + c0 + ct;
                 if (is_state ? key < count : key < T) part[is_state ? key : B + key] = s;
             }
         }
