@@ -19,6 +19,12 @@ only compiles it with gcc and marshals numpy arrays.  What it follows:
 * Sec. 4.1 / App. B -- the full self-attention baseline: the frame's queries
   attend to every earlier token and to the frame (causal within it), which
   is Eq. 5 with nothing ever evicted (``full_attention``, numpy matrix form).
+* App. A -- layer-level selection (``policy=2``: one ranking per layer by the
+  attention summed over all heads, applied to every KV head) and the
+  assumption diagnostics computed from the full-attention baseline's
+  layer-level scores: the concentration C_{n,B} of historical attention in
+  its top-B tokens (App. A.1), and candidate-pool recall, weighted recall,
+  retention and churn of consecutive top-B oracle states (App. A.2).
 
 Readings of silent points: score ties keep the older token; a pool of at most
 B tokens is kept whole; the state is stored in ascending position.
@@ -111,7 +117,9 @@ class OracleLayer:
 
     def __init__(self, n_q, n_kv, d, T, B, max_frames, causal=True, scale=None, policy=0):
         """policy 0: the method's top-B importance selection (Eq. 6); policy 1:
-        the recency window (keep the B most recent tokens), the baseline."""
+        the recency window (keep the B most recent tokens), the baseline;
+        policy 2: layer-level selection (App. A), one top-B by the importance
+        summed over every KV head, shared by all heads."""
         self.n_q, self.n_kv, self.d, self.T, self.B = n_q, n_kv, d, T, B
         self.policy = int(policy)
         self.causal = 1 if causal else 0
@@ -178,14 +186,18 @@ class OracleLayer:
 
 
 def full_attention(q_bits: np.ndarray, k_bits: np.ndarray, v_bits: np.ndarray, n_prefix: int,
-                   causal: bool = True, scale: float | None = None) -> np.ndarray:
+                   causal: bool = True, scale: float | None = None,
+                   return_scores: bool = False):
     """Exact softmax attention of one frame (fp64), the full-SA baseline.
 
     q: [T][n_q][d]; k, v: [n_prefix + T][n_kv][d] bf16 bits, the earlier
     tokens in order followed by the frame's own.  Query i of the frame sees
     every earlier token and frame token j iff j <= i (all frame tokens when
     not causal); query head h reads KV head h // (n_q / n_kv).  Returns O
-    [T][n_q][d] float64.
+    [T][n_q][d] float64; with ``return_scores``, also the layer-level score
+    of every key (App. A's shared protocol: the attention weights summed over
+    the frame's queries within each head, then over all heads), float64
+    [n_prefix + T].
     """
     q = bf16_bits_to_f64(q_bits)
     k = bf16_bits_to_f64(k_bits)
@@ -198,6 +210,7 @@ def full_attention(q_bits: np.ndarray, k_bits: np.ndarray, v_bits: np.ndarray, n
     if causal:
         visible[:, n_prefix:] = np.tril(np.ones((T, T), dtype=bool))
     out = np.empty((T, n_q, d))
+    scores = np.zeros(n_prefix + T)
     for h in range(n_q):
         s = (q[:, h, :] @ k[:, h // G, :].T) * sc
         s = np.where(visible, s, -np.inf)
@@ -205,4 +218,54 @@ def full_attention(q_bits: np.ndarray, k_bits: np.ndarray, v_bits: np.ndarray, n
         w = np.exp(s)
         w /= w.sum(axis=1, keepdims=True)
         out[:, h, :] = w @ v[:, h // G, :]
-    return out
+        scores += w.sum(axis=0)
+    return (out, scores) if return_scores else out
+
+
+# ---------------------------------------------------------------------------
+# App. A diagnostics, on layer-level scores (one float per key position).
+
+def top_b(scores: np.ndarray, B: int) -> np.ndarray:
+    """Positions of the B highest scores, ties to the lower position (the
+    older token), ascending.  Every position is kept when there are <= B."""
+    scores = np.asarray(scores, np.float64)
+    n = scores.shape[0]
+    order = np.lexsort((np.arange(n), -scores))  # last key is the primary one
+    return np.sort(order[: min(B, n)])
+
+
+def concentration(hist_scores: np.ndarray, budgets) -> np.ndarray:
+    """App. A.1: C_{n,B} = (sum of the B largest historical scores) / (sum of
+    all historical scores), for each B in ``budgets``.  ``hist_scores`` are
+    the layer-level scores of the keys of frames before n."""
+    hist_scores = np.asarray(hist_scores, np.float64)
+    mass = hist_scores.sum()
+    return np.array([hist_scores[top_b(hist_scores, B)].sum() / mass for B in budgets])
+
+
+def state_metrics(scores_n: np.ndarray, scores_next: np.ndarray, B: int) -> dict:
+    """App. A.2 on consecutive oracle states.
+
+    ``scores_n``: layer-level scores of frame n over every token seen up to
+    and including frame n (positions 0 .. len - 1); ``scores_next``: those of
+    frame n + 1 over every token up to and including it, so the tokens of
+    frame n + 1 are the positions len(scores_n) .. len(scores_next) - 1.
+    S_n and S_{n+1} are the top-B sets of each; the candidate pool is
+    P_{n+1} = S_n + frame n + 1.  Returns recall |S_{n+1} & P| / |S_{n+1}|,
+    weighted recall (weights = scores_next), retention |S_n & S_{n+1}| / |S_n|
+    and churn |S_{n+1} - S_n| / |S_{n+1}|.
+    """
+    scores_next = np.asarray(scores_next, np.float64)
+    n_seen = len(scores_n)
+    s_n = set(top_b(scores_n, B).tolist())
+    s_next = set(top_b(scores_next, B).tolist())
+    pool = s_n | set(range(n_seen, len(scores_next)))
+    hit = s_next & pool
+    w_all = sum(scores_next[j] for j in s_next)
+    w_hit = sum(scores_next[j] for j in hit)
+    return {
+        "recall": len(hit) / len(s_next),
+        "weighted_recall": w_hit / w_all,
+        "retention": len(s_n & s_next) / len(s_n),
+        "churn": len(s_next - s_n) / len(s_next),
+    }

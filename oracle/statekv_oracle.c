@@ -111,15 +111,21 @@ int oracle_prefill_frame(int n_q, int n_kv, int d, int T, int B, int causal, dou
  *   policy 0  the method (Eq. 6): the B highest importances, ties to the
  *             older token;
  *   policy 1  the recency window of the ReKV-style baseline the paper compares
- *             with (Sec. 2, Sec. 4): the B most recent positions.
- * The attention and the importance are computed the same way for both.
+ *             with (Sec. 2, Sec. 4): the B most recent positions;
+ *   policy 2  layer-level selection: one ranking per layer by the attention
+ *             summed over all heads (the score of Sec. 3.3 aggregated over
+ *             heads, and the layer-level score of App. A.1), applied to every
+ *             KV head, which therefore all hold the same positions.  The
+ *             states given must already agree across heads (-1 otherwise).
+ * The attention and the per-KV-head importance are computed the same way for
+ * all three.
  */
 int oracle_prefill_frame_policy(int n_q, int n_kv, int d, int T, int B, int causal, double scale,
                                 int64_t virtual_len, const uint16_t* q, const uint16_t* k,
                                 const uint16_t* v, int32_t* count, int64_t* pos, uint16_t* sk,
                                 uint16_t* sv, double* out, double* imp, int32_t* kept, int policy)
 {
-    if (policy != 0 && policy != 1) return -1;
+    if (policy < 0 || policy > 2) return -1;
     if (n_q <= 0 || n_kv <= 0 || n_q % n_kv != 0 || d <= 0 || T <= 0 || B < 0) return -1;
     const int G = n_q / n_kv;
     const int P = B + T;
@@ -129,14 +135,27 @@ int oracle_prefill_frame_policy(int n_q, int n_kv, int d, int T, int B, int caus
     candidate* pool = (candidate*)malloc(sizeof(candidate) * (size_t)P);
     uint16_t* nk = (uint16_t*)malloc(sizeof(uint16_t) * (size_t)(B > 0 ? B : 1) * (size_t)d);
     uint16_t* nv = (uint16_t*)malloc(sizeof(uint16_t) * (size_t)(B > 0 ? B : 1) * (size_t)d);
-    if (!z || !qd || !pool || !nk || !nv) {
-        free(z); free(qd); free(pool); free(nk); free(nv);
+    double* shared = (double*)calloc((size_t)P, sizeof(double));
+    if (!z || !qd || !pool || !nk || !nv || !shared) {
+        free(z); free(qd); free(pool); free(nk); free(nv); free(shared);
         return -1;
     }
+    for (int h = 0; h < n_kv; ++h)
+        if (count[h] < 0 || count[h] > B) {
+            free(z); free(qd); free(pool); free(nk); free(nv); free(shared);
+            return -1;
+        }
+    if (policy == 2)
+        for (int h = 1; h < n_kv; ++h) {
+            int same = count[h] == count[0];
+            for (int c = 0; same && c < count[0]; ++c)
+                same = pos[(size_t)h * B + c] == pos[c];
+            if (!same) { free(z); free(qd); free(pool); free(nk); free(nv); free(shared); return -1; }
+        }
 
+    /* Attention and importance of every KV head. */
     for (int h = 0; h < n_kv; ++h) {
         const int b = count[h];
-        if (b < 0 || b > B) { free(z); free(qd); free(pool); free(nk); free(nv); return -1; }
         const uint16_t* hk = sk + (size_t)h * B * d;
         const uint16_t* hv = sv + (size_t)h * B * d;
         double* himp = imp + (size_t)h * P;
@@ -182,6 +201,20 @@ int oracle_prefill_frame_policy(int n_q, int n_kv, int d, int T, int B, int caus
                 }
             }
         }
+    }
+    /* Layer-level score: the importance summed over the KV heads (each already
+     * a sum over its query heads), column by column; the columns name the
+     * same positions in every head. */
+    if (policy == 2)
+        for (int h = 0; h < n_kv; ++h)
+            for (int c = 0; c < P; ++c) shared[c] += imp[(size_t)h * P + c];
+
+    /* Selection and gather, per KV head. */
+    for (int h = 0; h < n_kv; ++h) {
+        const int b = count[h];
+        const uint16_t* hk = sk + (size_t)h * B * d;
+        const uint16_t* hv = sv + (size_t)h * B * d;
+        const double* himp = policy == 2 ? shared : imp + (size_t)h * P;
 
         /* Eq. 6: pool = state entries + frame tokens; keep the B best. */
         int np = 0;
@@ -238,7 +271,7 @@ int oracle_prefill_frame_policy(int n_q, int n_kv, int d, int T, int B, int caus
         count[h] = nkeep;
     }
 
-    free(z); free(qd); free(pool); free(nk); free(nv);
+    free(z); free(qd); free(pool); free(nk); free(nv); free(shared);
     return 0;
 }
 
