@@ -82,7 +82,12 @@ typedef struct {
                                  1 = recency window, the B most recent tokens (the
                                      ReKV-style baseline the paper compares with);
                                      no importance is computed, so the per-call
-                                     importance pointer must be NULL */
+                                     importance pointer must be NULL;
+                                 2 = layer-level selection (App. A): one top-B per
+                                     (stream, layer) by the importance summed over
+                                     every KV head, applied to all KV heads, which
+                                     then hold the same positions; the exported
+                                     importance stays per KV head */
 } statekv_config;
 
 /* Bytes of device arena the configuration needs.  Returns INVALID_ARG or
@@ -129,6 +134,75 @@ statekv_status statekv_prefill_frame(statekv_handle* h, const statekv_frame_args
  * statekv_prefill_frame's does not. */
 statekv_status statekv_full_attention_frame(statekv_handle* h, const statekv_frame_args* args,
                                            statekv_stream stream);
+
+/* ---- App. A assumption diagnostics -------------------------------------
+ * The paper validates its two assumptions on the full-attention baseline
+ * (App. A): layer-level scores (attention summed over the frame's queries
+ * within each head, then over every head of the layer), the concentration
+ * C_{n,B} of historical attention in the top-B historical tokens (App. A.1),
+ * and the candidate-pool recall, weighted recall, retention and churn of
+ * consecutive top-B oracle states (App. A.2).  These calls compute the same
+ * quantities on device buffers; ratios are the quotients of the sums they
+ * return. */
+
+/* Device workspace (bytes) statekv_full_attention_scores needs for a call
+ * covering stream_count x layer_count (stream, layer) units: one fp32 partial
+ * per (unit, KV head, 128-query tile, key slot of max_frames * T + T). */
+statekv_status statekv_scores_workspace_bytes(const statekv_handle* h, int32_t stream_count,
+                                              int32_t layer_count, size_t* bytes);
+
+/* The exact full self-attention of the next frame, as
+ * statekv_full_attention_frame (out written the same way, states, caches and
+ * counters unchanged), plus App. A's layer-level score of every key:
+ *   scores[u][j] = sum over every query head of the layer and every query of
+ *                  the frame of the attention weight on key position j,
+ * for j < L_n + T (the frames processed so far, then the frame's own tokens),
+ * and 0 for j in [L_n + T, max_frames * T).
+ *   scores     fp32 [stream_count][layer_count][max_frames * T] (device, 4-byte
+ *              aligned)
+ *   workspace  device memory (16-byte aligned) of at least
+ *              statekv_scores_workspace_bytes() bytes; its contents are scratch
+ * args->importance must be NULL.  INVALID_ARG for bad arguments or a covered
+ * (stream, layer) that holds decoded tokens; CACHE_FULL if one already holds
+ * max_frames frames (the scores row would not fit the next frame). */
+statekv_status statekv_full_attention_scores(statekv_handle* h, const statekv_frame_args* args,
+                                             float* scores, void* workspace,
+                                             size_t workspace_bytes, statekv_stream stream);
+
+/* Top-B membership (the T_{n,B} of App. A.1 and the oracle states S_n of
+ * App. A.2): for each of `rows` rows, mask[r][j] = 1 for the min(B, n)
+ * highest scores among scores[r][0 .. n) -- ties to the lower position j --
+ * and 0 for every other j < row_stride.  Scores are attention sums, >= 0;
+ * negative entries and NaN rank as 0.
+ *   scores  fp32 [rows][row_stride] (device, 4-byte aligned)
+ *   mask    uint8 [rows][row_stride] (device)
+ * Needs 0 <= n <= row_stride <= 2^31 and B >= 0.  No handle: the call only
+ * enqueues one kernel on `stream`. */
+statekv_status statekv_topb_mask(const float* scores, int32_t rows, int64_t n, int64_t row_stride,
+                                 int64_t B, uint8_t* mask, statekv_stream stream);
+
+/* App. A.1 sums per row r (fp64 [rows][2], device):
+ *   out[r][0] = sum of scores[r][j] over j < n with mask[r][j] != 0
+ *   out[r][1] = sum of scores[r][j] over j < n
+ * With n = L_n (historical keys only) and mask from statekv_topb_mask over the
+ * same n, C_{n,B} = out[r][0] / out[r][1]. */
+statekv_status statekv_concentration_sums(const float* scores, const uint8_t* mask, int32_t rows,
+                                          int64_t n, int64_t row_stride, double* out,
+                                          statekv_stream stream);
+
+/* App. A.2 counts per row r (fp64 [rows][6], device), with
+ *   S_n  = { j < n_seen : mask_n[r][j] }          (top-B of frame n's scores)
+ *   S_n1 = { j < n_seen + T : mask_n1[r][j] }     (top-B of frame n+1's scores)
+ *   P    = S_n plus the positions [n_seen, n_seen + T) of frame n+1
+ *   w    = scores_n1[r]
+ * out[r] = { |S_n1 & P|, |S_n1|, w(S_n1 & P), w(S_n1), |S_n & S_n1|, |S_n| }:
+ * recall = out[0] / out[1], weighted recall = out[2] / out[3], retention =
+ * out[4] / out[5], churn = (out[1] - out[4]) / out[1].  All three inputs are
+ * [rows][row_stride] with n_seen + T <= row_stride. */
+statekv_status statekv_state_metrics(const uint8_t* mask_n, const uint8_t* mask_n1,
+                                     const float* scores_n1, int32_t rows, int64_t n_seen,
+                                     int32_t T, int64_t row_stride, double* out,
+                                     statekv_stream stream);
 
 /* Decoding over the detailed cache D_N (Sec. 3.2 / 3.3: decoding reads only
  * the detailed state; the compressed state is not used).  For every covered

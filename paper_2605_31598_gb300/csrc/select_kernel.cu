@@ -4,7 +4,10 @@
 //
 // K3 runs one CTA per (unit, KV head):
 //   1. importance of every pool member = the fixed-order sum of the attention
-//      kernel's per-query-tile partials (deterministic);
+//      kernel's per-query-tile partials (deterministic); with layer-level
+//      selection (App. A) the ranking score is the same sum taken over every
+//      KV head of the unit, in one fixed order, so all the unit's CTAs rank
+//      identically and their states keep the same positions;
 //   2. if the pool (count + T) fits in B, every frame token is admitted;
 //      otherwise the B best members by (score desc, position asc) are found
 //      with an MSB-first radix select over the 64-bit key
@@ -80,12 +83,23 @@ __global__ void __launch_bounds__(kSelThreads)
     const int n = count + T;
 
     // 1. importance (fixed-order sum over query tiles) and selection keys
+    const float* part0 = p.partials + static_cast<size_t>(u) * p.Hkv * p.MT * P;
     for (int i = tid; i < n; i += kSelThreads) {
         const int col = i < count ? i : B + (i - count);
         float s = 0.f;
         for (int mt = 0; mt < p.MT; ++mt) s += part[static_cast<size_t>(mt) * P + col];
+        float r = s;  // ranking score
+        if (p.shared) {
+            r = 0.f;
+            for (int h2 = 0; h2 < p.Hkv; ++h2) {
+                float sh = 0.f;
+                for (int mt = 0; mt < p.MT; ++mt)
+                    sh += part0[(static_cast<size_t>(h2) * p.MT + mt) * P + col];
+                r += sh;
+            }
+        }
         const int ps = i < count ? pos[i] : L + (i - count);
-        key[i] = (static_cast<uint64_t>(__float_as_uint(s)) << 32) |
+        key[i] = (static_cast<uint64_t>(__float_as_uint(r)) << 32) |
                  static_cast<uint32_t>(0xFFFFFFFFu - static_cast<uint32_t>(ps));
         if (imp_out) imp_out[col] = s;
     }

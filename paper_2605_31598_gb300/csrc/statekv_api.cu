@@ -46,7 +46,7 @@ statekv_status check_config(const statekv_config* c, Derived* d)
         c->state_capacity < 0 || c->max_frames < 1 ||
         (c->causal_in_frame != 0 && c->causal_in_frame != 1) ||
         (c->host_staging != 0 && c->host_staging != 1) ||
-        (c->selection != 0 && c->selection != 1) || !(c->softmax_scale >= 0.f) ||
+        (c->selection < 0 || c->selection > 2) || !(c->softmax_scale >= 0.f) ||
         !std::isfinite(c->softmax_scale))
         return STATEKV_ERR_INVALID_ARG;
     if (static_cast<long long>(c->max_frames) * c->tokens_per_frame > 0x7FFFFFFFll)
@@ -246,7 +246,7 @@ statekv_status run_step(statekv_handle* h, const statekv_frame_args& a, cudaStre
     AttnParams pa{};
     pa.q = static_cast<const __nv_bfloat16*>(a.q);
     pa.out = static_cast<__nv_bfloat16*>(a.out);
-    pa.partials = c.selection == 0 ? partials : nullptr;  // recency: no importance
+    pa.partials = c.selection != 1 ? partials : nullptr;  // recency: no importance
     pa.counts = counts;
     pa.status = h->status_dev;
     pa.units = ur;
@@ -301,6 +301,7 @@ statekv_status run_step(statekv_handle* h, const statekv_frame_args& a, cudaStre
     ps.B = c.state_capacity;
     ps.P = d.P;
     ps.MT = d.MT;
+    ps.shared = c.selection == 2 ? 1 : 0;
     if (timed(h, 2, st, [&] { return launch_select(ps, U, st); }) != cudaSuccess)
         return STATEKV_ERR_CUDA;
     }
@@ -315,7 +316,8 @@ statekv_status run_step(statekv_handle* h, const statekv_frame_args& a, cudaStre
 // (the frames processed so far, all visible) followed by the frame's own
 // tokens (causal as configured): the attention kernel with the cache as its
 // key prefix, no importance, no change to any state.
-statekv_status run_full(statekv_handle* h, const statekv_frame_args& a, cudaStream_t st)
+statekv_status run_full(statekv_handle* h, const statekv_frame_args& a, cudaStream_t st,
+                        float* partials = nullptr, long long Bp = 0)
 {
     const statekv_config& c = h->cfg;
     const Derived& d = h->d;
@@ -336,7 +338,7 @@ statekv_status run_full(statekv_handle* h, const statekv_frame_args& a, cudaStre
     AttnParams pa{};
     pa.q = static_cast<const __nv_bfloat16*>(a.q);
     pa.out = static_cast<__nv_bfloat16*>(a.out);
-    pa.partials = nullptr;
+    pa.partials = partials;  // with partials: key j of the cache at column j, frame token t at Bp + t
     pa.counts = h->at<int32_t>(h->lay.frames);  // keys = frames * T + text rows
     pa.count_add = h->at<int32_t>(h->lay.text);
     pa.status = h->status_dev;
@@ -345,8 +347,8 @@ statekv_status run_full(statekv_handle* h, const statekv_frame_args& a, cudaStre
     pa.Hq = c.num_q_heads;
     pa.Hkv = Hkv;
     pa.G = d.G;
-    pa.B = 1;  // no importance pool
-    pa.P = 0;
+    pa.B = partials ? static_cast<int>(Bp) : 1;  // 1: no importance pool
+    pa.P = partials ? static_cast<int>(Bp + T) : 0;
     pa.MT = d.MT;
     pa.causal = c.causal_in_frame;
     pa.count_mul = T;
@@ -533,6 +535,104 @@ statekv_status statekv_full_attention_frame(statekv_handle* h, const statekv_fra
     if (s != STATEKV_OK) return s;
     if (args->importance) return STATEKV_ERR_INVALID_ARG;
     return run_full(h, *args, reinterpret_cast<cudaStream_t>(stream));
+}
+
+namespace {
+
+// Columns of the attention kernel's partials in scores mode: every cache row
+// (max_frames * T) then the frame's tokens.
+long long scores_bp(const statekv_config& c)
+{
+    return static_cast<long long>(c.max_frames) * c.tokens_per_frame;
+}
+
+}  // namespace
+
+statekv_status statekv_scores_workspace_bytes(const statekv_handle* h, int32_t stream_count,
+                                              int32_t layer_count, size_t* bytes)
+{
+    if (!h || !bytes || stream_count < 1 || layer_count < 1 ||
+        stream_count > h->cfg.num_streams || layer_count > h->cfg.num_layers)
+        return STATEKV_ERR_INVALID_ARG;
+    const long long pp = scores_bp(h->cfg) + h->cfg.tokens_per_frame;
+    if (pp > 0x7FFFFFFFll) return STATEKV_ERR_UNSUPPORTED;
+    *bytes = static_cast<size_t>(stream_count) * layer_count * h->cfg.num_kv_heads * h->d.MT *
+             static_cast<size_t>(pp) * sizeof(float);
+    return STATEKV_OK;
+}
+
+statekv_status statekv_full_attention_scores(statekv_handle* h, const statekv_frame_args* args,
+                                             float* scores, void* workspace,
+                                             size_t workspace_bytes, statekv_stream stream)
+{
+    const statekv_status s = check_args(h, args, false);
+    if (s != STATEKV_OK) return s;
+    if (args->importance || !scores || !workspace || !aligned(scores, 4) || !aligned(workspace, 16))
+        return STATEKV_ERR_INVALID_ARG;
+    size_t need = 0;
+    const statekv_status w = statekv_scores_workspace_bytes(h, args->stream_count,
+                                                            args->layer_count, &need);
+    if (w != STATEKV_OK) return w;
+    if (workspace_bytes < need) return STATEKV_ERR_INVALID_ARG;
+    const statekv_config& c = h->cfg;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    const long long bp = scores_bp(c);
+    float* part = static_cast<float*>(workspace);
+    const statekv_status r = run_full(h, *args, st, part, bp);
+    if (r != STATEKV_OK) return r;
+    ScoresParams sp{};
+    sp.partials = part;
+    sp.scores = scores;
+    sp.frames = h->at<int32_t>(h->lay.frames);
+    sp.units = UnitRange{args->stream_begin, args->layer_begin, args->layer_count, c.num_layers};
+    sp.T = c.tokens_per_frame;
+    sp.Hkv = c.num_kv_heads;
+    sp.MT = h->d.MT;
+    sp.Bp = bp;
+    sp.Pp = bp + c.tokens_per_frame;
+    sp.ncols = bp;
+    if (launch_scores_reduce(sp, args->stream_count * args->layer_count, st) != cudaSuccess)
+        return STATEKV_ERR_CUDA;
+    return STATEKV_OK;
+}
+
+statekv_status statekv_topb_mask(const float* scores, int32_t rows, int64_t n, int64_t row_stride,
+                                 int64_t B, uint8_t* mask, statekv_stream stream)
+{
+    if (!scores || !mask || !aligned(scores, 4) || rows < 0 || rows > 0x7FFFFFFF || n < 0 ||
+        row_stride < n || row_stride > (1ll << 31) || B < 0)
+        return STATEKV_ERR_INVALID_ARG;
+    if (launch_topb_mask(scores, rows, n, row_stride, B, mask,
+                         reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess)
+        return STATEKV_ERR_CUDA;
+    return STATEKV_OK;
+}
+
+statekv_status statekv_concentration_sums(const float* scores, const uint8_t* mask, int32_t rows,
+                                          int64_t n, int64_t row_stride, double* out,
+                                          statekv_stream stream)
+{
+    if (!scores || !mask || !out || !aligned(scores, 4) || !aligned(out, 8) || rows < 0 || n < 0 ||
+        row_stride < n)
+        return STATEKV_ERR_INVALID_ARG;
+    if (launch_concentration(scores, mask, rows, n, row_stride, out,
+                             reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess)
+        return STATEKV_ERR_CUDA;
+    return STATEKV_OK;
+}
+
+statekv_status statekv_state_metrics(const uint8_t* mask_n, const uint8_t* mask_n1,
+                                     const float* scores_n1, int32_t rows, int64_t n_seen,
+                                     int32_t T, int64_t row_stride, double* out,
+                                     statekv_stream stream)
+{
+    if (!mask_n || !mask_n1 || !scores_n1 || !out || !aligned(scores_n1, 4) || !aligned(out, 8) ||
+        rows < 0 || n_seen < 0 || T < 0 || n_seen + T > row_stride)
+        return STATEKV_ERR_INVALID_ARG;
+    if (launch_state_metrics(mask_n, mask_n1, scores_n1, rows, n_seen, T, row_stride, out,
+                             reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess)
+        return STATEKV_ERR_CUDA;
+    return STATEKV_OK;
 }
 
 statekv_status statekv_decode_step(statekv_handle* h, const statekv_decode_args* a,

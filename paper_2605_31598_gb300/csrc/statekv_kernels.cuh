@@ -69,6 +69,7 @@ struct SelectParams {
     int32_t* status;
     UnitRange units;
     int T, Hkv, D, B, P, MT;
+    int shared;                 // 1: rank by the importance summed over every KV head
 };
 
 struct AppendParams {
@@ -95,6 +96,26 @@ struct RecencyParams {
     UnitRange units;
     int U, T, Hkv, D, B;
 };
+
+struct ScoresParams {
+    const float* partials;      // [U][Hkv][MT][Pp] from the attention kernel
+    float* scores;              // [U][ncols]
+    const int32_t* frames;      // arena [S*L][Hkv]: frames before this one
+    UnitRange units;
+    int T, Hkv, MT;
+    long long Bp, Pp;           // frame keys sit at partial columns Bp + t; Pp = Bp + T
+    long long ncols;            // row length of scores (>= keys of every unit)
+};
+
+// App. A diagnostics (diag_kernel.cu).
+cudaError_t launch_scores_reduce(const ScoresParams& p, int U, cudaStream_t st);
+cudaError_t launch_topb_mask(const float* scores, int rows, long long n, long long stride,
+                             long long B, uint8_t* mask, cudaStream_t st);
+cudaError_t launch_concentration(const float* scores, const uint8_t* mask, int rows, long long n,
+                                 long long stride, double* out, cudaStream_t st);
+cudaError_t launch_state_metrics(const uint8_t* mask_n, const uint8_t* mask_n1, const float* w,
+                                 int rows, long long n_seen, int T, long long stride, double* out,
+                                 cudaStream_t st);
 
 // Recency-window state update (the baseline): the frame's tokens enter ring
 // slots position mod B, overwriting the tokens that leave the window.

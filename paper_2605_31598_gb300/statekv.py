@@ -26,6 +26,8 @@ EXPORTED = ("statekv_arena_bytes", "statekv_init", "statekv_prefill_frame",
             "statekv_state_view", "statekv_cache_view",
             "statekv_profile_enable", "statekv_profile_read", "statekv_sync",
             "statekv_device_error", "statekv_frame_attention_noalloc",
+            "statekv_scores_workspace_bytes", "statekv_full_attention_scores",
+            "statekv_topb_mask", "statekv_concentration_sums", "statekv_state_metrics",
             "statekv_destroy", "statekv_status_string")
 
 
@@ -117,6 +119,26 @@ def lib() -> ctypes.CDLL:
                 ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int32, ctypes.c_void_p,
                 ctypes.c_void_p, ctypes.c_void_p]
             L.statekv_frame_attention_noalloc.restype = st
+            L.statekv_scores_workspace_bytes.argtypes = [ctypes.c_void_p, ctypes.c_int32,
+                                                         ctypes.c_int32, P(ctypes.c_size_t)]
+            L.statekv_scores_workspace_bytes.restype = st
+            L.statekv_full_attention_scores.argtypes = [
+                ctypes.c_void_p, P(statekv_frame_args), ctypes.c_void_p, ctypes.c_void_p,
+                ctypes.c_size_t, ctypes.c_void_p]
+            L.statekv_full_attention_scores.restype = st
+            L.statekv_topb_mask.argtypes = [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64,
+                                            ctypes.c_int64, ctypes.c_int64, ctypes.c_void_p,
+                                            ctypes.c_void_p]
+            L.statekv_topb_mask.restype = st
+            L.statekv_concentration_sums.argtypes = [ctypes.c_void_p, ctypes.c_void_p,
+                                                     ctypes.c_int32, ctypes.c_int64,
+                                                     ctypes.c_int64, ctypes.c_void_p,
+                                                     ctypes.c_void_p]
+            L.statekv_concentration_sums.restype = st
+            L.statekv_state_metrics.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
+                                                ctypes.c_int32, ctypes.c_int64, ctypes.c_int32,
+                                                ctypes.c_int64, ctypes.c_void_p, ctypes.c_void_p]
+            L.statekv_state_metrics.restype = st
             L.statekv_destroy.argtypes = [ctypes.c_void_p]
             L.statekv_destroy.restype = None
             L.statekv_status_string.argtypes = [ctypes.c_int]
@@ -212,6 +234,40 @@ def statekv_frame_attention_noalloc(cfg: statekv_config, q: int, k: int, v: int,
         ctypes.c_void_p(importance), ctypes.c_void_p(stream))
 
 
+def statekv_scores_workspace_bytes(handle: int, stream_count: int, layer_count: int) -> int:
+    n = ctypes.c_size_t(0)
+    check(lib().statekv_scores_workspace_bytes(handle, stream_count, layer_count, ctypes.byref(n)),
+          "statekv_scores_workspace_bytes")
+    return n.value
+
+
+def statekv_full_attention_scores(handle: int, args: statekv_frame_args, scores: int,
+                                  workspace: int, workspace_bytes: int, stream: int) -> int:
+    return lib().statekv_full_attention_scores(handle, ctypes.byref(args), ctypes.c_void_p(scores),
+                                               ctypes.c_void_p(workspace), workspace_bytes,
+                                               ctypes.c_void_p(stream))
+
+
+def statekv_topb_mask(scores: int, rows: int, n: int, row_stride: int, B: int, mask: int,
+                      stream: int) -> int:
+    return lib().statekv_topb_mask(ctypes.c_void_p(scores), rows, n, row_stride, B,
+                                   ctypes.c_void_p(mask), ctypes.c_void_p(stream))
+
+
+def statekv_concentration_sums(scores: int, mask: int, rows: int, n: int, row_stride: int,
+                               out: int, stream: int) -> int:
+    return lib().statekv_concentration_sums(ctypes.c_void_p(scores), ctypes.c_void_p(mask), rows,
+                                            n, row_stride, ctypes.c_void_p(out),
+                                            ctypes.c_void_p(stream))
+
+
+def statekv_state_metrics(mask_n: int, mask_n1: int, scores_n1: int, rows: int, n_seen: int,
+                          T: int, row_stride: int, out: int, stream: int) -> int:
+    return lib().statekv_state_metrics(ctypes.c_void_p(mask_n), ctypes.c_void_p(mask_n1),
+                                       ctypes.c_void_p(scores_n1), rows, n_seen, T, row_stride,
+                                       ctypes.c_void_p(out), ctypes.c_void_p(stream))
+
+
 def statekv_destroy(handle: int):
     lib().statekv_destroy(handle)
 
@@ -223,6 +279,7 @@ def statekv_status_string(status: int) -> str:
 # ---------------------------------------------------------------- owner object
 SELECTION_IMPORTANCE = 0  # the method: top-B by importance (Eq. 6)
 SELECTION_RECENCY = 1     # the baseline: the B most recent tokens
+SELECTION_LAYER = 2       # App. A: one top-B per layer by the importance summed over heads
 
 
 def make_config(shape, *, causal=True, host_staging=False, softmax_scale=0.0,
@@ -286,6 +343,27 @@ class StateKV:
         st = (stream or torch.cuda.current_stream()).cuda_stream
         args = self._args(q, k, v, out, None, stream_begin, sc, layer_begin, lc)
         return statekv_full_attention_frame(self.handle, args, st)
+
+    def full_attention_scores(self, q, k, v, out, scores, workspace, *, stream_begin=0,
+                              stream_count=None, layer_begin=0, layer_count=None,
+                              stream=None) -> int:
+        """Full self-attention of the next frame plus App. A's layer-level score
+        of every key into ``scores`` (fp32 [S][L][max_frames * T]);
+        ``workspace``: a uint8 device tensor of ``scores_workspace_bytes``.
+        Changes no state.  Returns the C status."""
+        import torch
+
+        sc = self.cfg.num_streams - stream_begin if stream_count is None else stream_count
+        lc = self.cfg.num_layers - layer_begin if layer_count is None else layer_count
+        st = (stream or torch.cuda.current_stream()).cuda_stream
+        args = self._args(q, k, v, out, None, stream_begin, sc, layer_begin, lc)
+        return statekv_full_attention_scores(self.handle, args, scores.data_ptr(),
+                                             workspace.data_ptr(), workspace.numel(), st)
+
+    def scores_workspace_bytes(self, stream_count=None, layer_count=None) -> int:
+        sc = self.cfg.num_streams if stream_count is None else stream_count
+        lc = self.cfg.num_layers if layer_count is None else layer_count
+        return statekv_scores_workspace_bytes(self.handle, sc, lc)
 
     def decode_step(self, q, k, v, out, *, stream_begin=0, stream_count=None, layer_begin=0,
                     layer_count=None, stream=None) -> int:

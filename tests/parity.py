@@ -35,24 +35,28 @@ def _bits(t):
 
 def run_parity(shape, nframes, *, kind=None, seed=0, check_frames=None, causal=True,
                units=None, call_layers=None, want_importance=True, host_api=False,
-               stats=None):
+               stats=None, selection=0):
     """Run ``nframes`` frames on the GPU; compare the frames in ``check_frames``.
 
     units: (stream, layer) pairs to compare (default: all).  call_layers:
     split each frame into calls over these layer ranges [(begin, count), ...].
+    selection: 0 the per-KV-head top-B (Eq. 6), 2 the layer-level top-B
+    (App. A), whose ranking score is the importance summed over the KV heads
+    and whose kept positions must agree across heads.
     Returns the StateKV engine (for extra checks by the caller).
     """
     S, L = shape.num_streams, shape.num_layers
     T, Hq, Hkv, d, B = (shape.tokens_per_frame, shape.num_q_heads, shape.num_kv_heads,
                         shape.head_dim, shape.state_capacity)
     G = Hq // Hkv
-    eng = StateKV(make_config(shape, causal=causal, host_staging=host_api))
+    eng = StateKV(make_config(shape, causal=causal, host_staging=host_api, selection=selection))
     units = units or [(s, l) for s in range(S) for l in range(L)]
     check_frames = set(range(1, nframes + 1) if check_frames is None else check_frames)
     call_layers = call_layers or [(0, L)]
     hist_k = {u: [] for u in units}
     hist_v = {u: [] for u in units}
-    lays = {u: oracle.OracleLayer(Hq, Hkv, d, T, B, shape.max_frames, causal=causal)
+    lays = {u: oracle.OracleLayer(Hq, Hkv, d, T, B, shape.max_frames, causal=causal,
+                                  policy=selection)
             for u in units}
     stats = stats if stats is not None else {}
     stats.setdefault("max_out_err", 0.0)
@@ -116,6 +120,10 @@ def run_parity(shape, nframes, *, kind=None, seed=0, check_frames=None, causal=T
             post_k, post_v = _bits(kk), _bits(vv)
             allk = np.concatenate(hist_k[u])  # [n*T][Hkv][d]
             allv = np.concatenate(hist_v[u])
+            rank_score = imp_ref.sum(axis=0) if selection == 2 else None  # layer level
+            if selection == 2:
+                heads = [sorted(post_pos[h][post_pos[h] >= 0].tolist()) for h in range(Hkv)]
+                assert all(x == heads[0] for x in heads), f"frame {n} unit {u}: heads disagree"
             for h in range(Hkv):
                 # importance: map GPU slot j -> oracle column (position order)
                 order = {int(p): i for i, p in enumerate(np.sort(ppos[h, :count]))}
@@ -142,7 +150,8 @@ def run_parity(shape, nframes, *, kind=None, seed=0, check_frames=None, causal=T
                 assert len(set(gpos.tolist())) == len(gpos), f"frame {n} unit {u}: duplicate"
                 gset = set(int(x) for x in gpos)
                 cand_pos = np.concatenate([np.sort(ppos[h, :count]), vlen + np.arange(T)])
-                cand_score = np.concatenate([imp_ref[h, :count], imp_ref[h, B:]])
+                rs = imp_ref[h] if rank_score is None else rank_score
+                cand_score = np.concatenate([rs[:count], rs[B:]])
                 cand_kept = np.concatenate([kept_ref[h, :count], kept_ref[h, B:]]).astype(bool)
                 if count + T > B and B > 0:
                     tau = np.sort(cand_score)[::-1][B - 1]

@@ -64,7 +64,8 @@ def _cfg(**kw):
     (dict(state_capacity=-1), 1),
     (dict(max_frames=0), 1),
     (dict(causal_in_frame=2), 1),
-    (dict(selection=2), 1),               # neither top-B importance nor recency
+    (dict(selection=3), 1),               # no such selection policy
+    (dict(selection=-1), 1),
     (dict(softmax_scale=-1.0), 1),
     (dict(state_capacity=30000), 2),      # pool beyond the select kernel's limit
     (dict(tokens_per_frame=5000), 2),
@@ -100,3 +101,21 @@ def test_null_arguments_rejected(lib):
     assert lib.statekv_state_view(None, 0, 0, None) == 1
     assert lib.statekv_cache_view(None, 0, 0, None) == 1
     lib.statekv_destroy(None)
+
+
+def test_diagnostics_arguments_rejected_on_host(lib):
+    """Bad pointers or sizes come back as INVALID_ARG before any launch (the
+    dummy addresses below are never dereferenced)."""
+    fake = 1 << 20  # 16-byte aligned, never touched
+    assert statekv.statekv_topb_mask(0, 1, 10, 16, 4, fake, 0) == 1        # null scores
+    assert statekv.statekv_topb_mask(fake, 1, 10, 16, 4, 0, 0) == 1        # null mask
+    assert statekv.statekv_topb_mask(fake, 1, 20, 16, 4, fake, 0) == 1     # n > row_stride
+    assert statekv.statekv_topb_mask(fake, 1, 10, 16, -1, fake, 0) == 1    # B < 0
+    assert statekv.statekv_topb_mask(fake + 2, 1, 10, 16, 4, fake, 0) == 1  # misaligned
+    assert statekv.statekv_concentration_sums(fake, fake, 1, 20, 16, fake, 0) == 1
+    assert statekv.statekv_concentration_sums(fake, fake, 1, 10, 16, fake + 4, 0) == 1
+    assert statekv.statekv_state_metrics(fake, fake, fake, 1, 10, 7, 16, fake, 0) == 1
+    assert statekv.statekv_state_metrics(fake, 0, fake, 1, 4, 4, 16, fake, 0) == 1
+    assert lib.statekv_full_attention_scores(None, None, None, None, 0, None) == 1
+    n = ctypes.c_size_t(0)
+    assert lib.statekv_scores_workspace_bytes(None, 1, 1, ctypes.byref(n)) == 1
