@@ -292,11 +292,11 @@ def run_ours(args, world, rank, local):
     log(f"[bench] rank {rank}: generating {nframes} frames of {args.workload} inputs")
     frames = [batch_qkv(shape, n, streams=range(S), layers=range(L), seed=seed, device=device)
               for n in range(1, nframes + 1)]
-    sel = 1 if args.selection == "recency" else 0
+    sel = SELECTIONS[args.selection]
     eng = StateKV(make_config(shape, selection=sel))
     out = torch.empty_like(frames[0][0])
     imp = (torch.empty((S, L, Hkv, B + T), dtype=torch.float32, device=device)
-           if sel == 0 else None)
+           if sel != 1 else None)
 
     def step(n):
         q, k, v = frames[n]
@@ -390,8 +390,7 @@ def run_ours(args, world, rank, local):
         "dtype": "bf16",
         "data": "synthetic",
         "config": {"workload": WORKLOAD_TEXT[args.workload], "streams": S, "layers": L,
-                   "selection": ("top-B importance (the method)" if sel == 0 else
-                                 "recency window (baseline; no importance)"),
+                   "selection": SELECTION_TEXT[sel],
                    "steady_state_frames": f"{fill + args.warmup + 1}..{nframes}",
                    "l2": "no flush: each step reads fresh Q/K/V and the full state "
                          f"(~{(2 * S * L * Hkv * B * d * 2 + S * L * T * (shape.num_q_heads + 2 * Hkv) * d * 2) / 1e6:.0f} MB "
@@ -447,10 +446,10 @@ def run_e2e(args, shape, fill, seed, device, frames):
     steps = min(args.steps, 64)
     n_total = fill + args.warmup + steps
     host = [tuple(x.cpu().pin_memory() for x in frames[n]) for n in range(n_total)]
-    sel = 1 if args.selection == "recency" else 0
+    sel = SELECTIONS[args.selection]
     out_h = torch.empty(host[0][0].shape, dtype=torch.bfloat16).pin_memory()
     imp_h = (torch.empty((S, L, Hkv, B + T), dtype=torch.float32).pin_memory()
-             if sel == 0 else None)
+             if sel != 1 else None)
     eng = StateKV(make_config(shape, host_staging=True, selection=sel))
 
     def step(n):
@@ -644,6 +643,93 @@ def run_decode(args, local):
     print(json.dumps(line), flush=True)
 
 
+def run_diagnostics(args, local):
+    """App. A's assumption statistics on the full-attention baseline, on
+    synthetic inputs of the workload's shape: every frame runs through the
+    method (filling the decode cache); at sampled frames n the full-attention
+    scores pass runs for frames n and n + 1 of every layer, then the
+    concentration C_{n,B} (App. A.1) and the candidate-pool recall, weighted
+    recall, retention and churn (App. A.2) for the paper's budgets.  Prints one
+    JSON line with the means over sampled frames and layers and the device
+    times of the passes."""
+    import numpy as np
+    import torch
+
+    from paper_2605_31598_gb300 import StateKV, diagnostics, make_config
+    from paper_2605_31598_gb300.inputs import WORKLOADS, batch_qkv
+
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py needs a CUDA device (no CPU fallback exists)")
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    base = WORKLOADS[args.workload]
+    N = args.frames or 128
+    shape = dataclasses.replace(base, max_frames=N + 1, num_streams=1)
+    S, L, T = 1, shape.num_layers, shape.tokens_per_frame
+    budgets = [1, 4, 16, 64, 256, 1024, 4096, 16384]
+    sample = sorted({n for n in range(8, N, max(1, N // 8))} | {N - 1})
+    eng = StateKV(make_config(shape))
+    cap = shape.max_frames * T
+    ws = torch.empty(eng.scores_workspace_bytes(), dtype=torch.uint8, device=device)
+    st = torch.cuda.current_stream()
+    conc, a2, t_scores, t_stats = [], {b: [] for b in budgets}, [], []
+
+    def scores_of(q, k, v):
+        sc = torch.empty((S, L, cap), dtype=torch.float32, device=device)
+        out = torch.empty_like(q)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(st)
+        if eng.full_attention_scores(q, k, v, out, sc, ws) != 0:
+            raise RuntimeError("statekv_full_attention_scores failed")
+        e1.record(st)
+        torch.cuda.synchronize()
+        t_scores.append(e0.elapsed_time(e1))
+        return sc[0]
+
+    prev = None
+    for n in range(1, N + 1):
+        q, k, v = batch_qkv(shape, n, streams=[0], layers=range(L), seed=args.seed, device=device)
+        if n in sample or (n - 1) in sample:
+            sc = scores_of(q, k, v)
+            if n in sample:
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record(st)
+                conc.append(diagnostics.concentration(sc, (n - 1) * T, budgets))
+                e1.record(st)
+                torch.cuda.synchronize()
+                t_stats.append(e0.elapsed_time(e1))
+            if (n - 1) in sample and prev is not None:
+                for b in budgets:
+                    m = diagnostics.state_metrics(prev, sc, (n - 1) * T, T, b)
+                    a2[b].append(np.stack([m["recall"], m["weighted_recall"], m["retention"],
+                                           m["churn"]]))
+            prev = sc if n in sample else None
+        if eng.prefill_frame(q, k, v, torch.empty_like(q)) != 0:
+            raise RuntimeError(f"prefill failed at frame {n}")
+    assert eng.sync() == 0
+    c = np.concatenate(conc)  # [frames * layers][budgets]
+    line = {
+        "diagnostics": WORKLOAD_TEXT[args.workload],
+        "data": "synthetic (the values describe random inputs, not videos)",
+        "frames": N, "sampled_frames": sample, "budgets": budgets,
+        "concentration_mean": [float(x) for x in c.mean(axis=0)],
+        "recall_mean": [float(np.mean([x[0] for x in a2[b]])) for b in budgets],
+        "weighted_recall_mean": [float(np.mean([x[1] for x in a2[b]])) for b in budgets],
+        "retention_mean": [float(np.mean([x[2] for x in a2[b]])) for b in budgets],
+        "churn_mean": [float(np.mean([x[3] for x in a2[b]])) for b in budgets],
+        "scores_pass_ms_last": t_scores[-1],
+        "scores_pass_keys_last": (sample[-1] + 1) * T,
+        "concentration_all_budgets_ms_last": t_stats[-1],
+    }
+    print(json.dumps(line), flush=True)
+
+
+SELECTIONS = {"importance": 0, "recency": 1, "layer": 2}
+SELECTION_TEXT = {0: "top-B importance per KV head (the method)",
+                  1: "recency window (baseline; no importance)",
+                  2: "top-B of the layer-level importance, shared by the KV heads (App. A)"}
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__)
     ap.add_argument("--gpus", type=int, default=1)
@@ -657,9 +743,11 @@ def main():
     ap.add_argument("--max-frames", type=int, default=0,
                     help="decode-cache capacity in frames (default: the workload's); "
                          "a small value keeps the arena small for profiler captures")
-    ap.add_argument("--selection", choices=["importance", "recency"], default="importance",
-                    help="state policy: the method's top-B importance, or the recency-window "
-                         "baseline")
+    ap.add_argument("--selection", choices=sorted(SELECTIONS), default="importance",
+                    help="state policy: the method's top-B importance per KV head, the "
+                         "recency-window baseline, or the layer-level top-B of App. A")
+    ap.add_argument("--diagnostics", action="store_true",
+                    help="App. A assumption statistics on the full-attention baseline")
     ap.add_argument("--curve", action="store_true",
                     help="per-frame cost vs frame index, StateKV next to exact full attention")
     ap.add_argument("--frames", type=int, default=0, help="--curve: frames to run (default: "
@@ -673,6 +761,9 @@ def main():
         return
     if args.curve:
         run_curve(args, int(os.environ.get("LOCAL_RANK", 0)))
+        return
+    if args.diagnostics:
+        run_diagnostics(args, int(os.environ.get("LOCAL_RANK", 0)))
         return
     if args.warmup < 3:
         raise SystemExit("--warmup must be at least 3")
