@@ -724,6 +724,89 @@ def run_diagnostics(args, local):
     print(json.dumps(line), flush=True)
 
 
+def run_block(args, local):
+    """The full per-frame transformer block (synthetic random-init weights of
+    the workload's layer widths, Qwen2-7B: hidden 3584, MLP 18944): every
+    frame runs all layers in order -- RMSNorm, QKV projection + RoPE at the
+    virtual positions, the StateKV step, output projection, SiLU MLP -- so
+    the layers are sequential, as in a real model.  Times steady-state frames
+    with CUDA events; the library's profile splits the time by kind.  Prints
+    one JSON line."""
+    import numpy as np
+    import torch
+
+    from paper_2605_31598_gb300 import StateKV, make_config
+    from paper_2605_31598_gb300.inputs import BLOCKS, WORKLOADS, block_input, block_weights
+    from paper_2605_31598_gb300.statekv import block_weights_array, statekv_block_config
+
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py needs a CUDA device (no CPU fallback exists)")
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    base = WORKLOADS[args.workload]
+    S = args.streams or base.num_streams
+    T, B, L = base.tokens_per_frame, base.state_capacity, base.num_layers
+    Hq, Hkv, d = base.num_q_heads, base.num_kv_heads, base.head_dim
+    fill = math.ceil(B / T) if B > 0 else 0
+    steps = min(args.steps, 40)
+    nframes = fill + args.warmup + steps
+    shape = dataclasses.replace(base, max_frames=nframes, num_streams=S)
+    blk = BLOCKS["qwen7b"]
+    H, I = blk.hidden, blk.intermediate
+    eng = StateKV(make_config(shape))
+    bc = statekv_block_config(H, I, blk.rms_eps, blk.rope_theta, 1.0, 0)
+    wts = block_weights(shape, blk, device=device)
+    warr = block_weights_array(wts)
+    ws = torch.empty(eng.block_workspace_bytes(bc), dtype=torch.uint8, device=device)
+    xs = [block_input(shape, blk, n, device=device) for n in range(1, nframes + 1)]
+    y = torch.empty_like(xs[0])
+    st = torch.cuda.current_stream()
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    for n in range(fill + args.warmup):
+        if eng.block_frame(bc, warr, xs[n], y, ws) != 0:
+            raise RuntimeError(f"statekv_block_frame failed at frame {n + 1}")
+    torch.cuda.synchronize()
+    eng.profile(True)
+    for i in range(steps):
+        starts[i].record(st)
+        if eng.block_frame(bc, warr, xs[fill + args.warmup + i], y, ws) != 0:
+            raise RuntimeError("statekv_block_frame failed")
+        ends[i].record(st)
+    torch.cuda.synchronize()
+    prof = eng.profile_read()
+    eng.profile(False)
+    assert eng.sync() == 0
+    ms = sorted(a.elapsed_time(b) for a, b in zip(starts, ends))
+    p50 = ms[len(ms) // 2]
+    per = lambda k: prof[k][1] / steps
+    weight_bytes = L * 2 * (H * (Hq + 2 * Hkv) * d + (Hq + 2 * Hkv) * d + H * Hq * d
+                            + 2 * I * H + H * I)
+    gemm_flops = 2 * S * T * L * (H * (Hq + 2 * Hkv) * d + H * Hq * d + 3 * I * H)
+    attn_flops = L * S * 4 * d * Hq * (T * B + T * (T + 1) / 2)
+    hbm, tf_burst, _, _ = peaks()
+    line = {
+        "block": WORKLOAD_TEXT[args.workload] + "; decoder layer: hidden 3584, MLP 18944, "
+                 "QKV bias, RMSNorm, RoPE theta 1e6, SiLU MLP (synthetic random-init weights)",
+        "streams": S,
+        "frames_timed": steps,
+        "p50_us_per_frame": 1e3 * p50,
+        "frames_per_s": 1e3 / p50,
+        "ms_per_frame_by_kind": {"projection_gemms": per(3), "attention_importance": per(1),
+                                 "select_gather": per(2), "cache_append": per(0),
+                                 "norm_rope_silu": per(4)},
+        "gemm_weight_bytes_per_frame": weight_bytes,
+        "gemm_weight_read_gbs": weight_bytes / (per(3) * 1e-3) / 1e9,
+        "gemm_weight_read_frac_of_hbm": weight_bytes / (per(3) * 1e-3) / 1e9 / hbm,
+        "gemm_tflops": gemm_flops / (per(3) * 1e-3) / 1e12,
+        "attention_tflops": attn_flops / (per(1) * 1e-3) / 1e12,
+        "note": "layers run in sequence (layer l+1 reads layer l's output); at one stream the "
+                "projections read every weight once per frame for 196 rows, so they are "
+                "bound by HBM bandwidth, not by the tensor cores",
+    }
+    print(json.dumps(line), flush=True)
+
+
 SELECTIONS = {"importance": 0, "recency": 1, "layer": 2}
 SELECTION_TEXT = {0: "top-B importance per KV head (the method)",
                   1: "recency window (baseline; no importance)",
@@ -748,6 +831,10 @@ def main():
                          "recency-window baseline, or the layer-level top-B of App. A")
     ap.add_argument("--diagnostics", action="store_true",
                     help="App. A assumption statistics on the full-attention baseline")
+    ap.add_argument("--block", action="store_true",
+                    help="the full per-frame transformer block (all layers in sequence)")
+    ap.add_argument("--streams", type=int, default=0,
+                    help="--block: streams per call (default: the workload's)")
     ap.add_argument("--curve", action="store_true",
                     help="per-frame cost vs frame index, StateKV next to exact full attention")
     ap.add_argument("--frames", type=int, default=0, help="--curve: frames to run (default: "
@@ -764,6 +851,9 @@ def main():
         return
     if args.diagnostics:
         run_diagnostics(args, int(os.environ.get("LOCAL_RANK", 0)))
+        return
+    if args.block:
+        run_block(args, int(os.environ.get("LOCAL_RANK", 0)))
         return
     if args.warmup < 3:
         raise SystemExit("--warmup must be at least 3")

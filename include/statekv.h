@@ -204,6 +204,68 @@ statekv_status statekv_state_metrics(const uint8_t* mask_n, const uint8_t* mask_
                                      int32_t T, int64_t row_stride, double* out,
                                      statekv_stream stream);
 
+/* ---- Full per-frame transformer block ----------------------------------
+ * One frame of every layer of a Qwen2-style decoder around the StateKV step,
+ * layers in order (layer l + 1 reads layer l's output), per layer:
+ *   h  = RMSNorm(x) * norm_attn
+ *   [q k v] = h W_qkv^T + b_qkv;  q, k rotated by RoPE at the virtual
+ *            positions L_n + t (Sec. 3.3: positions follow the virtual
+ *            sequence length, not the cache size), with one RoPE scaling for
+ *            the whole run (Sec. 3.3, "consistent RoPE scaling")
+ *   o  = the StateKV step of statekv_prefill_frame on (q, k, v) (steps a1-a5:
+ *        the layer's state and decode cache advance by one frame)
+ *   x1 = x + o W_o^T
+ *   x2 = x1 + (SiLU(h2 W_gate^T) * (h2 W_up^T)) W_down^T,  h2 = RMSNorm(x1) * norm_mlp
+ * bf16 storage between steps, fp32 arithmetic; the projections are plain
+ * cuBLASLt GEMMs.  Weight matrices are row-major [out features][in features]
+ * (torch.nn.Linear layout). */
+typedef struct {
+    int32_t hidden;            /* model width (multiple of 8, at most 8192) */
+    int32_t intermediate;      /* MLP width (multiple of 8) */
+    float rms_eps;             /* RMSNorm epsilon */
+    float rope_theta;          /* RoPE base: pair k of head dim d turns at theta^(-2k/d) */
+    float yarn_factor;         /* <= 1: plain RoPE; s > 1: YaRN scaling by s over a
+                                  trained context of yarn_original_max tokens (pairs
+                                  whose wavelength fits the context fewer than once
+                                  turn s times slower, more than 32 times unchanged,
+                                  linear in between; q and k scaled by 0.1 ln s + 1) */
+    int32_t yarn_original_max;
+} statekv_block_config;
+
+typedef struct {
+    const void* norm_attn;     /* bf16 [hidden] */
+    const void* w_qkv;         /* bf16 [(Hq + 2 Hkv) d][hidden]: q, then k, then v rows */
+    const void* b_qkv;         /* bf16 [(Hq + 2 Hkv) d], or NULL for no bias */
+    const void* w_o;           /* bf16 [hidden][Hq d] */
+    const void* norm_mlp;      /* bf16 [hidden] */
+    const void* w_gate_up;     /* bf16 [2 intermediate][hidden]: gate rows, then up rows */
+    const void* w_down;        /* bf16 [hidden][intermediate] */
+} statekv_block_weights;
+
+/* Device workspace (bytes, 256-byte aligned by the caller) for one
+ * statekv_block_frame call over stream_count streams. */
+statekv_status statekv_block_workspace_bytes(const statekv_handle* h,
+                                             const statekv_block_config* bc,
+                                             int32_t stream_count, size_t* bytes);
+
+/* Runs the next frame of streams [stream_begin, stream_begin + stream_count)
+ * through layers [layer_begin, layer_begin + layer_count) in order.
+ *   weights  host array of num_layers entries (entry l for layer l; device
+ *            pointers, each 16-byte aligned)
+ *   x_in     bf16 [stream_count][T][hidden] (device): the frame's input to
+ *            layer layer_begin; not modified
+ *   x_out    bf16 [stream_count][T][hidden] (device): layer
+ *            layer_begin + layer_count - 1's output (may equal x_in)
+ * Every covered (stream, layer) advances by one frame.  Errors as
+ * statekv_prefill_frame, INVALID_ARG for a bad block config (head_dim > 128
+ * pairs, sizes not multiples of 8), UNSUPPORTED if cuBLASLt finds no GEMM
+ * plan; nothing is enqueued on an argument error. */
+statekv_status statekv_block_frame(statekv_handle* h, const statekv_block_config* bc,
+                                   const statekv_block_weights* weights, int32_t stream_begin,
+                                   int32_t stream_count, int32_t layer_begin, int32_t layer_count,
+                                   const void* x_in, void* x_out, void* workspace,
+                                   size_t workspace_bytes, statekv_stream stream);
+
 /* Decoding over the detailed cache D_N (Sec. 3.2 / 3.3: decoding reads only
  * the detailed state; the compressed state is not used).  For every covered
  * (stream, layer), the num_tokens new tokens (a prompt, or one generated
@@ -263,11 +325,12 @@ statekv_status statekv_cache_view(const statekv_handle* h, int32_t stream, int32
 /* Optional per-kernel timing with CUDA events recorded on the call's stream
  * around each launch.  enable != 0 starts a new record; read synchronises on
  * the recorded events and returns, per kernel kind (0 = decode-cache append,
- * 1 = frame attention + importance, 2 = state select/gather), the number of
- * launches and their summed device milliseconds. */
+ * 1 = frame attention + importance, 2 = state select/gather, 3 = the block's
+ * projection GEMMs, 4 = the block's RMSNorm / RoPE / SiLU kernels), the
+ * number of launches and their summed device milliseconds. */
 typedef struct {
-    int64_t launches[3];
-    double milliseconds[3];
+    int64_t launches[5];
+    double milliseconds[5];
 } statekv_profile;
 statekv_status statekv_profile_enable(statekv_handle* h, int32_t enable);
 statekv_status statekv_profile_read(statekv_handle* h, statekv_profile* out);

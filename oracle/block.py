@@ -128,7 +128,8 @@ class OracleBlock:
         inter = gu.shape[1] // 2
         a = round_bf16(silu(gu[:, :inter]) * gu[:, inter:])
         x2 = round_bf16(x1 + a @ w.w_down.T)
-        return x2, {"q": q, "k": k, "v": v, "attn": o, "x1": x1, "act": a}
+        return x2, {"q": q, "k": k, "v": v, "attn": o, "x1": x1, "act": a, "imp": imp,
+                    "kept": kept}
 
     def frame(self, x: np.ndarray) -> np.ndarray:
         for l in range(len(self.weights)):

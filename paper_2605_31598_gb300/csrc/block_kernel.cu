@@ -1,0 +1,284 @@
+// The per-frame transformer block around the StateKV step: the elementwise
+// kernels of one decoder layer and the projection GEMMs.
+//
+//   rmsnorm      y = x / sqrt(mean(x^2) + eps) * g        (fp32, one bf16 rounding)
+//   qkv_rope     the QKV projection's q and k rotated at their virtual
+//                positions p = L_n + t (Sec. 3.3, "virtual sequence length"),
+//                with one fixed RoPE scaling for the whole run ("consistent
+//                RoPE scaling"); v copied; written in the step's [T][H][d]
+//                layout.  Angles p * theta_k are formed and reduced modulo
+//                2 pi in fp64 (p reaches 2^20 and more), then sin/cos in fp32.
+//   silu_mul     a = SiLU(gate) * up                       (fp32, one rounding)
+//   projections  plain bf16 GEMMs on cuBLASLt (fp32 accumulation): the QKV
+//                projection with its bias in the epilogue, the output and
+//                down projections accumulating into the residual stream.
+// Rows are tokens (stream-major, then token): one CTA per row for the norm and
+// the rotation, 8 elements per thread for SiLU * up; 16-byte accesses where
+// the layout allows.
+#include <cublasLt.h>
+
+#include <vector>
+
+#include "statekv_kernels.cuh"
+
+namespace statekv {
+namespace {
+
+constexpr int kNormThreads = 256;
+constexpr int kNormChunks = 4;  // 8-element chunks a thread keeps: rows up to 8192 wide
+
+__device__ __forceinline__ void unpack8(const uint4& u, float (&f)[8])
+{
+    const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const float2 t = __bfloat1622float2(h[i]);
+        f[2 * i] = t.x;
+        f[2 * i + 1] = t.y;
+    }
+}
+
+__device__ __forceinline__ uint4 pack8(const float (&f)[8])
+{
+    uint4 u;
+    __nv_bfloat162* h = reinterpret_cast<__nv_bfloat162*>(&u);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) h[i] = __floats2bfloat162_rn(f[2 * i], f[2 * i + 1]);
+    return u;
+}
+
+// One CTA per row; the row stays in registers between the sum of squares and
+// the scaled write (16-byte loads and stores; H a multiple of 8, <= 8192).
+__global__ void __launch_bounds__(kNormThreads)
+    rmsnorm_kernel(const __nv_bfloat16* x, const __nv_bfloat16* g, float eps, __nv_bfloat16* y,
+                   int H)
+{
+    __shared__ float red[kNormThreads / 32];
+    const uint4* xr = reinterpret_cast<const uint4*>(x + static_cast<size_t>(blockIdx.x) * H);
+    uint4* yr = reinterpret_cast<uint4*>(y + static_cast<size_t>(blockIdx.x) * H);
+    const uint4* gr = reinterpret_cast<const uint4*>(g);
+    const int nc = H / 8;
+    float v[kNormChunks][8];
+    float ss = 0.f;
+#pragma unroll
+    for (int c = 0; c < kNormChunks; ++c) {
+        const int i = threadIdx.x + c * kNormThreads;
+        if (i < nc) {
+            unpack8(xr[i], v[c]);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) ss += v[c][e] * v[c][e];
+        }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
+    __syncthreads();
+    float tot = 0.f;
+#pragma unroll
+    for (int w = 0; w < kNormThreads / 32; ++w) tot += red[w];
+    const float r = rsqrtf(tot / static_cast<float>(H) + eps);
+#pragma unroll
+    for (int c = 0; c < kNormChunks; ++c) {
+        const int i = threadIdx.x + c * kNormThreads;
+        if (i < nc) {
+            float gw[8], o[8];
+            unpack8(gr[i], gw);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) o[e] = v[c][e] * r * gw[e];
+            yr[i] = pack8(o);
+        }
+    }
+}
+
+// One CTA per token: the d/2 angles of its position are formed once (fp64
+// product and reduction modulo 2 pi, fp32 sin/cos) into shared memory, then
+// every q and k head's pairs are rotated from that table and v is copied.
+__global__ void __launch_bounds__(256) qkv_rope_kernel(const RopeParams p)
+{
+    __shared__ float cs_tab[64], sn_tab[64];
+    const int half = p.d / 2;
+    const int row = blockIdx.x;  // s * T + t
+    const int s = row / p.T, t = row - s * p.T;
+    const __nv_bfloat16* src = p.qkv + static_cast<size_t>(row) * (p.Hq + 2 * p.Hkv) * p.d;
+    if (threadIdx.x < half) {
+        const long long ua = static_cast<long long>(p.stream_begin + s) * p.num_layers + p.layer;
+        const double pos = static_cast<double>(static_cast<long long>(p.frames[ua * p.Hkv]) * p.T + t);
+        const double twopi = 6.283185307179586476925286766559;
+        double ang = pos * p.freq[threadIdx.x];
+        ang -= twopi * floor(ang * (1.0 / twopi));
+        float sn, cs;
+        sincosf(static_cast<float>(ang), &sn, &cs);
+        cs_tab[threadIdx.x] = cs * p.scale;
+        sn_tab[threadIdx.x] = sn * p.scale;
+    }
+    __syncthreads();
+    const int qk_pairs = (p.Hq + p.Hkv) * half;
+    for (int e = threadIdx.x; e < qk_pairs; e += blockDim.x) {
+        const int hh = e / half, k = e - hh * half;
+        const float x1 = __bfloat162float(src[hh * p.d + k]);
+        const float x2 = __bfloat162float(src[hh * p.d + k + half]);
+        const float c = cs_tab[k], sn = sn_tab[k];
+        __nv_bfloat16* dst = hh < p.Hq ? p.q + (static_cast<size_t>(row) * p.Hq + hh) * p.d
+                                       : p.k + (static_cast<size_t>(row) * p.Hkv + (hh - p.Hq)) * p.d;
+        dst[k] = __float2bfloat16(x1 * c - x2 * sn);
+        dst[k + half] = __float2bfloat16(x2 * c + x1 * sn);
+    }
+    const uint4* vs = reinterpret_cast<const uint4*>(src + (p.Hq + p.Hkv) * p.d);
+    uint4* vd = reinterpret_cast<uint4*>(p.v + static_cast<size_t>(row) * p.Hkv * p.d);
+    for (int e = threadIdx.x; e < p.Hkv * p.d / 8; e += blockDim.x) vd[e] = vs[e];
+}
+
+// 8 outputs per thread: a = SiLU(gate) * up, gate in columns [0, I), up in [I, 2I).
+__global__ void silu_mul_kernel(const __nv_bfloat16* gu, __nv_bfloat16* a, int rows, int I)
+{
+    const int chunks = I / 8;
+    const long long idx = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (idx >= static_cast<long long>(rows) * chunks) return;
+    const int r = static_cast<int>(idx / chunks), c = static_cast<int>(idx - static_cast<long long>(r) * chunks);
+    const uint4* grow = reinterpret_cast<const uint4*>(gu + static_cast<size_t>(r) * 2 * I);
+    float g[8], u[8], o[8];
+    unpack8(grow[c], g);
+    unpack8(grow[chunks + c], u);
+#pragma unroll
+    for (int e = 0; e < 8; ++e) o[e] = g[e] / (1.f + expf(-g[e])) * u[e];
+    reinterpret_cast<uint4*>(a + static_cast<size_t>(r) * I)[c] = pack8(o);
+}
+
+}  // namespace
+
+cudaError_t launch_rmsnorm(const __nv_bfloat16* x, const __nv_bfloat16* g, float eps,
+                           __nv_bfloat16* y, int rows, int H, cudaStream_t st)
+{
+    if (rows <= 0) return cudaSuccess;
+    rmsnorm_kernel<<<rows, kNormThreads, 0, st>>>(x, g, eps, y, H);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_qkv_rope(const RopeParams& p, cudaStream_t st)
+{
+    const int rows = p.S * p.T;
+    if (rows <= 0) return cudaSuccess;
+    qkv_rope_kernel<<<rows, 256, 0, st>>>(p);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_silu_mul(const __nv_bfloat16* gu, __nv_bfloat16* a, long long rows, int I,
+                            cudaStream_t st)
+{
+    const long long total = rows * (I / 8);
+    if (total <= 0) return cudaSuccess;
+    silu_mul_kernel<<<static_cast<unsigned>((total + 255) / 256), 256, 0, st>>>(
+        gu, a, static_cast<int>(rows), I);
+    return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------ GEMMs
+struct LtPlan {
+    int M, N, K;
+    bool bias, add;
+    cublasLtMatmulDesc_t op = nullptr;
+    cublasLtMatrixLayout_t a = nullptr, b = nullptr, c = nullptr;
+    cublasLtMatmulAlgo_t algo;
+    size_t ws = 0;
+};
+
+struct LtContext {
+    cublasLtHandle_t h = nullptr;
+    std::vector<LtPlan> plans;
+};
+
+LtContext* lt_create()
+{
+    LtContext* c = new LtContext;
+    if (cublasLtCreate(&c->h) != CUBLAS_STATUS_SUCCESS) {
+        delete c;
+        return nullptr;
+    }
+    return c;
+}
+
+void lt_destroy(LtContext* c)
+{
+    if (!c) return;
+    for (LtPlan& p : c->plans) {
+        cublasLtMatrixLayoutDestroy(p.a);
+        cublasLtMatrixLayoutDestroy(p.b);
+        cublasLtMatrixLayoutDestroy(p.c);
+        cublasLtMatmulDescDestroy(p.op);
+    }
+    cublasLtDestroy(c->h);
+    delete c;
+}
+
+namespace {
+
+// Row-major D[M][N] = X[M][K] W[N][K]^T: in cuBLASLt's column-major terms
+// D^T (N x M) = op_T(W as K x N) * X^T (K x M).
+LtPlan* lt_plan(LtContext* c, int M, int N, int K, bool bias, bool add, size_t ws_bytes)
+{
+    for (LtPlan& p : c->plans)
+        if (p.M == M && p.N == N && p.K == K && p.bias == bias && p.add == add && p.ws <= ws_bytes)
+            return &p;
+    LtPlan p;
+    p.M = M;
+    p.N = N;
+    p.K = K;
+    p.bias = bias;
+    p.add = add;
+    bool ok = cublasLtMatmulDescCreate(&p.op, CUBLAS_COMPUTE_32F, CUDA_R_32F) == CUBLAS_STATUS_SUCCESS;
+    const cublasOperation_t ta = CUBLAS_OP_T, tb = CUBLAS_OP_N;
+    ok = ok &&
+         cublasLtMatmulDescSetAttribute(p.op, CUBLASLT_MATMUL_DESC_TRANSA, &ta, sizeof ta) ==
+             CUBLAS_STATUS_SUCCESS &&
+         cublasLtMatmulDescSetAttribute(p.op, CUBLASLT_MATMUL_DESC_TRANSB, &tb, sizeof tb) ==
+             CUBLAS_STATUS_SUCCESS;
+    if (ok && bias) {
+        const cublasLtEpilogue_t ep = CUBLASLT_EPILOGUE_BIAS;
+        ok = cublasLtMatmulDescSetAttribute(p.op, CUBLASLT_MATMUL_DESC_EPILOGUE, &ep, sizeof ep) ==
+             CUBLAS_STATUS_SUCCESS;
+    }
+    ok = ok &&
+         cublasLtMatrixLayoutCreate(&p.a, CUDA_R_16BF, K, N, K) == CUBLAS_STATUS_SUCCESS &&
+         cublasLtMatrixLayoutCreate(&p.b, CUDA_R_16BF, K, M, K) == CUBLAS_STATUS_SUCCESS &&
+         cublasLtMatrixLayoutCreate(&p.c, CUDA_R_16BF, N, M, N) == CUBLAS_STATUS_SUCCESS;
+    cublasLtMatmulPreference_t pref = nullptr;
+    ok = ok && cublasLtMatmulPreferenceCreate(&pref) == CUBLAS_STATUS_SUCCESS &&
+         cublasLtMatmulPreferenceSetAttribute(pref, CUBLASLT_MATMUL_PREF_MAX_WORKSPACE_BYTES,
+                                              &ws_bytes, sizeof ws_bytes) == CUBLAS_STATUS_SUCCESS;
+    cublasLtMatmulHeuristicResult_t res{};
+    int found = 0;
+    ok = ok && cublasLtMatmulAlgoGetHeuristic(c->h, p.op, p.a, p.b, p.c, p.c, pref, 1, &res,
+                                              &found) == CUBLAS_STATUS_SUCCESS &&
+         found > 0;
+    if (pref) cublasLtMatmulPreferenceDestroy(pref);
+    if (!ok) {
+        cublasLtMatrixLayoutDestroy(p.a);
+        cublasLtMatrixLayoutDestroy(p.b);
+        cublasLtMatrixLayoutDestroy(p.c);
+        cublasLtMatmulDescDestroy(p.op);
+        return nullptr;
+    }
+    p.algo = res.algo;
+    p.ws = res.workspaceSize;
+    c->plans.push_back(p);
+    return &c->plans.back();
+}
+
+}  // namespace
+
+bool lt_matmul(LtContext* c, const __nv_bfloat16* X, const __nv_bfloat16* W,
+               const __nv_bfloat16* bias, __nv_bfloat16* D, bool add, int M, int N, int K,
+               void* ws, size_t ws_bytes, cudaStream_t st)
+{
+    if (M <= 0) return true;
+    LtPlan* p = lt_plan(c, M, N, K, bias != nullptr, add, ws_bytes);
+    if (!p) return false;
+    if (bias && cublasLtMatmulDescSetAttribute(p->op, CUBLASLT_MATMUL_DESC_BIAS_POINTER, &bias,
+                                               sizeof bias) != CUBLAS_STATUS_SUCCESS)
+        return false;
+    const float alpha = 1.f, beta = add ? 1.f : 0.f;
+    return cublasLtMatmul(c->h, p->op, &alpha, W, p->a, X, p->b, &beta, D, p->c, D, p->c, &p->algo,
+                          ws, p->ws, st) == CUBLAS_STATUS_SUCCESS;
+}
+
+}  // namespace statekv

@@ -11,6 +11,7 @@
 #include <cudaTypedefs.h>
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstring>
 #include <mutex>
@@ -150,6 +151,7 @@ struct statekv_handle {
     bool prof_on;
     size_t prof_used;
     std::vector<ProfRec> prof;
+    LtContext* lt = nullptr;   // cuBLASLt, created by the first block call
 
     template <class T>
     T* at(size_t off) const { return reinterpret_cast<T*>(arena + off); }
@@ -635,6 +637,183 @@ statekv_status statekv_state_metrics(const uint8_t* mask_n, const uint8_t* mask_
     return STATEKV_OK;
 }
 
+namespace {
+
+// Workspace carve-up of one block call (all offsets 256-byte aligned).
+struct BlockBufs {
+    size_t h, qkv, q, k, v, attn, gu, act, lt, total;
+};
+
+constexpr size_t kLtWorkspace = 32u << 20;
+
+BlockBufs block_bufs(const statekv_config& c, const statekv_block_config& b, int streams)
+{
+    const size_t rows = static_cast<size_t>(streams) * c.tokens_per_frame;
+    const size_t d = c.head_dim, hq = c.num_q_heads, hkv = c.num_kv_heads;
+    auto up = [](size_t x) { return (x + 255) & ~static_cast<size_t>(255); };
+    BlockBufs o{};
+    size_t off = 0;
+    auto take = [&](size_t bytes) {
+        const size_t at = off;
+        off += up(bytes);
+        return at;
+    };
+    o.h = take(rows * b.hidden * 2);
+    o.qkv = take(rows * (hq + 2 * hkv) * d * 2);
+    o.q = take(rows * hq * d * 2);
+    o.k = take(rows * hkv * d * 2);
+    o.v = take(rows * hkv * d * 2);
+    o.attn = take(rows * hq * d * 2);
+    o.gu = take(rows * 2 * static_cast<size_t>(b.intermediate) * 2);
+    o.act = take(rows * static_cast<size_t>(b.intermediate) * 2);
+    o.lt = take(kLtWorkspace);
+    o.total = off;
+    return o;
+}
+
+bool block_config_ok(const statekv_config& c, const statekv_block_config* b)
+{
+    return b && b->hidden > 0 && b->hidden % 8 == 0 && b->hidden <= 8192 && b->intermediate > 0 &&
+           b->intermediate % 8 == 0 && b->rms_eps >= 0.f && std::isfinite(b->rms_eps) &&
+           b->rope_theta > 1.f && std::isfinite(b->rope_theta) && std::isfinite(b->yarn_factor) &&
+           (b->yarn_factor <= 1.f || b->yarn_original_max > 0) && c.head_dim / 2 <= 64;
+}
+
+}  // namespace
+
+statekv_status statekv_block_workspace_bytes(const statekv_handle* h,
+                                             const statekv_block_config* bc,
+                                             int32_t stream_count, size_t* bytes)
+{
+    if (!h || !bytes || !block_config_ok(h->cfg, bc) || stream_count < 1 ||
+        stream_count > h->cfg.num_streams)
+        return STATEKV_ERR_INVALID_ARG;
+    *bytes = block_bufs(h->cfg, *bc, stream_count).total;
+    return STATEKV_OK;
+}
+
+statekv_status statekv_block_frame(statekv_handle* h, const statekv_block_config* bc,
+                                   const statekv_block_weights* weights, int32_t stream_begin,
+                                   int32_t stream_count, int32_t layer_begin, int32_t layer_count,
+                                   const void* x_in, void* x_out, void* workspace,
+                                   size_t workspace_bytes, statekv_stream stream)
+{
+    if (!h || !weights || !x_in || !x_out || !workspace || !block_config_ok(h->cfg, bc) ||
+        !aligned(x_in, 16) || !aligned(x_out, 16) || !aligned(workspace, 256))
+        return STATEKV_ERR_INVALID_ARG;
+    const statekv_config& c = h->cfg;
+    const statekv_block_config& b = *bc;
+    if (stream_count < 1 || stream_begin < 0 || stream_begin + stream_count > c.num_streams ||
+        layer_count < 1 || layer_begin < 0 || layer_begin + layer_count > c.num_layers)
+        return STATEKV_ERR_INVALID_ARG;
+    const BlockBufs bb = block_bufs(c, b, stream_count);
+    if (workspace_bytes < bb.total) return STATEKV_ERR_INVALID_ARG;
+    for (int l = layer_begin; l < layer_begin + layer_count; ++l) {
+        const statekv_block_weights& w = weights[l];
+        if (!w.norm_attn || !w.w_qkv || !w.w_o || !w.norm_mlp || !w.w_gate_up || !w.w_down ||
+            !aligned(w.norm_attn, 16) || !aligned(w.w_qkv, 16) || !aligned(w.w_o, 16) ||
+            !aligned(w.norm_mlp, 16) || !aligned(w.w_gate_up, 16) || !aligned(w.w_down, 16) ||
+            (w.b_qkv && !aligned(w.b_qkv, 16)))
+            return STATEKV_ERR_INVALID_ARG;
+    }
+    uint8_t* ws = static_cast<uint8_t*>(workspace);
+    auto buf = [&](size_t off) { return reinterpret_cast<__nv_bfloat16*>(ws + off); };
+    // every covered (stream, layer) must be able to take the frame
+    statekv_frame_args probe{};
+    probe.stream_begin = stream_begin;
+    probe.stream_count = stream_count;
+    probe.layer_begin = layer_begin;
+    probe.layer_count = layer_count;
+    probe.q = buf(bb.q);
+    probe.k = buf(bb.k);
+    probe.v = buf(bb.v);
+    probe.out = buf(bb.attn);
+    const statekv_status s = check_args(h, &probe, false);
+    if (s != STATEKV_OK) return s;
+    if (!h->lt && !(h->lt = lt_create())) return STATEKV_ERR_CUDA;
+
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    const int T = c.tokens_per_frame, d = c.head_dim, Hq = c.num_q_heads, Hkv = c.num_kv_heads;
+    const int rows = stream_count * T;
+    const int H = b.hidden, I = b.intermediate, W = (Hq + 2 * Hkv) * d;
+    __nv_bfloat16* x = static_cast<__nv_bfloat16*>(x_out);
+    if (x_out != x_in &&
+        cudaMemcpyAsync(x, x_in, static_cast<size_t>(rows) * H * 2, cudaMemcpyDeviceToDevice,
+                        st) != cudaSuccess)
+        return STATEKV_ERR_CUDA;
+
+    RopeParams rp{};
+    rp.qkv = buf(bb.qkv);
+    rp.q = buf(bb.q);
+    rp.k = buf(bb.k);
+    rp.v = buf(bb.v);
+    rp.frames = h->at<int32_t>(h->lay.frames);
+    rp.stream_begin = stream_begin;
+    rp.num_layers = c.num_layers;
+    rp.S = stream_count;
+    rp.T = T;
+    rp.Hq = Hq;
+    rp.Hkv = Hkv;
+    rp.d = d;
+    {   // RoPE frequencies (fp64), with YaRN's blend when scaled
+        const double pi2 = 6.283185307179586476925286766559;
+        rp.scale = 1.f;
+        for (int k = 0; k < d / 2; ++k) {
+            double f = std::pow(static_cast<double>(b.rope_theta), -2.0 * k / d);
+            if (b.yarn_factor > 1.f) {
+                const double r = b.yarn_original_max * f / pi2;  // context / wavelength
+                const double g = std::min(1.0, std::max(0.0, (r - 1.0) / 31.0));
+                f = (1.0 - g) * f / b.yarn_factor + g * f;
+            }
+            rp.freq[k] = f;
+        }
+        if (b.yarn_factor > 1.f) rp.scale = static_cast<float>(0.1 * std::log(b.yarn_factor) + 1.0);
+    }
+    void* ltws = ws + bb.lt;
+    auto gemm = [&](const void* X, const void* Wt, const void* bias, __nv_bfloat16* D, bool add,
+                    int N, int K) {
+        return timed(h, 3, st, [&] {
+                   return lt_matmul(h->lt, static_cast<const __nv_bfloat16*>(X),
+                                    static_cast<const __nv_bfloat16*>(Wt),
+                                    static_cast<const __nv_bfloat16*>(bias), D, add, rows, N, K,
+                                    ltws, kLtWorkspace, st)
+                              ? cudaSuccess
+                              : cudaErrorNotSupported;
+               }) == cudaSuccess;
+    };
+    for (int l = layer_begin; l < layer_begin + layer_count; ++l) {
+        const statekv_block_weights& w = weights[l];
+        if (timed(h, 4, st, [&] {
+                return launch_rmsnorm(x, static_cast<const __nv_bfloat16*>(w.norm_attn), b.rms_eps,
+                                      buf(bb.h), rows, H, st);
+            }) != cudaSuccess)
+            return STATEKV_ERR_CUDA;
+        if (!gemm(buf(bb.h), w.w_qkv, w.b_qkv, buf(bb.qkv), false, W, H))
+            return STATEKV_ERR_UNSUPPORTED;
+        rp.layer = l;
+        if (timed(h, 4, st, [&] { return launch_qkv_rope(rp, st); }) != cudaSuccess)
+            return STATEKV_ERR_CUDA;
+        statekv_frame_args a = probe;
+        a.layer_begin = l;
+        a.layer_count = 1;
+        const statekv_status r = run_step(h, a, st);
+        if (r != STATEKV_OK) return r;
+        if (!gemm(buf(bb.attn), w.w_o, nullptr, x, true, H, Hq * d)) return STATEKV_ERR_UNSUPPORTED;
+        if (timed(h, 4, st, [&] {
+                return launch_rmsnorm(x, static_cast<const __nv_bfloat16*>(w.norm_mlp), b.rms_eps,
+                                      buf(bb.h), rows, H, st);
+            }) != cudaSuccess)
+            return STATEKV_ERR_CUDA;
+        if (!gemm(buf(bb.h), w.w_gate_up, nullptr, buf(bb.gu), false, 2 * I, H))
+            return STATEKV_ERR_UNSUPPORTED;
+        if (timed(h, 4, st, [&] { return launch_silu_mul(buf(bb.gu), buf(bb.act), rows, I, st); }) !=
+            cudaSuccess)
+            return STATEKV_ERR_CUDA;
+        if (!gemm(buf(bb.act), w.w_down, nullptr, x, true, H, I)) return STATEKV_ERR_UNSUPPORTED;
+    }
+    return STATEKV_OK;
+}
+
 statekv_status statekv_decode_step(statekv_handle* h, const statekv_decode_args* a,
                                   statekv_stream stream)
 {
@@ -782,6 +961,7 @@ void statekv_destroy(statekv_handle* h)
         cudaEventDestroy(r.b);
     }
     cudaFreeHost(const_cast<int32_t*>(h->status_host));
+    lt_destroy(h->lt);
     delete h;
 }
 

@@ -117,6 +117,32 @@ cudaError_t launch_state_metrics(const uint8_t* mask_n, const uint8_t* mask_n1, 
                                  int rows, long long n_seen, int T, long long stride, double* out,
                                  cudaStream_t st);
 
+// Per-frame transformer block (block_kernel.cu).
+struct RopeParams {
+    const __nv_bfloat16* qkv;   // [S*T][(Hq + 2 Hkv) * d]: q heads, k heads, v heads
+    __nv_bfloat16* q;           // [S][T][Hq][d]
+    __nv_bfloat16* k;           // [S][T][Hkv][d]
+    __nv_bfloat16* v;           // [S][T][Hkv][d]
+    const int32_t* frames;      // arena [S*L][Hkv]: frames before this one
+    int stream_begin, layer, num_layers;
+    int S, T, Hq, Hkv, d;
+    float scale;                // q and k scale of the RoPE scaling (1: none)
+    double freq[64];            // angular frequency of rotated pair k < d / 2
+};
+cudaError_t launch_rmsnorm(const __nv_bfloat16* x, const __nv_bfloat16* g, float eps,
+                           __nv_bfloat16* y, int rows, int H, cudaStream_t st);
+cudaError_t launch_qkv_rope(const RopeParams& p, cudaStream_t st);
+cudaError_t launch_silu_mul(const __nv_bfloat16* gu, __nv_bfloat16* a, long long rows, int I,
+                            cudaStream_t st);
+struct LtContext;
+LtContext* lt_create();
+void lt_destroy(LtContext* c);
+// Row-major D[M][N] = X[M][K] W[N][K]^T (+ bias[N]) (+ D when add), bf16 in and
+// out, fp32 accumulation; false if cuBLASLt has no plan or fails.
+bool lt_matmul(LtContext* c, const __nv_bfloat16* X, const __nv_bfloat16* W,
+               const __nv_bfloat16* bias, __nv_bfloat16* D, bool add, int M, int N, int K,
+               void* ws, size_t ws_bytes, cudaStream_t st);
+
 // Recency-window state update (the baseline): the frame's tokens enter ring
 // slots position mod B, overwriting the tokens that leave the window.
 cudaError_t launch_recency(const RecencyParams& p, cudaStream_t st);

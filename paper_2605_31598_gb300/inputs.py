@@ -139,3 +139,55 @@ def batch_qkv(shape: Shape, frame: int, *, streams, layers, seed: int = 0, devic
     T, Hq, Hkv, d = shape.tokens_per_frame, shape.num_q_heads, shape.num_kv_heads, shape.head_dim
     return (torch.stack(qs).view(S, L, T, Hq, d), torch.stack(ks).view(S, L, T, Hkv, d),
             torch.stack(vs).view(S, L, T, Hkv, d))
+
+
+# ------------------------------------------------------------ transformer block
+@dataclass(frozen=True)
+class BlockShape:
+    """Widths of the decoder layer around the StateKV step (Qwen2 naming)."""
+
+    hidden: int
+    intermediate: int
+    weight_std: float = 0.02
+    rms_eps: float = 1e-6
+    rope_theta: float = ROPE_THETA
+
+
+BLOCKS = {
+    "qwen7b": BlockShape(3584, 18944),
+    "tiny": BlockShape(128, 256, weight_std=0.08),
+}
+
+
+def block_weights(shape: Shape, block: BlockShape, *, seed: int = 0, device="cpu",
+                  bias: bool = True, layers=None):
+    """Synthetic (random-init) bf16 weights of every layer, torch.nn.Linear
+    layout [out][in]: dicts with norm_attn, w_qkv, b_qkv, w_o, norm_mlp,
+    w_gate_up (gate rows, then up rows), w_down."""
+    Hq, Hkv, d = shape.num_q_heads, shape.num_kv_heads, shape.head_dim
+    H, I, sd = block.hidden, block.intermediate, block.weight_std
+    out = []
+    for l in (range(shape.num_layers) if layers is None else layers):
+        g = _gen(device, seed, 0, l, 0, "block")
+        r = lambda *s: (torch.randn(s, generator=g, device=device) * sd).to(torch.bfloat16)
+        norm = lambda: (1.0 + 0.1 * torch.randn((H,), generator=g, device=device)).to(torch.bfloat16)
+        out.append({
+            "norm_attn": norm(),
+            "w_qkv": r((Hq + 2 * Hkv) * d, H),
+            "b_qkv": r((Hq + 2 * Hkv) * d) if bias else None,
+            "w_o": r(H, Hq * d),
+            "norm_mlp": norm(),
+            "w_gate_up": r(2 * I, H),
+            "w_down": r(H, I),
+        })
+    return out
+
+
+def block_input(shape: Shape, block: BlockShape, frame: int, *, seed: int = 0, device="cpu"):
+    """The frame's input hidden states (the vision tokens' embeddings), bf16
+    [streams][T][hidden], N(0, 1)."""
+    xs = []
+    for s in range(shape.num_streams):
+        g = _gen(device, seed, s, -1, frame, "x")
+        xs.append(torch.randn((shape.tokens_per_frame, block.hidden), generator=g, device=device))
+    return torch.stack(xs).to(torch.bfloat16).contiguous()

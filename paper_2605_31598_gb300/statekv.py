@@ -28,6 +28,7 @@ EXPORTED = ("statekv_arena_bytes", "statekv_init", "statekv_prefill_frame",
             "statekv_device_error", "statekv_frame_attention_noalloc",
             "statekv_scores_workspace_bytes", "statekv_full_attention_scores",
             "statekv_topb_mask", "statekv_concentration_sums", "statekv_state_metrics",
+            "statekv_block_workspace_bytes", "statekv_block_frame",
             "statekv_destroy", "statekv_status_string")
 
 
@@ -49,6 +50,19 @@ class statekv_decode_args(ctypes.Structure):
                 ("out", ctypes.c_void_p)]
 
 
+class statekv_block_config(ctypes.Structure):
+    _fields_ = [("hidden", ctypes.c_int32), ("intermediate", ctypes.c_int32),
+                ("rms_eps", ctypes.c_float), ("rope_theta", ctypes.c_float),
+                ("yarn_factor", ctypes.c_float), ("yarn_original_max", ctypes.c_int32)]
+
+
+class statekv_block_weights(ctypes.Structure):
+    _fields_ = [("norm_attn", ctypes.c_void_p), ("w_qkv", ctypes.c_void_p),
+                ("b_qkv", ctypes.c_void_p), ("w_o", ctypes.c_void_p),
+                ("norm_mlp", ctypes.c_void_p), ("w_gate_up", ctypes.c_void_p),
+                ("w_down", ctypes.c_void_p)]
+
+
 class statekv_frame_args(ctypes.Structure):
     _fields_ = [("stream_begin", ctypes.c_int32), ("stream_count", ctypes.c_int32),
                 ("layer_begin", ctypes.c_int32), ("layer_count", ctypes.c_int32),
@@ -68,7 +82,7 @@ class statekv_cache_info(ctypes.Structure):
 
 
 class statekv_profile(ctypes.Structure):
-    _fields_ = [("launches", ctypes.c_int64 * 3), ("milliseconds", ctypes.c_double * 3)]
+    _fields_ = [("launches", ctypes.c_int64 * 5), ("milliseconds", ctypes.c_double * 5)]
 
 
 _lock = threading.Lock()
@@ -139,6 +153,14 @@ def lib() -> ctypes.CDLL:
                                                 ctypes.c_int32, ctypes.c_int64, ctypes.c_int32,
                                                 ctypes.c_int64, ctypes.c_void_p, ctypes.c_void_p]
             L.statekv_state_metrics.restype = st
+            L.statekv_block_workspace_bytes.argtypes = [ctypes.c_void_p, P(statekv_block_config),
+                                                        ctypes.c_int32, P(ctypes.c_size_t)]
+            L.statekv_block_workspace_bytes.restype = st
+            L.statekv_block_frame.argtypes = [
+                ctypes.c_void_p, P(statekv_block_config), P(statekv_block_weights),
+                ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_void_p,
+                ctypes.c_void_p, ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p]
+            L.statekv_block_frame.restype = st
             L.statekv_destroy.argtypes = [ctypes.c_void_p]
             L.statekv_destroy.restype = None
             L.statekv_status_string.argtypes = [ctypes.c_int]
@@ -268,6 +290,36 @@ def statekv_state_metrics(mask_n: int, mask_n1: int, scores_n1: int, rows: int, 
                                        ctypes.c_void_p(out), ctypes.c_void_p(stream))
 
 
+def statekv_block_workspace_bytes(handle: int, bc: statekv_block_config, stream_count: int) -> int:
+    n = ctypes.c_size_t(0)
+    check(lib().statekv_block_workspace_bytes(handle, ctypes.byref(bc), stream_count,
+                                              ctypes.byref(n)), "statekv_block_workspace_bytes")
+    return n.value
+
+
+def statekv_block_frame(handle: int, bc: statekv_block_config, weights, stream_begin: int,
+                        stream_count: int, layer_begin: int, layer_count: int, x_in: int,
+                        x_out: int, workspace: int, workspace_bytes: int, stream: int) -> int:
+    """``weights``: a ctypes array of statekv_block_weights, one per layer."""
+    return lib().statekv_block_frame(handle, ctypes.byref(bc), weights, stream_begin, stream_count,
+                                     layer_begin, layer_count, ctypes.c_void_p(x_in),
+                                     ctypes.c_void_p(x_out), ctypes.c_void_p(workspace),
+                                     workspace_bytes, ctypes.c_void_p(stream))
+
+
+def block_weights_array(layers) -> ctypes.Array:
+    """ctypes array of statekv_block_weights from per-layer dicts of device
+    tensors (keys norm_attn, w_qkv, b_qkv (or None), w_o, norm_mlp, w_gate_up,
+    w_down)."""
+    arr = (statekv_block_weights * len(layers))()
+    for i, w in enumerate(layers):
+        arr[i] = statekv_block_weights(
+            w["norm_attn"].data_ptr(), w["w_qkv"].data_ptr(),
+            w["b_qkv"].data_ptr() if w.get("b_qkv") is not None else None, w["w_o"].data_ptr(),
+            w["norm_mlp"].data_ptr(), w["w_gate_up"].data_ptr(), w["w_down"].data_ptr())
+    return arr
+
+
 def statekv_destroy(handle: int):
     lib().statekv_destroy(handle)
 
@@ -365,6 +417,25 @@ class StateKV:
         lc = self.cfg.num_layers if layer_count is None else layer_count
         return statekv_scores_workspace_bytes(self.handle, sc, lc)
 
+    def block_frame(self, bc, weights, x_in, x_out, workspace, *, stream_begin=0,
+                    stream_count=None, layer_begin=0, layer_count=None, stream=None) -> int:
+        """The next frame of the streams through layers [layer_begin, +count) of
+        the transformer block (x: bf16 [S][T][hidden]); ``weights``: from
+        ``block_weights_array``; ``workspace``: uint8 device tensor of
+        ``block_workspace_bytes`` bytes.  Returns the C status."""
+        import torch
+
+        sc = self.cfg.num_streams - stream_begin if stream_count is None else stream_count
+        lc = self.cfg.num_layers - layer_begin if layer_count is None else layer_count
+        st = (stream or torch.cuda.current_stream()).cuda_stream
+        return statekv_block_frame(self.handle, bc, weights, stream_begin, sc, layer_begin, lc,
+                                   x_in.data_ptr(), x_out.data_ptr(), workspace.data_ptr(),
+                                   workspace.numel(), st)
+
+    def block_workspace_bytes(self, bc, stream_count=None) -> int:
+        sc = self.cfg.num_streams if stream_count is None else stream_count
+        return statekv_block_workspace_bytes(self.handle, bc, sc)
+
     def decode_step(self, q, k, v, out, *, stream_begin=0, stream_count=None, layer_begin=0,
                     layer_count=None, stream=None) -> int:
         """Enqueue ``q.shape[2]`` new tokens per (stream, layer) over the decode
@@ -428,7 +499,7 @@ class StateKV:
 
     def profile_read(self):
         p = statekv_profile_read(self.handle)
-        return [(int(p.launches[i]), float(p.milliseconds[i])) for i in range(3)]
+        return [(int(p.launches[i]), float(p.milliseconds[i])) for i in range(5)]
 
     def sync(self) -> int:
         return statekv_sync(self.handle)
