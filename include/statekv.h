@@ -95,9 +95,10 @@ typedef struct {
 statekv_status statekv_arena_bytes(const statekv_config* cfg, size_t* bytes);
 
 /* Creates a handle over a caller-owned device arena of at least
- * statekv_arena_bytes() bytes (256-byte aligned).  Zeroes the states
- * (synchronously); every stream/layer starts at frame 1 with an empty state.
- * The arena must outlive the handle. */
+ * statekv_arena_bytes() bytes (256-byte aligned), whose prior contents do not
+ * matter.  Zeroes the states and the decode caches (synchronously); every
+ * stream/layer starts at frame 1 with an empty state.  The arena must outlive
+ * the handle. */
 statekv_status statekv_init(const statekv_config* cfg, void* device_arena, size_t arena_bytes,
                             statekv_handle** out);
 
@@ -362,7 +363,10 @@ statekv_status statekv_device_error(const statekv_handle* h, int32_t* code);
  *                 state_capacity (B), causal_in_frame, softmax_scale,
  *                 watchdog_ms are used; the rest is ignored
  *   q, k, v       bf16 [T][Hq][d], [T][Hkv][d], [T][Hkv][d] (device)
- *   state_k/v     bf16 [Hkv][B][d] (device); rows [0, state_count) are valid
+ *   state_k/v     bf16 [Hkv][B][d] (device); rows [0, state_count) are valid;
+ *                 the rows after them, up to the next multiple of 128 (or B),
+ *                 are read by the last key tile and must hold finite values
+ *                 (zeros, say): their weights are 0, but 0 times NaN is NaN
  *   out           bf16 [T][Hq][d] (device)
  *   importance    fp32 [Hkv][B + T] (device), columns as in statekv_frame_args
  * Nothing of the handle-based state is read or written. */

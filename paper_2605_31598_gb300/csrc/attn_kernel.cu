@@ -24,7 +24,7 @@
 //
 // 384 threads, three warpgroups:
 //   WG0  warp 0 producer (TMA), warps 1 and 3 MMA issuers X and Y (warp 1
-//        also owns TMEM).  tcgen05.mma issue blocks at the tensor core's pace,
+//        also owns TMEM), warp 2 the pass-B column-sum reducer.  tcgen05.mma issue blocks at the tensor core's pace,
 //        so each barrier wait of an issuing thread idles the tensor core; with
 //        two issuers one waits while the other's MMAs run.  X issues the
 //        pass-A Q K^T of even tiles and every pass-B Q K^T; Y the pass-A Q K^T
@@ -36,8 +36,9 @@
 //        tile while the other computes exponentials.  Pass B: both work on
 //        every tile, warpgroup w on keys [64 w, 64 w + 64), so each tile's P
 //        is ready after half a tile's work.
-// The column sums add a thread's rows in registers, then lanes by a shuffle
-// reduce-scatter, then the four warps of a warpgroup through shared memory.
+// The column sums add a thread's rows in registers; the reducer warp adds the
+// four warps' staged values per lane, then the lanes by a shuffle
+// reduce-scatter, and writes the tile's importance partials.
 // Every mbarrier wait is bounded by the watchdog; on expiry the CTA records
 // DEV_TIMEOUT_ATTN, drains its in-flight copies and MMAs, frees TMEM and exits.
 #include "sm103_ptx.cuh"
@@ -72,12 +73,13 @@ template <int D>
 struct AttnLayout {
     static constexpr int kTileBytes = kBN * D * 2;  // one K or V tile
     static constexpr int kOffSlots = 0;
-    static constexpr int kOffRed = kOffSlots + kSlots * kTileBytes;  // float[2 wg][2][4][128]
-    static constexpr int kOffStat = kOffRed + 2 * 2 * 4 * kBM * 4;   // float[5][128]
+    // column-sum staging of one pass-B tile: float[2 wg][4 quadrants][4 chunks][32 lanes][4]
+    static constexpr int kOffStage = kOffSlots + kSlots * kTileBytes;
+    static constexpr int kOffStat = kOffStage + 2 * 4 * 4 * 32 * 4 * 4;  // float[5][128]
     static constexpr int kOffBar = kOffStat + 5 * kBM * 4;
     // slot_full[6] slot_empty[6] sa_full[6] sa_read[6] sb_full[2] sb_read[2]
-    // p_full[2] pv_done[2] q_full o_full drain a_done a_read
-    static constexpr int kNumBars = 40;
+    // p_full[2] pv_done[2] q_full o_full drain a_done a_read stage_full stage_free
+    static constexpr int kNumBars = 42;
     static constexpr int kOffMisc = kOffBar + kNumBars * 8;
     static constexpr int kBytes = kOffMisc + 16;
     static constexpr int kAlloc = kBytes + 1024;  // room to align the base to 1 KB
@@ -285,30 +287,29 @@ __device__ __forceinline__ void tmem_st_16x128b_x8(uint32_t taddr, const uint32_
         : "memory");
 }
 
-// Sums over the 8 lanes that share lane % 4 (lane bits 2..4) of 16 values,
-// as a reduce-scatter: lane l returns the sums of values 2 (l/4) and
-// 2 (l/4) + 1.
-__device__ __forceinline__ void lane8_reduce_scatter16(float (&x)[16], int lane, float (&out)[2])
+// Sums over the 8 lanes that share lane % 4 (lane bits 2..4) of 32 values,
+// as a reduce-scatter: lane l returns the sums of values 4 (l/4) .. +3.
+__device__ __forceinline__ void lane8_reduce_scatter(float (&x)[32], int lane, float (&out)[4])
 {
 #pragma unroll
-    for (int i = 0; i < 8; ++i) {
+    for (int i = 0; i < 16; ++i) {
         const bool up = (lane & 16) != 0;
-        const float send = up ? x[i] : x[i + 8];
-        const float keep = up ? x[i + 8] : x[i];
+        const float send = up ? x[i] : x[i + 16];
+        const float keep = up ? x[i + 16] : x[i];
         x[i] = keep + __shfl_xor_sync(0xffffffffu, send, 16);
     }
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
+    for (int i = 0; i < 8; ++i) {
         const bool up = (lane & 8) != 0;
-        const float send = up ? x[i] : x[i + 4];
-        const float keep = up ? x[i + 4] : x[i];
+        const float send = up ? x[i] : x[i + 8];
+        const float keep = up ? x[i + 8] : x[i];
         x[i] = keep + __shfl_xor_sync(0xffffffffu, send, 8);
     }
 #pragma unroll
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < 4; ++i) {
         const bool up = (lane & 4) != 0;
-        const float send = up ? x[i] : x[i + 2];
-        const float keep = up ? x[i + 2] : x[i];
+        const float send = up ? x[i] : x[i + 4];
+        const float keep = up ? x[i + 4] : x[i];
         out[i] = keep + __shfl_xor_sync(0xffffffffu, send, 4);
     }
 }
@@ -325,7 +326,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
     uint8_t* sSlot = sm + L::kOffSlots;
-    float* red = reinterpret_cast<float*>(sm + L::kOffRed);
+    float4* stage = reinterpret_cast<float4*>(sm + L::kOffStage);
     float* stat = reinterpret_cast<float*>(sm + L::kOffStat);
     uint64_t* bars = reinterpret_cast<uint64_t*>(sm + L::kOffBar);
     uint64_t* slot_full = bars + 0;
@@ -341,6 +342,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t* drain = bars + 34;
     uint64_t* a_done = bars + 35;   // every pass-A MMA has completed
     uint64_t* a_read = bars + 36;   // both warpgroups have read every pass-A score tile
+    uint64_t* stage_full = bars + 37;  // pass B: the tile's column sums are staged
+    uint64_t* stage_free = bars + 38;  // pass B: the reducer warp has read them
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + L::kOffMisc);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(sm + L::kOffMisc + 4);
 
@@ -401,6 +404,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(&pv_done[i], 1);
         }
         mbar_init(a_read, 256);
+        mbar_init(stage_full, 256);
+        mbar_init(stage_free, 32);
         mbar_init(q_full, 256);
         mbar_init(o_full, 1);
         mbar_init(drain, 2);   // one commit per MMA issuer
@@ -425,7 +430,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     };
 
     if (warp < 4) {
-        asm volatile("setmaxnreg.dec.sync.aligned.u32 80;" ::: "memory");
+        asm volatile("setmaxnreg.dec.sync.aligned.u32 96;" ::: "memory");
         if (warp == 0) {
             // ------------------------------------------------------------ producer
             // One ring of tiles for both passes; with a cluster, this CTA loads
@@ -493,6 +498,56 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             }
             __syncwarp();
+        } else if (warp == 2) {
+            // ------------------------------------------------------------ column-sum reducer
+            // Pass B, per tile: the softmax threads stage their 16 row-summed
+            // values (4 rows each); lane L adds the 4 quadrants' values of
+            // staging lane L, then the 8 lanes that share L % 4 reduce-scatter
+            // 32 values, leaving lane L with columns 64 wg + 16 jj + 8 h + 2 (L % 4) + e
+            // (wg = m / 4, jj = m % 4, m = L / 4; h, e in {0, 1}).
+            float* part = p.partials ? p.partials + ((static_cast<size_t>(u) * p.Hkv + hkv) * p.MT + mt) * p.P
+                                     : nullptr;
+            bool ok = true;
+            for (int j = 0; j < nt && ok && part != nullptr; ++j) {
+                ok = __all_sync(0xffffffffu, wait_until(stage_full, j & 1, deadline));
+                if (!ok) {
+                    if (lane == 0) fail(13);
+                    break;
+                }
+                float x[32];  // index (wg * 4 + jj) * 4 + i
+#pragma unroll
+                for (int w2 = 0; w2 < 2; ++w2)
+#pragma unroll
+                    for (int jj = 0; jj < 4; ++jj) {
+                        float4 a = stage[((w2 * 4 + 0) * 4 + jj) * 32 + lane];
+#pragma unroll
+                        for (int q = 1; q < 4; ++q) {
+                            const float4 b4 = stage[((w2 * 4 + q) * 4 + jj) * 32 + lane];
+                            a.x += b4.x;
+                            a.y += b4.y;
+                            a.z += b4.z;
+                            a.w += b4.w;
+                        }
+                        const int o = (w2 * 4 + jj) * 4;
+                        x[o] = a.x;
+                        x[o + 1] = a.y;
+                        x[o + 2] = a.z;
+                        x[o + 3] = a.w;
+                    }
+                mbar_arrive(stage_free);  // the softmax threads may stage the next tile
+                float sum4[4];
+                lane8_reduce_scatter(x, lane, sum4);
+                if (tile_valid) {
+                    const int m4 = lane >> 2, cbase = 64 * (m4 >> 2) + 16 * (m4 & 3) + 2 * (lane & 3);
+                    const bool is_state = j < nst;
+                    const int kb = (is_state ? state_tile(j) : j - nst) * kBN;
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        const int key = kb + cbase + 8 * (i >> 1) + (i & 1);
+                        if (is_state ? key < count : key < T) part[is_state ? key : B + key] = sum4[i];
+                    }
+                }
+            }
         } else if (warp == 1 || warp == 3) {
             // ------------------------------------------------------------ MMA issuers
             if (lane == 0) {
@@ -611,7 +666,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (warp == 1) tmem_dealloc(tbase, 512);
         if (C > 1) cluster_sync_all();  // no CTA leaves while its partner may still write to it
     } else {
-        asm volatile("setmaxnreg.inc.sync.aligned.u32 208;" ::: "memory");
+        asm volatile("setmaxnreg.inc.sync.aligned.u32 200;" ::: "memory");
         // ------------------------------------------------------------ softmax warpgroups
         const int wg = (warp >> 2) - 1;          // 0 or 1
         const int quad = warp & 3;               // TMEM lane quadrant of this warp
@@ -668,6 +723,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             tmem_ld_wait();
             tc_fence_before();
             mbar_arrive(&sa_read[it % kSA2]);
+            // after its last tile is in registers, this thread holds no pass-A
+            // score buffer: pass B's Q K^T may start while the sums finish
+            if (it + 2 >= nt) mbar_arrive(a_read);
             if (lim < kBN) {
 #pragma unroll
                 for (int ch = 0; ch < 4; ++ch)
@@ -702,7 +760,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 m = m_new;
             }
         }
-        mbar_arrive(a_read);  // every pass-A tile of this thread has been read
+        if (wg >= nt) mbar_arrive(a_read);  // a warpgroup without pass-A tiles
         if (ok) site = 11;
         stat[(wg * 2 + 0) * kBM + row] = m;
         stat[(wg * 2 + 1) * kBM + row] = l;
@@ -742,8 +800,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
         float* part = p.partials ? p.partials + ((static_cast<size_t>(u) * p.Hkv + hkv) * p.MT + mt) * p.P
                                  : nullptr;
-        float* myred = red + wg * (2 * 4 * kBM);
-        const int ct = threadIdx.x - 128 - 128 * wg;  // 0..127 within the warpgroup
+        float4* mystage = stage + (wg * 4 + quad) * 4 * 32 + lane;  // chunk jj at + jj * 32
         const int cq = 2 * (lane & 3);                // this thread's column offset in 8
         const int c0 = 64 * wg;                       // this warpgroup's first key of a tile
         const uint32_t tSh0 = tbase + lane_off + kColS0 + c0;   // this warpgroup's S0 half
@@ -755,7 +812,6 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int b = j & 1;
             if (ok) ok = __all_sync(0xffffffffu, wait_until(&sb_full[b], (j >> 1) & 1, deadline));
             const bool is_state = j < nst;
-            float* rb = myred + b * (4 * kBM);  // [4 warps][64 columns]
             if (ok) {
                 tc_fence_after();
                 int lim4[4];  // keys [0, lim) of this tile are visible to each row
@@ -818,27 +874,27 @@ __global__ void __launch_bounds__(kThreads, 1)
                     tc_fence_before();
                     mbar_arrive(&p_full[b]);
                     // the column sums run while the tensor core does this tile's P V:
-                    // value 2r + e is column 8r + cq + e summed over the thread's rows
-                    float cs[16];
+                    // value 2r + e is column 8r + cq + e summed over the thread's rows;
+                    // the reducer warp adds them across lanes and warps
+                    if (part != nullptr) {
+                        float cs[16];
 #pragma unroll
-                    for (int r = 0; r < 8; ++r) {
-                        const f2 a = add2(pk(v[0][4 * r], v[0][4 * r + 1]), pk(v[0][4 * r + 2], v[0][4 * r + 3]));
-                        const f2 bb = add2(pk(v[1][4 * r], v[1][4 * r + 1]), pk(v[1][4 * r + 2], v[1][4 * r + 3]));
-                        upk(add2(a, bb), cs[2 * r], cs[2 * r + 1]);
+                        for (int r = 0; r < 8; ++r) {
+                            const f2 a = add2(pk(v[0][4 * r], v[0][4 * r + 1]), pk(v[0][4 * r + 2], v[0][4 * r + 3]));
+                            const f2 bb = add2(pk(v[1][4 * r], v[1][4 * r + 1]), pk(v[1][4 * r + 2], v[1][4 * r + 3]));
+                            upk(add2(a, bb), cs[2 * r], cs[2 * r + 1]);
+                        }
+                        if (j >= 1)  // the reducer has read the previous tile's values
+                            ok = __all_sync(0xffffffffu, wait_until(stage_free, (j - 1) & 1, deadline));
+                        if (ok) {
+#pragma unroll
+                            for (int jj = 0; jj < 4; ++jj)
+                                mystage[jj * 32] = make_float4(cs[4 * jj], cs[4 * jj + 1], cs[4 * jj + 2],
+                                                               cs[4 * jj + 3]);
+                            mbar_arrive(stage_full);
+                        }
                     }
-                    float sum2[2];
-                    lane8_reduce_scatter16(cs, lane, sum2);
-                    // this lane holds values 2m, 2m + 1 (m = lane / 4): columns 8m + cq + e
-                    const int m4 = lane >> 2;
-                    rb[quad * 64 + 8 * m4 + cq] = sum2[0];
-                    rb[quad * 64 + 8 * m4 + cq + 1] = sum2[1];
                 }
-            }
-            named_bar_sync(2 + wg, 128);
-            if (ok && tile_valid && part != nullptr && ct < 64) {
-                const float s = rb[0 * 64 + ct] + rb[1 * 64 + ct] + rb[2 * 64 + ct] + rb[3 * 64 + ct];
-                const int key = (is_state ? state_tile(j) : j - nst) * kBN + c0 + ct;
-                if (is_state ? key < count : key < T) part[is_state ? key : B + key] = s;
             }
         }
         if (ok) site = 12;
@@ -882,11 +938,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 }
 
-// The register split (WG0 down to 80, the softmax warpgroups up to 208 per
+// The register split (WG0 down to 96, the softmax warpgroups up to 200 per
 // thread) must fit the registers the CTA is launched with, or setmaxnreg.inc
-// would wait forever: 128 * 80 + 256 * 208 = 63488 <= 384 threads * 168.
+// would wait forever: 128 * 96 + 256 * 200 = 63488 <= 384 threads * 168.
 constexpr int kLaunchRegs = 168;
-static_assert(128 * 80 + 256 * 208 <= kThreads * kLaunchRegs, "register split");
+static_assert(128 * 96 + 256 * 200 <= kThreads * kLaunchRegs, "register split");
 
 // Query tiles per cluster for head dim D: two CTAs share each K/V tile by
 // multicast (one 64-column half each) when D = 128.

@@ -508,10 +508,14 @@ statekv_status statekv_init(const statekv_config* cfg, void* device_arena, size_
         ok = encode_4d(&h->tm_ck, h->arena + lay.cache_k, dims, strides, box) &&
              encode_4d(&h->tm_cv, h->arena + lay.cache_v, dims, strides, box);
     }
-    // Empty states: zero rows (masked keys must still be finite), positions -1.
+    // Empty states and decode caches: zero rows, positions -1.  A key tile that
+    // runs past the valid rows of a state or of the cache still reads them;
+    // their scores are masked, but P = 0 times a non-finite value row would
+    // still be NaN, so every row a tile can reach must hold finite values.
     ok = ok && cudaMemset(h->arena + lay.state_k, 0, lay.positions - lay.state_k) == cudaSuccess &&
          cudaMemset(h->arena + lay.positions, 0xFF, lay.counts - lay.positions) == cudaSuccess &&
          cudaMemset(h->arena + lay.counts, 0, lay.cache_k - lay.counts) == cudaSuccess &&
+         cudaMemset(h->arena + lay.cache_k, 0, lay.partials - lay.cache_k) == cudaSuccess &&
          cudaDeviceSynchronize() == cudaSuccess;
     if (!ok) {
         cudaFreeHost(st_host);

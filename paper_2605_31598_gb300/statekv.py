@@ -346,12 +346,17 @@ def make_config(shape, *, causal=True, host_staging=False, softmax_scale=0.0,
 class StateKV:
     """Owns a handle and its torch-allocated device arena."""
 
-    def __init__(self, cfg: statekv_config, device="cuda"):
+    def __init__(self, cfg: statekv_config, device="cuda", arena=None):
+        """``arena``: optional caller-owned uint8 device tensor of at least
+        ``statekv_arena_bytes(cfg)`` bytes (its prior contents do not matter)."""
         import torch
 
         self.cfg = cfg
         self.nbytes = statekv_arena_bytes(cfg)
-        self.arena = torch.empty(max(self.nbytes, 256), dtype=torch.uint8, device=device)
+        if arena is None:
+            arena = torch.empty(max(self.nbytes, 256), dtype=torch.uint8, device=device)
+        assert arena.dtype == torch.uint8 and arena.numel() >= self.nbytes
+        self.arena = arena
         self.handle = statekv_init(cfg, self.arena.data_ptr(), self.nbytes)
 
     def close(self):

@@ -90,3 +90,42 @@ def test_full_attention_changes_no_state_and_refuses_importance():
         assert torch.equal(a, b)
     assert (info_before.count, info_before.virtual_len) == (info_after.count, info_after.virtual_len)
     assert eng.sync() == 0
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("name", ["toy", "qwen7b_layer"])
+def test_arena_prefilled_with_nan_changes_nothing(name):
+    """The arena's prior contents do not matter: every byte 0xFF (bf16 NaN)
+    before statekv_init.  Key tiles that run past the valid cache or state
+    rows read them, so init must leave them finite; full attention and the
+    method's step must match the oracle as on fresh memory."""
+    import __graft_entry__ as g
+
+    g.build()
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    shape = dataclasses.replace(WORKLOADS[name], max_frames=5)
+    S, L, T = shape.num_streams, shape.num_layers, shape.tokens_per_frame
+    cfg = make_config(shape)
+    from paper_2605_31598_gb300 import statekv
+
+    arena = torch.full((statekv.statekv_arena_bytes(cfg),), 0xFF, dtype=torch.uint8, device="cuda")
+    eng = StateKV(cfg, arena=arena)
+    hk, hv = [], []
+    for n in range(1, 5):
+        q, k, v = batch_qkv(shape, n, streams=range(S), layers=range(L), device="cuda")
+        hk.append(oracle.as_bf16_bits(k[0, 0]))
+        hv.append(oracle.as_bf16_bits(v[0, 0]))
+        out = torch.full_like(q, float("nan"))
+        assert eng.full_attention_frame(q, k, v, out) == 0
+        torch.cuda.synchronize()
+        ref = oracle.full_attention(oracle.as_bf16_bits(q[0, 0]), np.concatenate(hk),
+                                    np.concatenate(hv), (n - 1) * T)
+        got = out[0, 0].float().cpu().numpy()
+        assert np.isfinite(got).all(), f"frame {n}: non-finite output"
+        assert float(np.abs(got - ref).max()) <= OUT_ATOL
+        step_out = torch.full_like(q, float("nan"))
+        assert eng.prefill_frame(q, k, v, step_out) == 0
+        torch.cuda.synchronize()
+        assert torch.isfinite(step_out.float()).all(), f"frame {n}: non-finite step output"
+    assert eng.sync() == 0
