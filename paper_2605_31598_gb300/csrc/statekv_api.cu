@@ -152,6 +152,11 @@ struct statekv_handle {
     size_t prof_used;
     std::vector<ProfRec> prof;
     LtContext* lt = nullptr;   // cuBLASLt, created by the first block call
+    // The decode-cache append runs on a side stream forked from the call's
+    // stream and joined before the selection: it depends on nothing the
+    // attention kernel writes, so it fills SMs the attention grid leaves idle.
+    cudaStream_t side = nullptr;
+    cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
 
     template <class T>
     T* at(size_t off) const { return reinterpret_cast<T*>(arena + off); }
@@ -242,7 +247,12 @@ statekv_status run_step(statekv_handle* h, const statekv_frame_args& a, cudaStre
     ap.D = D;
     ap.row_mul = T;
     ap.cap = d.cap;
-    if (timed(h, 0, st, [&] { return launch_append(ap, st); }) != cudaSuccess)
+    // append on the side stream; it reads the frame counters, so the join
+    // comes before the selection kernel advances them
+    if (cudaEventRecord(h->ev_fork, st) != cudaSuccess ||
+        cudaStreamWaitEvent(h->side, h->ev_fork, 0) != cudaSuccess ||
+        timed(h, 0, h->side, [&] { return launch_append(ap, h->side); }) != cudaSuccess ||
+        cudaEventRecord(h->ev_join, h->side) != cudaSuccess)
         return STATEKV_ERR_CUDA;
 
     AttnParams pa{};
@@ -263,9 +273,10 @@ statekv_status run_step(statekv_handle* h, const statekv_frame_args& a, cudaStre
     pa.count_mul = 1;
     pa.scale_log2 = d.scale * 1.4426950408889634f;
     pa.watchdog_ns = 1000000ull * (c.watchdog_ms ? c.watchdog_ms : 2000u);
-    if (timed(h, 1, st, [&] { return launch_attn(D, h->tm_sk, h->tm_sv, tm_fk, tm_fv, pa, U, st); }) !=
-        cudaSuccess)
-        return STATEKV_ERR_CUDA;
+    const cudaError_t ek =
+        timed(h, 1, st, [&] { return launch_attn(D, h->tm_sk, h->tm_sv, tm_fk, tm_fv, pa, U, st); });
+    const cudaError_t ej = cudaStreamWaitEvent(st, h->ev_join, 0);  // the append is done
+    if (ek != cudaSuccess || ej != cudaSuccess) return STATEKV_ERR_CUDA;
 
     if (c.selection == 1) {
         RecencyParams pr{};
@@ -508,6 +519,9 @@ statekv_status statekv_init(const statekv_config* cfg, void* device_arena, size_
         ok = encode_4d(&h->tm_ck, h->arena + lay.cache_k, dims, strides, box) &&
              encode_4d(&h->tm_cv, h->arena + lay.cache_v, dims, strides, box);
     }
+    ok = ok && cudaStreamCreateWithFlags(&h->side, cudaStreamNonBlocking) == cudaSuccess &&
+         cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming) == cudaSuccess &&
+         cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming) == cudaSuccess;
     // Empty states and decode caches: zero rows, positions -1.  A key tile that
     // runs past the valid rows of a state or of the cache still reads them;
     // their scores are masked, but P = 0 times a non-finite value row would
@@ -519,6 +533,9 @@ statekv_status statekv_init(const statekv_config* cfg, void* device_arena, size_
          cudaDeviceSynchronize() == cudaSuccess;
     if (!ok) {
         cudaFreeHost(st_host);
+        if (h->ev_fork) cudaEventDestroy(h->ev_fork);
+        if (h->ev_join) cudaEventDestroy(h->ev_join);
+        if (h->side) cudaStreamDestroy(h->side);
         delete h;
         return STATEKV_ERR_CUDA;
     }
@@ -966,6 +983,9 @@ void statekv_destroy(statekv_handle* h)
     }
     cudaFreeHost(const_cast<int32_t*>(h->status_host));
     lt_destroy(h->lt);
+    if (h->ev_fork) cudaEventDestroy(h->ev_fork);
+    if (h->ev_join) cudaEventDestroy(h->ev_join);
+    if (h->side) cudaStreamDestroy(h->side);
     delete h;
 }
 
