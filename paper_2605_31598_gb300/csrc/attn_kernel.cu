@@ -1,6 +1,6 @@
 // K1: frame attention with saved log-sum-exp and fused importance partials.
 //
-// One CTA owns 128 query rows of one KV-head group of one (stream, layer).
+// A work unit is 128 query rows of one KV-head group of one (stream, layer).
 // Rows are packed token-major, row r = t * G + g (query head hkv*G + g of
 // token t), so a tile covers ~128/G consecutive tokens and the in-frame
 // causal mask of Eq. 5 skips every frame-key tile beyond its last token.
@@ -18,18 +18,22 @@
 // K and V tiles stream through a ring of six 32 KB shared-memory slots in one
 // sequence, pass A's K tiles, then pass B's K(0) V(0) K(1) V(1) ...; a slot is
 // refilled once the MMAs that read it have completed (their commit arrives on
-// the slot's barrier).  Optionally (cluster_size() below) two CTAs of
-// consecutive query tiles share each K/V tile by TMA multicast, each loading
-// one 64-column half into both CTAs' shared memory.
+// the slot's barrier).
+//
+// The kernel is persistent: one CTA per SM walks work units (query tile, KV
+// head, unit) in a fixed stride.  Ring, TMEM and barriers carry over from one
+// unit to the next, so the producer loads the next unit's first tiles while
+// the current one finishes, the next unit's Q goes into TMEM as soon as the
+// last P V completes, and its first Q K^T run while the previous O is read out.
 //
 // 384 threads, three warpgroups:
 //   WG0  warp 0 producer (TMA), warps 1 and 3 MMA issuers X and Y (warp 1
-//        also owns TMEM), warp 2 the pass-B column-sum reducer.  tcgen05.mma issue blocks at the tensor core's pace,
-//        so each barrier wait of an issuing thread idles the tensor core; with
-//        two issuers one waits while the other's MMAs run.  X issues the
-//        pass-A Q K^T of even tiles and every pass-B Q K^T; Y the pass-A Q K^T
-//        of odd tiles and every P V (in order, so O accumulates
-//        deterministically).  Descriptors are precomputed words, so an MMA
+//        also owns TMEM), warp 2 the pass-B column-sum reducer.  tcgen05.mma
+//        issue blocks at the tensor core's pace, so each barrier wait of an
+//        issuing thread idles the tensor core; with two issuers one waits
+//        while the other's MMAs run.  X issues the pass-A Q K^T of even tiles
+//        and every pass-B Q K^T; Y the pass-A Q K^T of odd tiles and every
+//        P V (in order, so O accumulates deterministically).  Descriptors are precomputed words, so an MMA
 //        costs the issuing warp an add or two besides itself.
 //   WG1, WG2  softmax warpgroups.  Pass A: thread = query row; they take
 //        alternate key tiles, so the tensor core works on one warpgroup's
@@ -79,7 +83,8 @@ struct AttnLayout {
     static constexpr int kOffBar = kOffStat + 5 * kBM * 4;
     // slot_full[6] slot_empty[6] sa_full[6] sa_read[6] sb_full[2] sb_read[2]
     // p_full[2] pv_done[2] q_full o_full drain a_done a_read stage_full stage_free
-    static constexpr int kNumBars = 42;
+    // o_read
+    static constexpr int kNumBars = 40;
     static constexpr int kOffMisc = kOffBar + kNumBars * 8;
     static constexpr int kBytes = kOffMisc + 16;
     static constexpr int kAlloc = kBytes + 1024;  // room to align the base to 1 KB
@@ -188,45 +193,6 @@ __device__ __forceinline__ void mma_group(uint32_t d, uint32_t a, uint32_t blo, 
     }
 }
 
-__device__ __forceinline__ uint32_t cluster_ctarank()
-{
-    uint32_t r;
-    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
-    return r;
-}
-
-// Every thread of every CTA in the cluster arrives and waits.
-__device__ __forceinline__ void cluster_sync_all()
-{
-    asm volatile(
-        "barrier.cluster.arrive.release.aligned;\n\t"
-        "barrier.cluster.wait.acquire.aligned;" ::: "memory");
-}
-
-// TMA tile load delivered to the same shared-memory offset, and completing on
-// the same mbarrier offset, in every CTA of `mask`.
-__device__ __forceinline__ void tma_load_4d_mc(void* dst, const void* tmap, uint64_t* bar, int c0,
-                                               int c1, int c2, int c3, uint16_t mask)
-{
-    asm volatile(
-        "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes"
-        ".multicast::cluster [%0], [%1, {%3, %4, %5, %6}], [%2], %7;" ::"r"(smem_addr(dst)),
-        "l"(reinterpret_cast<uint64_t>(tmap)), "r"(smem_addr(bar)), "r"(c0), "r"(c1), "r"(c2),
-        "r"(c3), "h"(mask)
-        : "memory");
-}
-
-// Arrives once on `bar` in every CTA of `mask` when this thread's MMAs so far
-// have completed.
-__device__ __forceinline__ void umma_commit_mc(uint64_t* bar, uint16_t mask)
-{
-    asm volatile(
-        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
-        " [%0], %1;" ::"r"(smem_addr(bar)),
-        "h"(mask)
-        : "memory");
-}
-
 // 16 consecutive 32-bit TMEM columns of this thread's lane <- registers.
 __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16])
 {
@@ -242,14 +208,6 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16
 __device__ __forceinline__ void tmem_st_wait()
 {
     asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
-}
-
-// The ring carries pass A's K tiles (items 0 .. nt-1), then pass B's K(j)
-// (item nt + 2j) and V(j) (item nt + 2j + 1); item n sits in slot n % 6 as the
-// slot's use n / 6.
-__device__ __forceinline__ int qk_item(int nt, int it)  // it: Q K^T sequence index
-{
-    return it < nt ? it : nt + 2 * (it - nt);
 }
 
 // 16 TMEM lanes x 64 columns -> 32 registers (.16x256b layout): register
@@ -314,7 +272,52 @@ __device__ __forceinline__ void lane8_reduce_scatter(float (&x)[32], int lane, f
     }
 }
 
-template <int D, int C>  // C: CTAs per cluster sharing K/V tiles (1 or 2)
+// One work unit: the 128 query rows of tile mt of KV head hkv of the call's
+// unit u, with the key range the unit sees.  Units are numbered with the tile
+// fastest, then the KV head, then the unit.
+struct WorkUnit {
+    int mt, hkv, u, ua;
+    int count;  // visible keys before the frame (state slots or cache rows)
+    int nst;    // key tiles over them
+    int nft;    // frame key tiles the tile's last row can see
+    int nt;     // nst + nft
+    int rot;    // first state tile (see state_tile)
+};
+
+__device__ __forceinline__ WorkUnit work_unit(const AttnParams& p, int w)
+{
+    WorkUnit x;
+    x.mt = w % p.MT;
+    const int r = w / p.MT;
+    x.hkv = r % p.Hkv;
+    x.u = r / p.Hkv;
+    x.ua = p.units.unit_abs(x.u);
+    const int head = x.ua * p.Hkv + x.hkv;
+    x.count = p.count_mul * ((p.B > 0 || p.count_mul > 1) ? p.counts[head] : 0) +
+              (p.count_add ? p.count_add[head] : 0);
+    x.nst = (x.count + kBN - 1) / kBN;
+    const int row_hi = min(p.G * p.T, (x.mt + 1) * kBM) - 1;
+    x.nft = p.causal ? (row_hi / p.G) / kBN + 1 : (p.T + kBN - 1) / kBN;
+    x.nt = x.nst + x.nft;
+    // The query tiles of one KV head read the same state tiles; each starts at
+    // a different one (a fixed rotation) so they do not all request the same
+    // L2 lines at the same moment.  Frame tiles keep their order.
+    x.rot = x.nst > 0 ? (x.mt * 3) % x.nst : 0;
+    return x;
+}
+
+__device__ __forceinline__ int state_tile(const WorkUnit& x, int t)
+{
+    return t + x.rot < x.nst ? t + x.rot : t + x.rot - x.nst;
+}
+
+// Persistent: one CTA per SM walks the work units w = blockIdx.x, + gridDim.x,
+// ...  The ring, the TMEM allocation and every barrier live across units: the
+// producer loads the next unit's first tiles while the current one finishes,
+// and the per-tile barrier phases continue from unit to unit (tb below counts
+// the key tiles of the CTA's earlier units, so tile it of pass A is global
+// tile tb + it, and item i of the ring is global item 3 tb + i).
+template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
     frame_attn_lse_importance(const __grid_constant__ CUtensorMap tm_sk,
                               const __grid_constant__ CUtensorMap tm_sv,
@@ -331,67 +334,52 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t* bars = reinterpret_cast<uint64_t*>(sm + L::kOffBar);
     uint64_t* slot_full = bars + 0;
     uint64_t* slot_empty = bars + 6;
-    uint64_t* sa_full = bars + 12;  // pass A: Q K^T of tile i done (index i % 6)
-    uint64_t* sa_read = bars + 18;  // pass A: tile i read by its warpgroup (index i % 6)
-    uint64_t* sb_full = bars + 24;  // pass B: Q K^T of tile j in score buffer j & 1
+    uint64_t* sa_full = bars + 12;  // pass A: Q K^T of global tile g done (index g % 6)
+    uint64_t* sa_read = bars + 18;  // pass A: global tile g read by its warpgroup (index g % 6)
+    uint64_t* sb_full = bars + 24;  // pass B: Q K^T of global tile g in score buffer g & 1
     uint64_t* sb_read = bars + 26;  // pass B: both warpgroups have read S0 ([1] unused)
-    uint64_t* p_full = bars + 28;   // pass B: both warpgroups have written P of tile j (j & 1)
-    uint64_t* pv_done = bars + 30;  // pass B: P V(j) has completed (index j & 1)
-    uint64_t* q_full = bars + 32;
-    uint64_t* o_full = bars + 33;
+    uint64_t* p_full = bars + 28;   // pass B: both warpgroups have written P of tile g (g & 1)
+    uint64_t* pv_done = bars + 30;  // pass B: P V of tile g has completed (index g & 1)
+    uint64_t* q_full = bars + 32;   // per unit: Q is in TMEM
+    uint64_t* o_full = bars + 33;   // per unit: every P V has completed
     uint64_t* drain = bars + 34;
-    uint64_t* a_done = bars + 35;   // every pass-A MMA has completed
-    uint64_t* a_read = bars + 36;   // both warpgroups have read every pass-A score tile
+    uint64_t* a_done = bars + 35;   // per unit: every pass-A MMA has completed
+    uint64_t* a_read = bars + 36;   // per unit: both warpgroups have read every pass-A tile
     uint64_t* stage_full = bars + 37;  // pass B: the tile's column sums are staged
     uint64_t* stage_free = bars + 38;  // pass B: the reducer warp has read them
+    uint64_t* o_read = bars + 39;   // per unit: O has been read out of TMEM
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + L::kOffMisc);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(sm + L::kOffMisc + 4);
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
-    const int mt = blockIdx.x;  // query tile; tiles >= MT (cluster padding) have no valid row
-    const int hkv = blockIdx.y;
-    const int u = blockIdx.z;
-    const int ua = p.units.unit_abs(u);
     const int T = p.T, G = p.G, B = p.B;
     const int rows = G * T;
-    const bool tile_valid = mt < p.MT;
-    const int crank = C > 1 ? static_cast<int>(cluster_ctarank()) : 0;
-    const int count = p.count_mul * ((B > 0 || p.count_mul > 1) ? p.counts[ua * p.Hkv + hkv] : 0) +
-                      (p.count_add ? p.count_add[ua * p.Hkv + hkv] : 0);
-    const int nst = (count + kBN - 1) / kBN;
-    // frame tiles seen by the cluster's last query tile (the union over the cluster)
-    const int mt_last = min(mt - crank + C - 1, p.MT - 1);
-    const int row_hi = min(rows, (mt_last + 1) * kBM) - 1;
-    const int nft = p.causal ? (row_hi / G) / kBN + 1 : (T + kBN - 1) / kBN;
-    const int nt = nst + nft;
-    const int nitems = 3 * nt;  // pass-A K tiles + pass-B K and V tiles
-    // The clusters of one KV head read the same state tiles; each starts at a
-    // different one (a fixed rotation) so they do not all request the same L2
-    // lines at the same moment.  Frame tiles keep their order.
-    const int rot = nst > 0 ? ((mt / C) * 3) % nst : 0;
-    auto state_tile = [&](int t) { return t + rot < nst ? t + rot : t + rot - nst; };
-    const unsigned long long deadline = globaltimer() + p.watchdog_ns;
+    const int W = p.MT * p.Hkv * p.U;
+    const int w0 = blockIdx.x, wstep = gridDim.x;
 
-    // The softmax threads start loading their Q row now, so its global-memory
-    // latency overlaps the barrier and TMEM setup (thread 128 + i: warpgroup
-    // i / 128 - 1, row i % 128; warpgroup wg holds d in [64 wg, 64 wg + 64)).
+    // A softmax thread's Q row of unit w (thread 128 + i: warpgroup i / 128 - 1,
+    // row i % 128; warpgroup wg holds d in [64 wg, 64 wg + 64)).
     uint4 qreg[8];
-    {
+    auto load_q = [&](int w) {
+        const int mt = w % p.MT, r = w / p.MT, hkv = r % p.Hkv, u = r / p.Hkv;
         const int tq = static_cast<int>(threadIdx.x) - 128;
         const int qwg = tq >> 7, qrow = tq & 127, qr = mt * kBM + qrow;
-        const bool loads = tq >= 0 && qwg * 64 < D && qr < rows;
+        const bool loads = w < W && tq >= 0 && qwg * 64 < D && qr < rows;
         const int t = loads ? qr / G : 0, g = loads ? qr - t * G : 0;
         const uint4* src = reinterpret_cast<const uint4*>(
-            p.q + ((static_cast<size_t>(u) * T + t) * p.Hq + hkv * G + g) * D + (loads ? qwg * 64 : 0));
+            p.q + ((static_cast<size_t>(loads ? u : 0) * T + t) * p.Hq + (loads ? hkv : 0) * G + g) * D +
+            (loads ? qwg * 64 : 0));
 #pragma unroll
         for (int i = 0; i < 8; ++i) qreg[i] = loads ? src[i] : make_uint4(0u, 0u, 0u, 0u);
-    }
+    };
+    // the first unit's rows load while the barriers and TMEM are set up
+    load_q(w0);
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < kSlots; ++i) {
             mbar_init(&slot_full[i], 1);
-            mbar_init(&slot_empty[i], C);  // one MMA commit per CTA of the cluster
+            mbar_init(&slot_empty[i], 1);
         }
         for (int i = 0; i < kSA2; ++i) {
             mbar_init(&sa_full[i], 1);
@@ -408,6 +396,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_init(stage_free, 32);
         mbar_init(q_full, 256);
         mbar_init(o_full, 1);
+        mbar_init(o_read, 256);
         mbar_init(drain, 2);   // one commit per MMA issuer
         mbar_init(a_done, 2);
         *abort_flag = 0;
@@ -418,7 +407,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_relinquish();
     }
     __syncthreads();
-    if (C > 1) cluster_sync_all();  // the partner's barriers exist before any multicast
     tc_fence_after();
     const uint32_t tbase = *tmem_slot;
 
@@ -433,8 +421,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         asm volatile("setmaxnreg.dec.sync.aligned.u32 96;" ::: "memory");
         if (warp == 0) {
             // ------------------------------------------------------------ producer
-            // One ring of tiles for both passes; with a cluster, this CTA loads
-            // the d-half `crank` of every tile for both CTAs.
+            // One ring of tiles for both passes of every unit: per unit, pass A's
+            // K tiles, then pass B's K(0) V(0) K(1) V(1) ...
             if (lane == 0) {
                 tma_prefetch_desc(&tm_fk);
                 tma_prefetch_desc(&tm_fv);
@@ -445,56 +433,46 @@ __global__ void __launch_bounds__(kThreads, 1)
                 int last_use[kSlots];
 #pragma unroll
                 for (int sl = 0; sl < kSlots; ++sl) last_use[sl] = -1;
-                // map and coordinates of item n (this CTA's d-half when C = 2)
-                auto item_src = [&](int n, const CUtensorMap*& map, int& c1, int& c2, int& c3) {
-                    const bool is_v = n >= nt && ((n - nt) & 1);
-                    const int tile = n < nt ? n : (n - nt) >> 1;
-                    map = tile < nst ? (is_v ? &tm_sv : &tm_sk) : (is_v ? &tm_fv : &tm_fk);
-                    c1 = tile < nst ? state_tile(tile) * kBN : hkv;
-                    c2 = tile < nst ? hkv : (tile - nst) * kBN;
-                    c3 = tile < nst ? ua : u;
-                };
                 bool ok = true;
-                for (int n = 0; n < nitems; ++n) {
-                    if (*abort_flag) {
-                        ok = false;
-                        break;
-                    }
-                    const int slot = n % kSlots, use = n / kSlots;
-                    if (use >= 1 && !wait_until(&slot_empty[slot], (use - 1) & 1, deadline)) {
-                        fail(2);
-                        ok = false;
-                        break;
-                    }
-                    const CUtensorMap* map;
-                    int c1, c2, c3;
-                    item_src(n, map, c1, c2, c3);
-                    uint8_t* dst = sSlot + slot * L::kTileBytes;
-                    mbar_arrive_expect_tx(&slot_full[slot], L::kTileBytes);
-                    if (C == 1) {
+                int n = 0;  // global item
+                for (int w = w0; ok && w < W; w += wstep) {
+                    const WorkUnit x = work_unit(p, w);
+                    const unsigned long long deadline = globaltimer() + p.watchdog_ns;
+                    for (int i = 0; i < 3 * x.nt; ++i, ++n) {
+                        if (*abort_flag) {
+                            ok = false;
+                            break;
+                        }
+                        const int slot = n % kSlots, use = n / kSlots;
+                        if (use >= 1 && !wait_until(&slot_empty[slot], (use - 1) & 1, deadline)) {
+                            fail(2);
+                            ok = false;
+                            break;
+                        }
+                        const bool is_v = i >= x.nt && ((i - x.nt) & 1);
+                        const int tile = i < x.nt ? i : (i - x.nt) >> 1;
+                        const bool st = tile < x.nst;
+                        const CUtensorMap* map = st ? (is_v ? &tm_sv : &tm_sk) : (is_v ? &tm_fv : &tm_fk);
+                        const int c1 = st ? state_tile(x, tile) * kBN : x.hkv;
+                        const int c2 = st ? x.hkv : (tile - x.nst) * kBN;
+                        const int c3 = st ? x.ua : x.u;
+                        uint8_t* dst = sSlot + slot * L::kTileBytes;
+                        mbar_arrive_expect_tx(&slot_full[slot], L::kTileBytes);
 #pragma unroll
                         for (int h = 0; h < D / 64; ++h)
                             tma_load_4d(dst + h * (kBN * 128), map, &slot_full[slot], h * 64, c1, c2, c3);
-                    } else {
-                        tma_load_4d_mc(dst + crank * (kBN * 128), map, &slot_full[slot], crank * 64, c1,
-                                       c2, c3, static_cast<uint16_t>((1u << C) - 1));
+                        last_use[slot] = use;
                     }
-                    last_use[slot] = use;
                 }
                 const unsigned long long dl = globaltimer() + p.watchdog_ns;
                 if (ok) {
-                    // Every CTA's MMAs have released every slot: no commit from the
-                    // partner is still on its way to this CTA's barriers.
-                    for (int sl = 0; sl < kSlots && sl < nitems; ++sl)
-                        wait_until(&slot_empty[sl], last_use[sl] & 1, dl);
+                    // every slot's last tile has been read by its MMAs
+                    for (int sl = 0; sl < kSlots; ++sl)
+                        if (last_use[sl] >= 0) wait_until(&slot_empty[sl], last_use[sl] & 1, dl);
                 } else {
-                    // Let copies already in flight land before the CTA's memory goes away.
+                    // let copies already in flight land before the CTA's memory goes away
                     for (int sl = 0; sl < kSlots; ++sl)
                         if (last_use[sl] >= 0) wait_until(&slot_full[sl], last_use[sl] & 1, dl);
-                    if (C > 1) {  // and those the partner may have sent
-                        const unsigned long long t_end = globaltimer() + 20000;
-                        while (globaltimer() < t_end) __nanosleep(1000);
-                    }
                 }
             }
             __syncwarp();
@@ -505,48 +483,52 @@ __global__ void __launch_bounds__(kThreads, 1)
             // staging lane L, then the 8 lanes that share L % 4 reduce-scatter
             // 32 values, leaving lane L with columns 64 wg + 16 jj + 8 h + 2 (L % 4) + e
             // (wg = m / 4, jj = m % 4, m = L / 4; h, e in {0, 1}).
-            float* part = p.partials ? p.partials + ((static_cast<size_t>(u) * p.Hkv + hkv) * p.MT + mt) * p.P
-                                     : nullptr;
             bool ok = true;
-            for (int j = 0; j < nt && ok && part != nullptr; ++j) {
-                ok = __all_sync(0xffffffffu, wait_until(stage_full, j & 1, deadline));
-                if (!ok) {
-                    if (lane == 0) fail(13);
-                    break;
-                }
-                float x[32];  // index (wg * 4 + jj) * 4 + i
-#pragma unroll
-                for (int w2 = 0; w2 < 2; ++w2)
-#pragma unroll
-                    for (int jj = 0; jj < 4; ++jj) {
-                        float4 a = stage[((w2 * 4 + 0) * 4 + jj) * 32 + lane];
-#pragma unroll
-                        for (int q = 1; q < 4; ++q) {
-                            const float4 b4 = stage[((w2 * 4 + q) * 4 + jj) * 32 + lane];
-                            a.x += b4.x;
-                            a.y += b4.y;
-                            a.z += b4.z;
-                            a.w += b4.w;
-                        }
-                        const int o = (w2 * 4 + jj) * 4;
-                        x[o] = a.x;
-                        x[o + 1] = a.y;
-                        x[o + 2] = a.z;
-                        x[o + 3] = a.w;
+            int tb = 0;
+            for (int w = w0; ok && w < W && p.partials != nullptr; w += wstep) {
+                const WorkUnit x = work_unit(p, w);
+                const unsigned long long deadline = globaltimer() + p.watchdog_ns;
+                float* part = p.partials + ((static_cast<size_t>(x.u) * p.Hkv + x.hkv) * p.MT + x.mt) * p.P;
+                for (int j = 0; j < x.nt; ++j) {
+                    const int g = tb + j;
+                    ok = __all_sync(0xffffffffu, wait_until(stage_full, g & 1, deadline));
+                    if (!ok) {
+                        if (lane == 0) fail(13);
+                        break;
                     }
-                mbar_arrive(stage_free);  // the softmax threads may stage the next tile
-                float sum4[4];
-                lane8_reduce_scatter(x, lane, sum4);
-                if (tile_valid) {
+                    float xs[32];  // index (wg * 4 + jj) * 4 + i
+#pragma unroll
+                    for (int w2 = 0; w2 < 2; ++w2)
+#pragma unroll
+                        for (int jj = 0; jj < 4; ++jj) {
+                            float4 a = stage[((w2 * 4 + 0) * 4 + jj) * 32 + lane];
+#pragma unroll
+                            for (int q = 1; q < 4; ++q) {
+                                const float4 b4 = stage[((w2 * 4 + q) * 4 + jj) * 32 + lane];
+                                a.x += b4.x;
+                                a.y += b4.y;
+                                a.z += b4.z;
+                                a.w += b4.w;
+                            }
+                            const int o = (w2 * 4 + jj) * 4;
+                            xs[o] = a.x;
+                            xs[o + 1] = a.y;
+                            xs[o + 2] = a.z;
+                            xs[o + 3] = a.w;
+                        }
+                    mbar_arrive(stage_free);  // the softmax threads may stage the next tile
+                    float sum4[4];
+                    lane8_reduce_scatter(xs, lane, sum4);
                     const int m4 = lane >> 2, cbase = 64 * (m4 >> 2) + 16 * (m4 & 3) + 2 * (lane & 3);
-                    const bool is_state = j < nst;
-                    const int kb = (is_state ? state_tile(j) : j - nst) * kBN;
+                    const bool is_state = j < x.nst;
+                    const int kb = (is_state ? state_tile(x, j) : j - x.nst) * kBN;
 #pragma unroll
                     for (int i = 0; i < 4; ++i) {
                         const int key = kb + cbase + 8 * (i >> 1) + (i & 1);
-                        if (is_state ? key < count : key < T) part[is_state ? key : B + key] = sum4[i];
+                        if (is_state ? key < x.count : key < T) part[is_state ? key : B + key] = sum4[i];
                     }
                 }
+                tb += x.nt;
             }
         } else if (warp == 1 || warp == 3) {
             // ------------------------------------------------------------ MMA issuers
@@ -562,97 +544,92 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const uint32_t tS0 = tbase + kColS0, tS1 = tbase + kColS1;
                 constexpr uint32_t kIdQK = idesc_bf16_f32(kBM, kBN, false, false);
                 constexpr uint32_t kIdPV = idesc_bf16_f32(kBM, D, false, true);
-                constexpr uint16_t kAll = static_cast<uint16_t>((1u << C) - 1);
-                // the slot's barrier in every CTA of the cluster: this CTA's MMAs are
-                // done with the tile
-                auto release = [&](int slot) {
-                    if (C == 1)
-                        umma_commit(&slot_empty[slot]);
-                    else
-                        umma_commit_mc(&slot_empty[slot], kAll);
-                };
                 int site = 4;  // first wait that expired, for the status word
-                bool ok = wait_until(q_full, 0, deadline);
-                // S(it & 1) = Q K^T for sequence index it (pass A: it < nt; pass B: nt + j)
-                // pass A: S(it % 3) = Q K^T of tile it; pass B (it = nt + j): S(j')
-                // with j' = (nt + j) & 1
-                auto issue_qk = [&](int it) -> bool {
-                    const bool pass_b = it >= nt;
-                    const int item = qk_item(nt, it);
+                bool ok = true;
+                int tb = 0, k = 0;
+                unsigned long long deadline = 0;
+                // S = Q K^T of one tile into buffer tS; its slot is released by the commit
+                auto qk = [&](int item, uint32_t tS, uint64_t* done) {
                     const int slot = item % kSlots;
-                    site = 5;
-                    if (!wait_until(&slot_full[slot], (item / kSlots) & 1, deadline)) return false;
-                    site = 6;
-                    uint32_t tS;
-                    uint64_t* done;
-                    if (!pass_b) {
-                        // the buffer's previous tile (it - 3) has been read by its warpgroup
-                        const int b = it % kSA;
-                        if (it >= kSA) {
-                            const int prev = it - kSA;
-                            if (!wait_until(&sa_read[prev % kSA2], (prev / kSA2) & 1, deadline)) return false;
-                        }
-                        tS = b == 0 ? tS0 : b == 1 ? tS1 : tO;
-                        done = &sa_full[it % kSA2];
-                    } else {
-                        // the buffer's previous pass-B tile (j - 2) is consumed: read by
-                        // both warpgroups (S0: its P went to the P buffer), or read by
-                        // its P V (S1: its P overwrote the scores)
-                        const int j = it - nt, b = j & 1;
-                        if (j >= 2 && !(b == 0 ? wait_until(&sb_read[0], ((j - 2) >> 1) & 1, deadline)
-                                               : wait_until(&pv_done[1], ((j - 2) >> 1) & 1, deadline)))
-                            return false;
-                        tS = b ? tS1 : tS0;
-                        done = &sb_full[b];
-                    }
                     tc_fence_after();
                     mma_group<D / 16, true>(tS, tQ, dk_lo + slot * kSlotStep, d_hi, kIdQK, false);
                     umma_commit(done);
-                    release(slot);
-                    return true;
+                    umma_commit(&slot_empty[slot]);
                 };
-                // O += P(j) V(j): P of even tiles in the P buffer (keys 0..63 then
-                // 64..127), of odd tiles over S1 (keys 0..63 at its columns 0..31,
-                // keys 64..127 at 64..95: each warpgroup over its own scores)
-                auto issue_pv = [&](int j) -> bool {
-                    const int b = j & 1;
-                    const int item = nt + 2 * j + 1;
-                    const int slot = item % kSlots;
-                    // the V tile usually landed long ago: its wait goes first, so the
-                    // wait that P ends is the last before the MMAs
-                    site = 8;
-                    if (!wait_until(&slot_full[slot], (item / kSlots) & 1, deadline)) return false;
-                    site = 7;
-                    if (!wait_until(&p_full[b], (j >> 1) & 1, deadline)) return false;
-                    tc_fence_after();
-                    if (b == 0)
-                        mma_group<kBN / 16, false>(tO, tbase + kColP, dv_lo + slot * kSlotStep, d_hi,
-                                                   kIdPV, j > 0);
-                    else
-                        mma_group<kBN / 16, false, 32>(tO, tS1, dv_lo + slot * kSlotStep, d_hi, kIdPV,
-                                                       j > 0);
-                    umma_commit(&pv_done[b]);
-                    release(slot);
-                    return true;
-                };
-                // pass A: X takes even tiles, Y odd tiles
-                for (int it = isx ? 0 : 1; ok && it < nt; it += 2) ok = issue_qk(it);
-                if (ok) umma_commit(a_done);
-                if (isx) {  // pass B Q K^T, in tile order
-                    // A slot's previous occupant may be one of Y's pass-A tiles, possibly
-                    // still in flight; waiting on the slot before that load lands could
-                    // match an earlier phase of the same parity.  Once every pass-A MMA
-                    // has completed, every pass-A load has landed.
-                    // The first pass-B tiles reuse S0 and S1: both warpgroups must have
-                    // read every pass-A tile.
-                    if (ok) {
-                        site = 9;
-                        ok = wait_until(a_done, 0, deadline) && wait_until(a_read, 0, deadline);
+                for (int w = w0; ok && w < W; w += wstep, ++k) {
+                    const WorkUnit x = work_unit(p, w);
+                    deadline = globaltimer() + p.watchdog_ns;
+                    const int nb = 3 * tb;  // the unit's first ring item
+                    site = 4;
+                    ok = wait_until(q_full, k & 1, deadline);
+                    // pass A: X takes the even global tiles, Y the odd ones; buffer
+                    // g % 3 (S0, S1, or O's columns, free once the previous unit's O
+                    // has been read out)
+                    for (int it = (isx ? 0 : 1) ^ (tb & 1); ok && it < x.nt; it += 2) {
+                        const int g = tb + it, item = nb + it;
+                        site = 5;
+                        if (!(ok = wait_until(&slot_full[item % kSlots], (item / kSlots) & 1, deadline)))
+                            break;
+                        site = 6;
+                        const int b = g % kSA;
+                        if (g >= kSA && !(ok = wait_until(&sa_read[(g - kSA) % kSA2],
+                                                          ((g - kSA) / kSA2) & 1, deadline)))
+                            break;
+                        if (b == 2 && it < kSA && k >= 1 &&
+                            !(ok = wait_until(o_read, (k - 1) & 1, deadline)))
+                            break;
+                        qk(item, b == 0 ? tS0 : b == 1 ? tS1 : tO, &sa_full[g % kSA2]);
                     }
-                    for (int j = 0; ok && j < nt; ++j) ok = issue_qk(nt + j);
-                } else {    // pass B P V, in tile order
-                    for (int j = 0; ok && j < nt; ++j) ok = issue_pv(j);
-                    if (ok) umma_commit(o_full);
+                    if (ok) umma_commit(a_done);
+                    if (isx) {
+                        // Pass B Q K^T, in tile order.  Every pass-A MMA has completed
+                        // (so every pass-A load has landed: a slot's earlier occupant
+                        // may have been the other issuer's) and both warpgroups have
+                        // read every pass-A tile (the first tiles reuse S0 and S1).
+                        if (ok) {
+                            site = 9;
+                            ok = wait_until(a_done, k & 1, deadline) && wait_until(a_read, k & 1, deadline);
+                        }
+                        for (int j = 0; ok && j < x.nt; ++j) {
+                            const int g = tb + j, item = nb + x.nt + 2 * j, b = g & 1;
+                            site = 5;
+                            if (!(ok = wait_until(&slot_full[item % kSlots], (item / kSlots) & 1, deadline)))
+                                break;
+                            // the buffer's previous tile (g - 2) is consumed: read by both
+                            // warpgroups (S0: its P went to the P buffer), or read by its
+                            // P V (S1: its P overwrote the scores)
+                            site = 6;
+                            if (g >= 2 && !(ok = b == 0 ? wait_until(&sb_read[0], ((g - 2) >> 1) & 1, deadline)
+                                                        : wait_until(&pv_done[1], ((g - 2) >> 1) & 1, deadline)))
+                                break;
+                            qk(item, b ? tS1 : tS0, &sb_full[b]);
+                        }
+                    } else {
+                        // O += P(j) V(j): P of even global tiles in the P buffer (keys
+                        // 0..63 then 64..127), of odd ones over S1 (keys 0..63 at its
+                        // columns 0..31, keys 64..127 at 64..95)
+                        for (int j = 0; ok && j < x.nt; ++j) {
+                            const int g = tb + j, item = nb + x.nt + 2 * j + 1, b = g & 1;
+                            const int slot = item % kSlots;
+                            // the V tile usually landed long ago: its wait goes first, so
+                            // the wait that P ends is the last before the MMAs
+                            site = 8;
+                            if (!(ok = wait_until(&slot_full[slot], (item / kSlots) & 1, deadline))) break;
+                            site = 7;
+                            if (!(ok = wait_until(&p_full[b], (g >> 1) & 1, deadline))) break;
+                            tc_fence_after();
+                            if (b == 0)
+                                mma_group<kBN / 16, false>(tO, tbase + kColP, dv_lo + slot * kSlotStep,
+                                                           d_hi, kIdPV, j > 0);
+                            else
+                                mma_group<kBN / 16, false, 32>(tO, tS1, dv_lo + slot * kSlotStep, d_hi,
+                                                               kIdPV, j > 0);
+                            umma_commit(&pv_done[b]);
+                            umma_commit(&slot_empty[slot]);
+                        }
+                        if (ok) umma_commit(o_full);
+                    }
+                    tb += x.nt;
                 }
                 if (!ok) fail(site + (isx ? 0 : 16));
                 // Every MMA issued so far must finish before TMEM is released.
@@ -664,7 +641,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_before();
         __syncthreads();
         if (warp == 1) tmem_dealloc(tbase, 512);
-        if (C > 1) cluster_sync_all();  // no CTA leaves while its partner may still write to it
     } else {
         asm volatile("setmaxnreg.inc.sync.aligned.u32 200;" ::: "memory");
         // ------------------------------------------------------------ softmax warpgroups
@@ -673,244 +649,22 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int row = quad * 32 + lane;        // TMEM lane = query row of the tile
         const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
         const float c = p.scale_log2;
-        const int my_r = mt * kBM + row;
-        const bool row_valid = my_r < rows;
-        const int my_tq = row_valid ? my_r / G : T;  // padding rows see every frame key
-
-        {   // Q row -> TMEM columns [0, D/2) (bf16 pairs); warpgroup wg stores
-            // d in [64 wg, 64 wg + 64) when D = 128, warpgroup 0 all of D = 64.
-            if (wg * 64 < D) {
-                uint32_t w32[32];  // the row loaded at kernel entry
-#pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    w32[4 * i] = qreg[i].x;
-                    w32[4 * i + 1] = qreg[i].y;
-                    w32[4 * i + 2] = qreg[i].z;
-                    w32[4 * i + 3] = qreg[i].w;
-                }
-                tmem_st16(tbase + lane_off + wg * 32, *reinterpret_cast<uint32_t(*)[16]>(&w32[0]));
-                tmem_st16(tbase + lane_off + wg * 32 + 16,
-                          *reinterpret_cast<uint32_t(*)[16]>(&w32[16]));
-                tmem_st_wait();
-            }
-            tc_fence_before();
-            mbar_arrive(q_full);
-        }
-
-        bool ok = true;
-        int site = 10;  // first wait that expired, for the status word
-        // ---------------- pass A: online max / sum of exp2 over this warpgroup's tiles
-        float m = -INFINITY, l = 0.f;  // log2 units, scaled
-        for (int it = wg; it < nt; it += 2) {
-            const int b = it % kSA;  // score buffer of this tile
-            ok = __all_sync(0xffffffffu, wait_until(&sa_full[it % kSA2], (it / kSA2) & 1, deadline));
-            if (!ok) break;
-            tc_fence_after();
-            const uint32_t tSa =
-                tbase + lane_off + (b == 0 ? kColS0 : b == 1 ? kColS1 : kColO);
-            int lim;  // keys [0, lim) of this tile are visible to this row
-            if (it < nst) {
-                lim = min(kBN, count - state_tile(it) * kBN);
-            } else {
-                const int f0 = (it - nst) * kBN;
-                lim = min(kBN, (p.causal ? min(T, my_tq + 1) : T) - f0);
-            }
-            // the whole tile into registers, then release the buffer at once so
-            // the next Q K^T into it can start while this one is reduced
-            float v[4][32];
-#pragma unroll
-            for (int ch = 0; ch < 4; ++ch) tmem_ld32(tSa + ch * 32, v[ch]);
-            tmem_ld_wait();
-            tc_fence_before();
-            mbar_arrive(&sa_read[it % kSA2]);
-            // after its last tile is in registers, this thread holds no pass-A
-            // score buffer: pass B's Q K^T may start while the sums finish
-            if (it + 2 >= nt) mbar_arrive(a_read);
-            if (lim < kBN) {
-#pragma unroll
-                for (int ch = 0; ch < 4; ++ch)
-#pragma unroll
-                    for (int e = 0; e < 32; ++e)
-                        v[ch][e] = (ch * 32 + e < lim) ? v[ch][e] : -INFINITY;
-            }
-            float mx[4];
-#pragma unroll
-            for (int q4 = 0; q4 < 4; ++q4) mx[q4] = fmaxf(v[q4][0], v[q4][1]);
-#pragma unroll
-            for (int ch = 0; ch < 4; ++ch)
-#pragma unroll
-                for (int e = 2; e < 32; e += 2)
-                    mx[ch] = max3(mx[ch], v[ch][e], v[ch][e + 1]);
-            const float m_new =
-                fmaxf(m, fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])) * c);  // c > 0
-            if (m_new != -INFINITY) {
-                const f2 cc = pk(c, c), nm = pk(-m_new, -m_new);
-                f2 acc[4] = {pk(0.f, 0.f), pk(0.f, 0.f), pk(0.f, 0.f), pk(0.f, 0.f)};
-#pragma unroll
-                for (int ch = 0; ch < 4; ++ch)
-#pragma unroll
-                    for (int e = 0; e < 32; e += 2) {
-                        float x0, x1;
-                        upk(fma2(pk(v[ch][e], v[ch][e + 1]), cc, nm), x0, x1);
-                        acc[(e >> 1) & 3] = add2(acc[(e >> 1) & 3], pk(ex2(x0), ex2(x1)));
-                    }
-                float s0, s1;
-                upk(add2(add2(acc[0], acc[1]), add2(acc[2], acc[3])), s0, s1);
-                l = l * ex2(m - m_new) + (s0 + s1);
-                m = m_new;
-            }
-        }
-        if (wg >= nt) mbar_arrive(a_read);  // a warpgroup without pass-A tiles
-        if (ok) site = 11;
-        stat[(wg * 2 + 0) * kBM + row] = m;
-        stat[(wg * 2 + 1) * kBM + row] = l;
-        named_bar_sync(1, 256);
-        float nlse;  // -log2-sum-exp of this row (scaled); -inf for padding rows
-        {
-            const float m0 = stat[0 * kBM + row], l0 = stat[1 * kBM + row];
-            const float m1 = stat[2 * kBM + row], l1 = stat[3 * kBM + row];
-            const float mm = fmaxf(m0, m1);
-            const float ll = l0 * ex2(m0 - mm) + l1 * ex2(m1 - mm);
-            nlse = row_valid ? -(mm + __log2f(ll)) : -INFINITY;
-        }
-
-        // ---------------- pass B: P = exp2(S c - lse) -> TMEM (bf16) and column sums
-        // Both warpgroups work on every tile, warpgroup wg on its keys
-        // [64 wg, 64 wg + 64), so a tile's P is ready after half a tile's work.
-        // TMEM is read in 16-lane x 256-bit groups: a thread holds 4 rows
-        // (quadrant rows 16h + t/4 + 8k, h, k in {0, 1}) x 16 columns
-        // (8r + 2(t%4) + e); the column sums add 4 rows in registers and the 8
-        // lanes that share t % 4 by a 3-step reduce-scatter.
-        // P of even tiles goes to the P buffer (so Q K^T can refill S0 once both
-        // warpgroups have read it); P of odd tiles overwrites the first half of
-        // this warpgroup's own S1 columns (Q K^T into S1 waits for that P V).
-        float* nl_row = stat + 4 * kBM;  // -lse of every row of the tile
-        if (wg == 0) nl_row[row] = nlse;
-        named_bar_sync(1, 256);
-        float nl4[4];       // -lse of this thread's 4 rows, index 2h + k
-        int tq4[4];         // token of each row (T for padding rows)
-#pragma unroll
-        for (int h = 0; h < 2; ++h)
-#pragma unroll
-            for (int k = 0; k < 2; ++k) {
-                const int rr = quad * 32 + 16 * h + lane / 4 + 8 * k;
-                nl4[2 * h + k] = nl_row[rr];
-                const int gr = mt * kBM + rr;
-                tq4[2 * h + k] = gr < rows ? gr / G : T;
-            }
-        float* part = p.partials ? p.partials + ((static_cast<size_t>(u) * p.Hkv + hkv) * p.MT + mt) * p.P
-                                 : nullptr;
-        float4* mystage = stage + (wg * 4 + quad) * 4 * 32 + lane;  // chunk jj at + jj * 32
-        const int cq = 2 * (lane & 3);                // this thread's column offset in 8
-        const int c0 = 64 * wg;                       // this warpgroup's first key of a tile
+        const int cq = 2 * (lane & 3);           // this thread's column offset in 8
+        const int c0 = 64 * wg;                  // this warpgroup's first key of a tile
         const uint32_t tSh0 = tbase + lane_off + kColS0 + c0;   // this warpgroup's S0 half
         const uint32_t tSh1 = tbase + lane_off + kColS1 + c0;   // its S1 half (and odd P)
         const uint32_t tPh = tbase + lane_off + kColP + c0 / 2;  // its even-tile P
-        // Every warp runs every iteration and arrives at the per-tile barrier;
-        // after a timeout it only skips the work (a bar.sync cannot time out).
-        for (int j = 0; j < nt; ++j) {
-            const int b = j & 1;
-            if (ok) ok = __all_sync(0xffffffffu, wait_until(&sb_full[b], (j >> 1) & 1, deadline));
-            const bool is_state = j < nst;
-            if (ok) {
-                tc_fence_after();
-                int lim4[4];  // keys [0, lim) of this tile are visible to each row
-                if (is_state) {
-                    const int lim = min(kBN, count - state_tile(j) * kBN);
-#pragma unroll
-                    for (int q4 = 0; q4 < 4; ++q4) lim4[q4] = lim;
-                } else {
-                    const int f0 = (j - nst) * kBN;
-#pragma unroll
-                    for (int q4 = 0; q4 < 4; ++q4)
-                        lim4[q4] = min(kBN, (p.causal ? min(T, tq4[q4] + 1) : T) - f0);
-                }
-                const int lmin = min(min(lim4[0], lim4[1]), min(lim4[2], lim4[3]));
-                const bool full = lmin >= c0 + 64;
-                const f2 cc = pk(c, c);
-                float v[2][32];
-#pragma unroll
-                for (int h = 0; h < 2; ++h) tmem_ld_16x256b_x8((b ? tSh1 : tSh0) + ((16u * h) << 16), v[h]);
-                tmem_ld_wait();
-                if (b == 0) {
-                    tc_fence_before();
-                    mbar_arrive(&sb_read[0]);  // Q K^T of tile j + 2 may overwrite S0
-                }
-#pragma unroll
-                for (int h = 0; h < 2; ++h)
-#pragma unroll
-                    for (int r = 0; r < 8; ++r)
-#pragma unroll
-                        for (int k = 0; k < 2; ++k) {
-                            const int i = 4 * r + 2 * k;
-                            const float nk = nl4[2 * h + k];
-                            float x0, x1;
-                            upk(fma2(pk(v[h][i], v[h][i + 1]), cc, pk(nk, nk)), x0, x1);
-                            v[h][i] = ex2(x0);
-                            v[h][i + 1] = ex2(x1);
-                            if (!full) {
-                                const int col = c0 + 8 * r + cq, lim = lim4[2 * h + k];
-                                v[h][i] = col < lim ? v[h][i] : 0.f;
-                                v[h][i + 1] = col + 1 < lim ? v[h][i + 1] : 0.f;
-                            }
-                        }
-                // the P buffer is free once the P V of tile j - 2 has read it
-                if (b == 0 && j >= 2)
-                    ok = __all_sync(0xffffffffu,
-                                    wait_until(&pv_done[0], ((j - 2) >> 1) & 1, deadline));
-                if (ok) {
-                    tc_fence_after();
-#pragma unroll
-                    for (int h = 0; h < 2; ++h) {
-                        uint32_t pw[16];  // register 2r + k: row k, P column 4r + t%4
-#pragma unroll
-                        for (int r = 0; r < 8; ++r)
-#pragma unroll
-                            for (int k = 0; k < 2; ++k)
-                                pw[2 * r + k] = pack_bf16x2(v[h][4 * r + 2 * k], v[h][4 * r + 2 * k + 1]);
-                        tmem_st_16x128b_x8((b ? tSh1 : tPh) + ((16u * h) << 16), pw);
-                    }
-                    tmem_st_wait();
-                    tc_fence_before();
-                    mbar_arrive(&p_full[b]);
-                    // the column sums run while the tensor core does this tile's P V:
-                    // value 2r + e is column 8r + cq + e summed over the thread's rows;
-                    // the reducer warp adds them across lanes and warps
-                    if (part != nullptr) {
-                        float cs[16];
-#pragma unroll
-                        for (int r = 0; r < 8; ++r) {
-                            const f2 a = add2(pk(v[0][4 * r], v[0][4 * r + 1]), pk(v[0][4 * r + 2], v[0][4 * r + 3]));
-                            const f2 bb = add2(pk(v[1][4 * r], v[1][4 * r + 1]), pk(v[1][4 * r + 2], v[1][4 * r + 3]));
-                            upk(add2(a, bb), cs[2 * r], cs[2 * r + 1]);
-                        }
-                        if (j >= 1)  // the reducer has read the previous tile's values
-                            ok = __all_sync(0xffffffffu, wait_until(stage_free, (j - 1) & 1, deadline));
-                        if (ok) {
-#pragma unroll
-                            for (int jj = 0; jj < 4; ++jj)
-                                mystage[jj * 32] = make_float4(cs[4 * jj], cs[4 * jj + 1], cs[4 * jj + 2],
-                                                               cs[4 * jj + 3]);
-                            mbar_arrive(stage_full);
-                        }
-                    }
-                }
-            }
-        }
-        if (ok) site = 12;
-        // Frame keys no row of this tile can see receive zero importance here.
-        if (tile_valid && part != nullptr)
-            for (int t = nft * kBN + (threadIdx.x - 128); t < T; t += 256) part[B + t] = 0.f;
+        float4* mystage = stage + (wg * 4 + quad) * 4 * 32 + lane;  // chunk jj at + jj * 32
+        float* nl_row = stat + 4 * kBM;  // -lse of every row of the tile
+        const f2 cc = pk(c, c);
 
-        // ---------------- epilogue: O rows -> bf16 out; warpgroup wg stores
-        // columns [wg*D/2, (wg+1)*D/2)
-        if (ok) ok = __all_sync(0xffffffffu, wait_until(o_full, 0, deadline));
-        if (ok) {
-            tc_fence_after();
+        // O rows of unit x -> bf16 out; warpgroup wg stores columns [wg D/2, (wg+1) D/2)
+        auto store_o = [&](const WorkUnit& x) {
+            const int my_r = x.mt * kBM + row;
             __nv_bfloat16* dst = p.out;
-            if (row_valid) {
+            if (my_r < rows) {
                 const int t = my_r / G, g = my_r - t * G;
-                dst += ((static_cast<size_t>(u) * T + t) * p.Hq + hkv * G + g) * D;
+                dst += ((static_cast<size_t>(x.u) * T + t) * p.Hq + x.hkv * G + g) * D;
             }
 #pragma unroll
             for (int cc2 = 0; cc2 < D / 64; ++cc2) {
@@ -918,23 +672,258 @@ __global__ void __launch_bounds__(kThreads, 1)
                 float o[32];
                 tmem_ld32(tbase + lane_off + kColO + col, o);
                 tmem_ld_wait();
-                if (row_valid) {
+                if (my_r < rows) {
 #pragma unroll
                     for (int e = 0; e < 4; ++e) {
-                        const uint4 w = make_uint4(
-                            pack_bf16x2(o[e * 8 + 0], o[e * 8 + 1]),
-                            pack_bf16x2(o[e * 8 + 2], o[e * 8 + 3]),
-                            pack_bf16x2(o[e * 8 + 4], o[e * 8 + 5]),
-                            pack_bf16x2(o[e * 8 + 6], o[e * 8 + 7]));
-                        *reinterpret_cast<uint4*>(dst + col + e * 8) = w;
+                        const uint4 v4 = make_uint4(
+                            pack_bf16x2(o[e * 8 + 0], o[e * 8 + 1]), pack_bf16x2(o[e * 8 + 2], o[e * 8 + 3]),
+                            pack_bf16x2(o[e * 8 + 4], o[e * 8 + 5]), pack_bf16x2(o[e * 8 + 6], o[e * 8 + 7]));
+                        *reinterpret_cast<uint4*>(dst + col + e * 8) = v4;
                     }
                 }
             }
+        };
+
+        bool ok = true;
+        int site = 10;  // first wait that expired, for the status word
+        int tb = 0, k = 0;
+        WorkUnit prev{};
+        for (int w = w0; ok && w < W; w += wstep, ++k) {
+            const WorkUnit x = work_unit(p, w);
+            const unsigned long long deadline = globaltimer() + p.watchdog_ns;
+            const int my_r = x.mt * kBM + row;
+            const bool row_valid = my_r < rows;
+            const int my_tq = row_valid ? my_r / G : T;  // padding rows see every frame key
+
+            {   // Q row -> TMEM columns [0, D/2) (bf16 pairs); warpgroup wg stores
+                // d in [64 wg, 64 wg + 64) when D = 128, warpgroup 0 all of D = 64.
+                // Every Q K^T of the previous unit has completed (its P V have).
+                if (wg * 64 < D) {
+                    uint32_t w32[32];
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) {
+                        w32[4 * i] = qreg[i].x;
+                        w32[4 * i + 1] = qreg[i].y;
+                        w32[4 * i + 2] = qreg[i].z;
+                        w32[4 * i + 3] = qreg[i].w;
+                    }
+                    tmem_st16(tbase + lane_off + wg * 32, *reinterpret_cast<uint32_t(*)[16]>(&w32[0]));
+                    tmem_st16(tbase + lane_off + wg * 32 + 16,
+                              *reinterpret_cast<uint32_t(*)[16]>(&w32[16]));
+                    tmem_st_wait();
+                }
+                tc_fence_before();
+                mbar_arrive(q_full);
+            }
+            if (k >= 1) {  // the previous unit's O, while this unit's first Q K^T run
+                store_o(prev);
+                tc_fence_before();
+                mbar_arrive(o_read);
+            }
+
+            // ---------------- pass A: online max / sum of exp2 over this warpgroup's tiles
+            float m = -INFINITY, l = 0.f;  // log2 units, scaled
+            const int it0 = wg ^ (tb & 1);  // this warpgroup takes the global tiles of parity wg
+            for (int it = it0; it < x.nt; it += 2) {
+                const int g = tb + it;
+                const int b = g % kSA;  // score buffer of this tile
+                ok = __all_sync(0xffffffffu, wait_until(&sa_full[g % kSA2], (g / kSA2) & 1, deadline));
+                if (!ok) break;
+                tc_fence_after();
+                const uint32_t tSa = tbase + lane_off + (b == 0 ? kColS0 : b == 1 ? kColS1 : kColO);
+                int lim;  // keys [0, lim) of this tile are visible to this row
+                if (it < x.nst) {
+                    lim = min(kBN, x.count - state_tile(x, it) * kBN);
+                } else {
+                    const int f0 = (it - x.nst) * kBN;
+                    lim = min(kBN, (p.causal ? min(T, my_tq + 1) : T) - f0);
+                }
+                // the whole tile into registers, then release the buffer at once so
+                // the next Q K^T into it can start while this one is reduced
+                float v[4][32];
+#pragma unroll
+                for (int ch = 0; ch < 4; ++ch) tmem_ld32(tSa + ch * 32, v[ch]);
+                tmem_ld_wait();
+                tc_fence_before();
+                mbar_arrive(&sa_read[g % kSA2]);
+                // after its last tile is in registers, this thread holds no pass-A
+                // score buffer: pass B's Q K^T may start while the sums finish
+                if (it + 2 >= x.nt) mbar_arrive(a_read);
+                if (lim < kBN) {
+#pragma unroll
+                    for (int ch = 0; ch < 4; ++ch)
+#pragma unroll
+                        for (int e = 0; e < 32; ++e)
+                            v[ch][e] = (ch * 32 + e < lim) ? v[ch][e] : -INFINITY;
+                }
+                float mx[4];
+#pragma unroll
+                for (int q4 = 0; q4 < 4; ++q4) mx[q4] = fmaxf(v[q4][0], v[q4][1]);
+#pragma unroll
+                for (int ch = 0; ch < 4; ++ch)
+#pragma unroll
+                    for (int e = 2; e < 32; e += 2)
+                        mx[ch] = max3(mx[ch], v[ch][e], v[ch][e + 1]);
+                const float m_new =
+                    fmaxf(m, fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])) * c);  // c > 0
+                if (m_new != -INFINITY) {
+                    const f2 nm = pk(-m_new, -m_new);
+                    f2 acc[4] = {pk(0.f, 0.f), pk(0.f, 0.f), pk(0.f, 0.f), pk(0.f, 0.f)};
+#pragma unroll
+                    for (int ch = 0; ch < 4; ++ch)
+#pragma unroll
+                        for (int e = 0; e < 32; e += 2) {
+                            float x0, x1;
+                            upk(fma2(pk(v[ch][e], v[ch][e + 1]), cc, nm), x0, x1);
+                            acc[(e >> 1) & 3] = add2(acc[(e >> 1) & 3], pk(ex2(x0), ex2(x1)));
+                        }
+                    float s0, s1;
+                    upk(add2(add2(acc[0], acc[1]), add2(acc[2], acc[3])), s0, s1);
+                    l = l * ex2(m - m_new) + (s0 + s1);
+                    m = m_new;
+                }
+            }
+            if (it0 >= x.nt) mbar_arrive(a_read);  // a warpgroup without pass-A tiles
+            if (!ok) break;
+            site = 11;
+            stat[(wg * 2 + 0) * kBM + row] = m;
+            stat[(wg * 2 + 1) * kBM + row] = l;
+            named_bar_sync(1, 256);
+            float nlse;  // -log2-sum-exp of this row (scaled); -inf for padding rows
+            {
+                const float m0 = stat[0 * kBM + row], l0 = stat[1 * kBM + row];
+                const float m1 = stat[2 * kBM + row], l1 = stat[3 * kBM + row];
+                const float mm = fmaxf(m0, m1);
+                const float ll = l0 * ex2(m0 - mm) + l1 * ex2(m1 - mm);
+                nlse = row_valid ? -(mm + __log2f(ll)) : -INFINITY;
+            }
+            if (wg == 0) nl_row[row] = nlse;
+            named_bar_sync(1, 256);
+            float nl4[4];  // -lse of this thread's 4 rows, index 2h + k
+            int tq4[4];    // token of each row (T for padding rows)
+#pragma unroll
+            for (int h = 0; h < 2; ++h)
+#pragma unroll
+                for (int k2 = 0; k2 < 2; ++k2) {
+                    const int rr = quad * 32 + 16 * h + lane / 4 + 8 * k2;
+                    nl4[2 * h + k2] = nl_row[rr];
+                    const int gr = x.mt * kBM + rr;
+                    tq4[2 * h + k2] = gr < rows ? gr / G : T;
+                }
+            // the next unit's Q rows load during pass B
+            load_q(w + wstep);
+
+            // ---------------- pass B: P = exp2(S c - lse) -> TMEM (bf16) and column sums
+            // Both warpgroups work on every tile, warpgroup wg on its keys
+            // [64 wg, 64 wg + 64), so a tile's P is ready after half a tile's work.
+            // TMEM is read in 16-lane x 256-bit groups: a thread holds 4 rows
+            // (quadrant rows 16h + t/4 + 8k, h, k in {0, 1}) x 16 columns
+            // (8r + 2(t%4) + e).  P of even global tiles goes to the P buffer (so
+            // Q K^T can refill S0 once both warpgroups have read it); P of odd
+            // tiles overwrites the first half of this warpgroup's own S1 columns
+            // (Q K^T into S1 waits for that P V).
+            float* part = p.partials ? p.partials + ((static_cast<size_t>(x.u) * p.Hkv + x.hkv) * p.MT + x.mt) * p.P
+                                     : nullptr;
+            site = 12;
+            for (int j = 0; ok && j < x.nt; ++j) {
+                const int g = tb + j, b = g & 1;
+                ok = __all_sync(0xffffffffu, wait_until(&sb_full[b], (g >> 1) & 1, deadline));
+                if (!ok) break;
+                tc_fence_after();
+                int lim4[4];  // keys [0, lim) of this tile are visible to each row
+                if (j < x.nst) {
+                    const int lim = min(kBN, x.count - state_tile(x, j) * kBN);
+#pragma unroll
+                    for (int q4 = 0; q4 < 4; ++q4) lim4[q4] = lim;
+                } else {
+                    const int f0 = (j - x.nst) * kBN;
+#pragma unroll
+                    for (int q4 = 0; q4 < 4; ++q4)
+                        lim4[q4] = min(kBN, (p.causal ? min(T, tq4[q4] + 1) : T) - f0);
+                }
+                const int lmin = min(min(lim4[0], lim4[1]), min(lim4[2], lim4[3]));
+                const bool full = lmin >= c0 + 64;
+                float v[2][32];
+#pragma unroll
+                for (int h = 0; h < 2; ++h) tmem_ld_16x256b_x8((b ? tSh1 : tSh0) + ((16u * h) << 16), v[h]);
+                tmem_ld_wait();
+                if (b == 0) {
+                    tc_fence_before();
+                    mbar_arrive(&sb_read[0]);  // Q K^T of tile g + 2 may overwrite S0
+                }
+#pragma unroll
+                for (int h = 0; h < 2; ++h)
+#pragma unroll
+                    for (int r = 0; r < 8; ++r)
+#pragma unroll
+                        for (int k2 = 0; k2 < 2; ++k2) {
+                            const int i = 4 * r + 2 * k2;
+                            const float nk = nl4[2 * h + k2];
+                            float x0, x1;
+                            upk(fma2(pk(v[h][i], v[h][i + 1]), cc, pk(nk, nk)), x0, x1);
+                            v[h][i] = ex2(x0);
+                            v[h][i + 1] = ex2(x1);
+                            if (!full) {
+                                const int col = c0 + 8 * r + cq, lim = lim4[2 * h + k2];
+                                v[h][i] = col < lim ? v[h][i] : 0.f;
+                                v[h][i + 1] = col + 1 < lim ? v[h][i + 1] : 0.f;
+                            }
+                        }
+                // the P buffer is free once the P V of tile g - 2 has read it
+                if (b == 0 && g >= 2)
+                    ok = __all_sync(0xffffffffu, wait_until(&pv_done[0], ((g - 2) >> 1) & 1, deadline));
+                if (!ok) break;
+                tc_fence_after();
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    uint32_t pw[16];  // register 2r + k: row k, P column 4r + t%4
+#pragma unroll
+                    for (int r = 0; r < 8; ++r)
+#pragma unroll
+                        for (int k2 = 0; k2 < 2; ++k2)
+                            pw[2 * r + k2] = pack_bf16x2(v[h][4 * r + 2 * k2], v[h][4 * r + 2 * k2 + 1]);
+                    tmem_st_16x128b_x8((b ? tSh1 : tPh) + ((16u * h) << 16), pw);
+                }
+                tmem_st_wait();
+                tc_fence_before();
+                mbar_arrive(&p_full[b]);
+                // the column sums run while the tensor core does this tile's P V:
+                // value 2r + e is column 8r + cq + e summed over the thread's rows;
+                // the reducer warp adds them across lanes and warps
+                if (part != nullptr) {
+                    float cs[16];
+#pragma unroll
+                    for (int r = 0; r < 8; ++r) {
+                        const f2 a = add2(pk(v[0][4 * r], v[0][4 * r + 1]), pk(v[0][4 * r + 2], v[0][4 * r + 3]));
+                        const f2 bb = add2(pk(v[1][4 * r], v[1][4 * r + 1]), pk(v[1][4 * r + 2], v[1][4 * r + 3]));
+                        upk(add2(a, bb), cs[2 * r], cs[2 * r + 1]);
+                    }
+                    if (g >= 1)  // the reducer has read the previous tile's values
+                        ok = __all_sync(0xffffffffu, wait_until(stage_free, (g - 1) & 1, deadline));
+                    if (!ok) break;
+#pragma unroll
+                    for (int jj = 0; jj < 4; ++jj)
+                        mystage[jj * 32] = make_float4(cs[4 * jj], cs[4 * jj + 1], cs[4 * jj + 2], cs[4 * jj + 3]);
+                    mbar_arrive(stage_full);
+                }
+            }
+            if (!ok) break;
+            // Frame keys no row of this tile can see receive zero importance here.
+            if (part != nullptr)
+                for (int t = x.nft * kBN + (threadIdx.x - 128); t < T; t += 256) part[B + t] = 0.f;
+            // every P V of the unit has completed: O is final, and TMEM's Q and
+            // score columns are free for the next unit
+            site = 14;
+            ok = __all_sync(0xffffffffu, wait_until(o_full, k & 1, deadline));
+            if (!ok) break;
+            tc_fence_after();
+            prev = x;
+            tb += x.nt;
         }
+        if (ok && k >= 1) store_o(prev);  // the last unit's O
         if (!ok) fail(site + 32 * wg);
         tc_fence_before();
         __syncthreads();
-        if (C > 1) cluster_sync_all();
     }
 }
 
@@ -944,41 +933,39 @@ __global__ void __launch_bounds__(kThreads, 1)
 constexpr int kLaunchRegs = 168;
 static_assert(128 * 96 + 256 * 200 <= kThreads * kLaunchRegs, "register split");
 
-// Query tiles per cluster for head dim D: two CTAs share each K/V tile by
-// multicast (one 64-column half each) when D = 128.
-constexpr int cluster_size(int D) { return D == 128 ? 1 : 1; }
+int g_num_sms = 0;  // SMs of the device, read once by attn_prepare
 
 template <int D>
 cudaError_t prepare_one()
 {
-    constexpr int C = cluster_size(D);
     cudaFuncAttributes fa;
-    cudaError_t e = cudaFuncGetAttributes(&fa, frame_attn_lse_importance<D, C>);
+    cudaError_t e = cudaFuncGetAttributes(&fa, frame_attn_lse_importance<D>);
     if (e != cudaSuccess) return e;
     if (fa.numRegs < kLaunchRegs) return cudaErrorInvalidConfiguration;
-    return cudaFuncSetAttribute(frame_attn_lse_importance<D, C>,
+    int dev = 0;
+    if ((e = cudaGetDevice(&dev)) != cudaSuccess ||
+        (e = cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
+        return e;
+    return cudaFuncSetAttribute(frame_attn_lse_importance<D>,
                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 AttnLayout<D>::kAlloc);
 }
 
+// One CTA per SM (at most one per work unit); each walks its units in order.
 template <int D>
 cudaError_t launch_one(const CUtensorMap& tm_sk, const CUtensorMap& tm_sv, const CUtensorMap& tm_fk,
-                       const CUtensorMap& tm_fv, const AttnParams& p, int U, cudaStream_t st)
+                       const CUtensorMap& tm_fv, const AttnParams& p0, int U, cudaStream_t st)
 {
-    constexpr int C = cluster_size(D);
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((p.MT + C - 1) / C * C, p.Hkv, U);
-    cfg.blockDim = dim3(kThreads, 1, 1);
-    cfg.dynamicSmemBytes = AttnLayout<D>::kAlloc;
-    cfg.stream = st;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = C;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, frame_attn_lse_importance<D, C>, tm_sk, tm_sv, tm_fk, tm_fv, p);
+    AttnParams p = p0;
+    p.U = U;
+    const long long W = static_cast<long long>(p.MT) * p.Hkv * U;
+    if (W <= 0) return cudaSuccess;
+    if (W > 0x7FFFFFFFll) return cudaErrorInvalidValue;
+    const int sms = g_num_sms > 0 ? g_num_sms : 1;
+    const int grid = static_cast<int>(W < sms ? W : sms);
+    frame_attn_lse_importance<D><<<grid, kThreads, AttnLayout<D>::kAlloc, st>>>(tm_sk, tm_sv, tm_fk,
+                                                                              tm_fv, p);
+    return cudaSuccess;
 }
 
 }  // namespace

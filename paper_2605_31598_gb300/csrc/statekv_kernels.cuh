@@ -17,11 +17,12 @@ namespace statekv {
 
 // Device error codes written to the status word (0 = no error).  The low
 // byte is the kind; an attention-kernel timeout carries the waiting site in
-// bits 8..15 (the first expired wait of the CTA): 1 V producer (pass A
-// done), 2/3 K/V producer (free slot), 4..9 the MMA issuer's waiter (4 Q
-// ready, 5 K tile landed, 6 score buffer read in pass A, 7 P written, 8 V
-// tile landed, 9 score buffer's P V done in pass B), 10..12 softmax
-// warpgroup 0 (pass A, pass B, O ready; +32 for warpgroup 1).
+// bits 8..15 (the first expired wait of the CTA): 2 producer (free slot),
+// 4..9 MMA issuer X (4 Q ready, 5 K tile landed, 6 score buffer free, 7 P
+// written, 8 V tile landed, 9 pass A done and read; +16 for issuer Y),
+// 10..12 and 14 softmax warpgroup 0 (10 Q K^T in pass A, 11 pass-B scores
+// ready, 12 the P buffer or the staging area free, 14 O final; +32 for
+// warpgroup 1), 13 the column-sum reducer.
 enum DeviceError : int32_t {
     DEV_OK = 0,
     DEV_TIMEOUT_ATTN = 1,
@@ -50,6 +51,7 @@ struct AttnParams {
     int32_t* status;          // device-visible status word
     UnitRange units;
     int T, Hq, Hkv, G, B, P, MT;
+    int U;                    // units of the call (set by launch_attn)
     int causal;
     int count_mul;            // 1: counts are state sizes; T: counts are frame counters
     float scale_log2;         // softmax scale * log2(e)
