@@ -56,6 +56,24 @@ __device__ __forceinline__ int block_exclusive_scan(int x, int* warp_sums, int& 
     return total;
 }
 
+// Sum of x[mt * stride] over mt < MT in order (the same rounding as a plain
+// loop), with eight loads in flight per step: the partials come from L2, and
+// a load-add chain would wait for each of them in turn.
+__device__ __forceinline__ float tile_sum(const float* x, int MT, int stride)
+{
+    float s = 0.f;
+    int mt = 0;
+    for (; mt + 8 <= MT; mt += 8) {
+        float v[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) v[e] = __ldg(x + static_cast<size_t>(mt + e) * stride);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) s += v[e];
+    }
+    for (; mt < MT; ++mt) s += __ldg(x + static_cast<size_t>(mt) * stride);
+    return s;
+}
+
 __global__ void __launch_bounds__(kSelThreads)
     state_select_gather(const SelectParams p)
 {
@@ -86,17 +104,12 @@ __global__ void __launch_bounds__(kSelThreads)
     const float* part0 = p.partials + static_cast<size_t>(u) * p.Hkv * p.MT * P;
     for (int i = tid; i < n; i += kSelThreads) {
         const int col = i < count ? i : B + (i - count);
-        float s = 0.f;
-        for (int mt = 0; mt < p.MT; ++mt) s += part[static_cast<size_t>(mt) * P + col];
+        const float s = tile_sum(part + col, p.MT, P);
         float r = s;  // ranking score
         if (p.shared) {
             r = 0.f;
-            for (int h2 = 0; h2 < p.Hkv; ++h2) {
-                float sh = 0.f;
-                for (int mt = 0; mt < p.MT; ++mt)
-                    sh += part0[(static_cast<size_t>(h2) * p.MT + mt) * P + col];
-                r += sh;
-            }
+            for (int h2 = 0; h2 < p.Hkv; ++h2)
+                r += tile_sum(part0 + static_cast<size_t>(h2) * p.MT * P + col, p.MT, P);
         }
         const int ps = i < count ? pos[i] : L + (i - count);
         key[i] = (static_cast<uint64_t>(__float_as_uint(r)) << 32) |
