@@ -56,22 +56,30 @@ __device__ __forceinline__ int block_exclusive_scan(int x, int* warp_sums, int& 
     return total;
 }
 
-// Sum of x[mt * stride] over mt < MT in order (the same rounding as a plain
-// loop), with eight loads in flight per step: the partials come from L2, and
-// a load-add chain would wait for each of them in turn.
-__device__ __forceinline__ float tile_sum(const float* x, int MT, int stride)
+// For each of 8 pool members (columns col[e], active act[e]): the sum of
+// x[mt * stride + col] over mt < MT, added in mt order.  Four tiles' loads of
+// all 8 members (32 independent loads) are in flight before any addition.
+__device__ __forceinline__ void tiles_sum(const float* x, int MT, int stride, const int (&col)[8],
+                                          const bool (&act)[8], float (&s)[8])
 {
-    float s = 0.f;
-    int mt = 0;
-    for (; mt + 8 <= MT; mt += 8) {
-        float v[8];
 #pragma unroll
-        for (int e = 0; e < 8; ++e) v[e] = __ldg(x + static_cast<size_t>(mt + e) * stride);
+    for (int e = 0; e < 8; ++e) s[e] = 0.f;
+#pragma unroll 1
+    for (int mt = 0; mt < MT; mt += 4) {
+        float v[4][8];
 #pragma unroll
-        for (int e = 0; e < 8; ++e) s += v[e];
+        for (int m4 = 0; m4 < 4; ++m4)
+#pragma unroll
+            for (int e = 0; e < 8; ++e)
+                v[m4][e] = (act[e] && mt + m4 < MT)
+                               ? __ldg(x + static_cast<size_t>(mt + m4) * stride + col[e])
+                               : 0.f;
+#pragma unroll
+        for (int m4 = 0; m4 < 4; ++m4)
+#pragma unroll
+            for (int e = 0; e < 8; ++e)
+                if (mt + m4 < MT) s[e] += v[m4][e];
     }
-    for (; mt < MT; ++mt) s += __ldg(x + static_cast<size_t>(mt) * stride);
-    return s;
 }
 
 __global__ void __launch_bounds__(kSelThreads)
@@ -100,21 +108,41 @@ __global__ void __launch_bounds__(kSelThreads)
         p.importance ? p.importance + (static_cast<size_t>(u) * p.Hkv + hkv) * P : nullptr;
     const int n = count + T;
 
-    // 1. importance (fixed-order sum over query tiles) and selection keys
+    // 1. importance (fixed-order sum over query tiles) and selection keys.  A
+    // thread takes up to 8 pool members at once and walks the query tiles
+    // outside them, so all its loads are independent (the partials come from
+    // L2); each member's sum still adds the tiles in order.
     const float* part0 = p.partials + static_cast<size_t>(u) * p.Hkv * p.MT * P;
-    for (int i = tid; i < n; i += kSelThreads) {
-        const int col = i < count ? i : B + (i - count);
-        const float s = tile_sum(part + col, p.MT, P);
-        float r = s;  // ranking score
-        if (p.shared) {
-            r = 0.f;
-            for (int h2 = 0; h2 < p.Hkv; ++h2)
-                r += tile_sum(part0 + static_cast<size_t>(h2) * p.MT * P + col, p.MT, P);
+    for (int i0 = 0; i0 < n; i0 += 8 * kSelThreads) {
+        int col[8], ps[8];
+        bool act[8];
+        float s[8], r[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {  // positions first: their loads overlap the sums'
+            const int i = i0 + tid + e * kSelThreads;
+            act[e] = i < n;
+            col[e] = !act[e] ? 0 : i < count ? i : B + (i - count);
+            ps[e] = !act[e] ? 0 : i < count ? pos[i] : L + (i - count);
+            r[e] = 0.f;
         }
-        const int ps = i < count ? pos[i] : L + (i - count);
-        key[i] = (static_cast<uint64_t>(__float_as_uint(r)) << 32) |
-                 static_cast<uint32_t>(0xFFFFFFFFu - static_cast<uint32_t>(ps));
-        if (imp_out) imp_out[col] = s;
+        tiles_sum(part, p.MT, P, col, act, s);
+        if (p.shared) {  // the ranking score: the same sums for every KV head, heads in order
+            for (int h2 = 0; h2 < p.Hkv; ++h2) {
+                float sh[8];
+                tiles_sum(part0 + static_cast<size_t>(h2) * p.MT * P, p.MT, P, col, act, sh);
+#pragma unroll
+                for (int e = 0; e < 8; ++e) r[e] += sh[e];
+            }
+        }
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            if (!act[e]) continue;
+            const int i = i0 + tid + e * kSelThreads;
+            const float rank = p.shared ? r[e] : s[e];
+            key[i] = (static_cast<uint64_t>(__float_as_uint(rank)) << 32) |
+                     static_cast<uint32_t>(0xFFFFFFFFu - static_cast<uint32_t>(ps[e]));
+            if (imp_out) imp_out[col[e]] = s[e];
+        }
     }
     if (imp_out)
         for (int c = count + tid; c < B; c += kSelThreads) imp_out[c] = 0.f;
@@ -187,25 +215,25 @@ __global__ void __launch_bounds__(kSelThreads)
         prefix = 0;  // every member kept
     }
 
-    // 3. free slots (evicted or empty, ascending) and admitted tokens (ascending)
+    // 3. free slots (evicted or empty, ascending) and admitted tokens (ascending):
+    // one block scan over both counts, packed as free + (admitted << 16)
+    // (at most kMaxPool < 2^16 free slots, and kMaxFrameTokens admitted)
     const int per = (B + kSelThreads - 1) / kSelThreads;
-    int local_free = 0;
+    const int tper = (T + kSelThreads - 1) / kSelThreads;
+    int local_free = 0, local_adm = 0;
     for (int s = tid * per; s < min(B, (tid + 1) * per); ++s)
         local_free += (s >= count || (key[s] & mask) < prefix) ? 1 : 0;
+    for (int t = tid * tper; t < min(T, (tid + 1) * tper); ++t)
+        local_adm += ((key[count + t] & mask) >= prefix) ? 1 : 0;
     int excl;
-    const int nfree = block_exclusive_scan(local_free, warp_sums, excl);
-    int slot_rank = excl;
+    const int tot = block_exclusive_scan(local_free + (local_adm << 16), warp_sums, excl);
+    const int nfree = tot & 0xFFFF, nadm = tot >> 16;
+    int slot_rank = excl & 0xFFFF, tok_rank = excl >> 16;
     for (int s = tid * per; s < min(B, (tid + 1) * per); ++s)
         if (s >= count || (key[s] & mask) < prefix) {
             if (slot_rank < T) free_slot[slot_rank] = s;
             ++slot_rank;
         }
-    const int tper = (T + kSelThreads - 1) / kSelThreads;
-    int local_adm = 0;
-    for (int t = tid * tper; t < min(T, (tid + 1) * tper); ++t)
-        local_adm += ((key[count + t] & mask) >= prefix) ? 1 : 0;
-    const int nadm = block_exclusive_scan(local_adm, warp_sums, excl);
-    int tok_rank = excl;
     for (int t = tid * tper; t < min(T, (tid + 1) * tper); ++t)
         if ((key[count + t] & mask) >= prefix) adm_tok[tok_rank++] = t;
     __syncthreads();
