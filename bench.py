@@ -650,7 +650,9 @@ def run_decode(args, local):
         "token_p50_us": 1e3 * p50,
         "tokens_per_s": 1e3 / p50,
         "kv_read_gbs_at_p50": cache_bytes / (p50 * 1e-3) / 1e9,
-        "note": "one call = every (stream, layer); the attention kernel reads K twice (two passes)",
+        "note": "one call = every (stream, layer); single tokens (<= 16 query rows per KV head) "
+                "run the one-pass split-K decode kernel, which reads each K and V row once; the "
+                "prompt runs the two-pass attention kernel",
     }
     print(json.dumps(line), flush=True)
 

@@ -19,7 +19,7 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 OUT = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libstatekv.so")
-SOURCES = ["attn_kernel.cu", "select_kernel.cu", "diag_kernel.cu", "block_kernel.cu",
+SOURCES = ["attn_kernel.cu", "select_kernel.cu", "diag_kernel.cu", "block_kernel.cu", "decode_kernel.cu",
            "statekv_api.cu", "noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",

@@ -970,6 +970,8 @@ cudaError_t launch_one(const CUtensorMap& tm_sk, const CUtensorMap& tm_sv, const
 
 }  // namespace
 
+int device_sm_count() { return g_num_sms > 0 ? g_num_sms : 1; }
+
 size_t attn_smem_bytes(int D)
 {
     return D == 64 ? AttnLayout<64>::kAlloc : AttnLayout<128>::kAlloc;

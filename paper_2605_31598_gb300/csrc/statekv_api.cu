@@ -87,7 +87,10 @@ Layout make_layout(const statekv_config& c, const Derived& d)
     L.text = take(heads * 4);  // decode-cache rows appended after the video frames
     L.cache_k = take(heads * static_cast<size_t>(d.cap) * D * 2);
     L.cache_v = take(heads * static_cast<size_t>(d.cap) * D * 2);
-    L.partials = take(heads * d.MT * static_cast<size_t>(d.P) * 4);
+    // importance partials of a frame step; a decode step's split-K partials
+    // use the same bytes (the two never overlap in time on a handle)
+    L.partials = take(std::max(heads * d.MT * static_cast<size_t>(d.P) * 4,
+                               heads * kDecodeMaxChunks * kDecodeRows * (static_cast<size_t>(D) + 2) * 4));
     if (c.host_staging) {
         L.stg_q = take(static_cast<size_t>(d.SL) * T * c.num_q_heads * D * 2);
         L.stg_k = take(heads * T * D * 2);
@@ -383,6 +386,75 @@ statekv_status run_decode(statekv_handle* h, const statekv_decode_args& a, cudaS
     const int U = a.stream_count * a.layer_count;
     const int D = c.head_dim, T = c.tokens_per_frame, Hkv = c.num_kv_heads, n = a.num_tokens;
     const UnitRange ur{a.stream_begin, a.layer_begin, a.layer_count, c.num_layers};
+    int32_t* frames = h->at<int32_t>(h->lay.frames);
+    int32_t* text = h->at<int32_t>(h->lay.text);
+    AppendParams ap{};
+    ap.k = static_cast<const __nv_bfloat16*>(a.k);
+    ap.v = static_cast<const __nv_bfloat16*>(a.v);
+    ap.cache_k = h->at<__nv_bfloat16>(h->lay.cache_k);
+    ap.cache_v = h->at<__nv_bfloat16>(h->lay.cache_v);
+    ap.frames = frames;
+    ap.row_add = text;
+    ap.units = ur;
+    ap.U = U;
+    ap.T = n;
+    ap.Hkv = Hkv;
+    ap.D = D;
+    ap.row_mul = T;
+    ap.cap = d.cap;
+    if (n * d.G <= kDecodeRows) {
+        // A few rows: the new tokens' K/V go into the cache first, then the
+        // one-pass split-K kernel reads every key once from the cache.
+        long long maxlen = 0;
+        for (int s = a.stream_begin; s < a.stream_begin + a.stream_count; ++s)
+            for (int l = a.layer_begin; l < a.layer_begin + a.layer_count; ++l) {
+                const size_t unit = static_cast<size_t>(s) * c.num_layers + l;
+                maxlen = std::max(maxlen, static_cast<long long>(h->frames_host[unit]) * T +
+                                              h->text_host[unit] + n);
+            }
+        // chunk count: the one whose waves of CTAs (one per SM) take the least
+        // time, counting each CTA's fixed cost as ~512 keys of streaming
+        DecodeParams dp{};
+        {
+            const long long units = static_cast<long long>(U) * Hkv, sms = device_sm_count();
+            long long best = -1;
+            for (int nc = 1; nc <= kDecodeMaxChunks; ++nc) {
+                const long long ck = std::max(128ll, ((maxlen + nc - 1) / nc + 127) / 128 * 128);
+                const long long used = (maxlen + ck - 1) / ck;
+                const long long waves = (units * used + sms - 1) / sms;
+                const long long cost = waves * (ck + 512);
+                if (best < 0 || cost < best) {
+                    best = cost;
+                    dp.ck = static_cast<int>(ck);
+                    dp.nchunk = static_cast<int>(used);
+                }
+            }
+        }
+        dp.q = static_cast<const __nv_bfloat16*>(a.q);
+        dp.out = static_cast<__nv_bfloat16*>(a.out);
+        dp.cache_k = ap.cache_k;
+        dp.cache_v = ap.cache_v;
+        dp.frames = frames;
+        dp.text = text;
+        dp.part_o = h->at<float>(h->lay.partials);
+        dp.part_ml = dp.part_o + static_cast<size_t>(U) * Hkv * dp.nchunk * kDecodeRows * D;
+        dp.units = ur;
+        dp.n = n;
+        dp.G = d.G;
+        dp.Hq = c.num_q_heads;
+        dp.Hkv = Hkv;
+        dp.T = T;
+        dp.cap = d.cap;
+        dp.scale_log2 = d.scale * 1.4426950408889634f;
+        if (timed(h, 0, st, [&] { return launch_append(ap, st); }) != cudaSuccess ||
+            timed(h, 1, st, [&] { return launch_decode(dp, D, U, st); }) != cudaSuccess ||
+            launch_advance(text, ur, U, Hkv, n, st) != cudaSuccess)
+            return STATEKV_ERR_CUDA;
+        for (int s = a.stream_begin; s < a.stream_begin + a.stream_count; ++s)
+            for (int l = a.layer_begin; l < a.layer_begin + a.layer_count; ++l)
+                h->text_host[static_cast<size_t>(s) * c.num_layers + l] += n;
+        return STATEKV_OK;
+    }
     CUtensorMap tm_nk, tm_nv;
     {
         const cuuint64_t dims[4] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(Hkv),
@@ -395,8 +467,6 @@ statekv_status run_decode(statekv_handle* h, const statekv_decode_args& a, cudaS
             !encode_4d(&tm_nv, a.v, dims, strides, box))
             return STATEKV_ERR_CUDA;
     }
-    int32_t* frames = h->at<int32_t>(h->lay.frames);
-    int32_t* text = h->at<int32_t>(h->lay.text);
     AttnParams pa{};
     pa.q = static_cast<const __nv_bfloat16*>(a.q);
     pa.out = static_cast<__nv_bfloat16*>(a.out);
@@ -419,20 +489,6 @@ statekv_status run_decode(statekv_handle* h, const statekv_decode_args& a, cudaS
     if (timed(h, 1, st, [&] { return launch_attn(D, h->tm_ck, h->tm_cv, tm_nk, tm_nv, pa, U, st); }) !=
         cudaSuccess)
         return STATEKV_ERR_CUDA;
-    AppendParams ap{};
-    ap.k = static_cast<const __nv_bfloat16*>(a.k);
-    ap.v = static_cast<const __nv_bfloat16*>(a.v);
-    ap.cache_k = h->at<__nv_bfloat16>(h->lay.cache_k);
-    ap.cache_v = h->at<__nv_bfloat16>(h->lay.cache_v);
-    ap.frames = frames;
-    ap.row_add = text;
-    ap.units = ur;
-    ap.U = U;
-    ap.T = n;
-    ap.Hkv = Hkv;
-    ap.D = D;
-    ap.row_mul = T;
-    ap.cap = d.cap;
     if (timed(h, 0, st, [&] { return launch_append(ap, st); }) != cudaSuccess ||
         launch_advance(text, ur, U, Hkv, n, st) != cudaSuccess)
         return STATEKV_ERR_CUDA;
@@ -498,7 +554,8 @@ statekv_status statekv_init(const statekv_config* cfg, void* device_arena, size_
     h->status_dev = static_cast<int32_t*>(st_dev);
 
     const int D = cfg->head_dim, B = cfg->state_capacity, Hkv = cfg->num_kv_heads;
-    bool ok = attn_prepare(D) == cudaSuccess && select_prepare() == cudaSuccess;
+    bool ok = attn_prepare(D) == cudaSuccess && select_prepare() == cudaSuccess &&
+              decode_prepare() == cudaSuccess;
     if (ok && B > 0) {
         const cuuint64_t dims[4] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(B),
                                     static_cast<cuuint64_t>(Hkv), static_cast<cuuint64_t>(d.SL)};

@@ -145,6 +145,28 @@ bool lt_matmul(LtContext* c, const __nv_bfloat16* X, const __nv_bfloat16* W,
                const __nv_bfloat16* bias, __nv_bfloat16* D, bool add, int M, int N, int K,
                void* ws, size_t ws_bytes, cudaStream_t st);
 
+// One-pass split-K decoding over the cache (decode_kernel.cu): for up to
+// kDecodeRows query rows (new tokens x query heads of a KV head).
+constexpr int kDecodeRows = 16;
+constexpr int kDecodeMaxChunks = 64;
+struct DecodeParams {
+    const __nv_bfloat16* q;     // [U][n][Hq][D]
+    __nv_bfloat16* out;         // [U][n][Hq][D]
+    const __nv_bfloat16* cache_k;  // arena [S*L][Hkv][cap][D]
+    const __nv_bfloat16* cache_v;
+    const int32_t* frames;      // arena [S*L][Hkv]: rows before = frames * T + text
+    const int32_t* text;
+    float* part_o;              // [U][Hkv][nchunk][kDecodeRows][D]
+    float* part_ml;             // [U][Hkv][nchunk][kDecodeRows][2]
+    UnitRange units;
+    int n, G, Hq, Hkv, T;
+    long long cap;
+    int ck, nchunk;             // keys per chunk (a multiple of 256), chunks
+    float scale_log2;
+};
+cudaError_t launch_decode(const DecodeParams& p, int D, int U, cudaStream_t st);
+cudaError_t decode_prepare();  // once, before the first launch_decode
+
 // Recency-window state update (the baseline): the frame's tokens enter ring
 // slots position mod B, overwriting the tokens that leave the window.
 cudaError_t launch_recency(const RecencyParams& p, cudaStream_t st);
@@ -162,6 +184,7 @@ constexpr int kMaxFrameTokens = 4096;
 size_t select_smem_bytes(int P, int T);
 
 cudaError_t attn_prepare(int D);
+int device_sm_count();  // SMs of the device (read by attn_prepare)
 cudaError_t select_prepare();
 cudaError_t launch_attn(int D, const CUtensorMap& tm_sk, const CUtensorMap& tm_sv,
                         const CUtensorMap& tm_fk, const CUtensorMap& tm_fv, const AttnParams& p,
