@@ -257,10 +257,13 @@ statekv_status statekv_block_workspace_bytes(const statekv_handle* h,
  *            layer layer_begin; not modified
  *   x_out    bf16 [stream_count][T][hidden] (device): layer
  *            layer_begin + layer_count - 1's output (may equal x_in)
- * Every covered (stream, layer) advances by one frame.  Errors as
- * statekv_prefill_frame, INVALID_ARG for a bad block config (head_dim > 128
- * pairs, sizes not multiples of 8), UNSUPPORTED if cuBLASLt finds no GEMM
- * plan; nothing is enqueued on an argument error. */
+ * Every covered (stream, layer) advances by one frame.  The first call for a
+ * given stream count times cuBLASLt's candidate algorithms for each projection
+ * shape on the call's operands and keeps the fastest; that call synchronises
+ * the stream (so it cannot be captured into a CUDA graph), later calls do not.
+ * Errors as statekv_prefill_frame, INVALID_ARG for a bad block config
+ * (head_dim > 128 pairs, sizes not multiples of 8), UNSUPPORTED if cuBLASLt
+ * finds no GEMM plan; nothing is enqueued on an argument error. */
 statekv_status statekv_block_frame(statekv_handle* h, const statekv_block_config* bc,
                                    const statekv_block_weights* weights, int32_t stream_begin,
                                    int32_t stream_count, int32_t layer_begin, int32_t layer_count,

@@ -173,13 +173,21 @@ cudaError_t launch_silu_mul(const __nv_bfloat16* gu, __nv_bfloat16* a, long long
 }
 
 // ------------------------------------------------------------------ GEMMs
+// cuBLASLt's first heuristic choice is not always its fastest for the block's
+// shapes (196 rows per stream against thousands of output features), so the
+// first call of each shape times up to kLtCandidates of its candidates on the
+// call's own operands and keeps the fastest.
+constexpr int kLtCandidates = 8;
+
 struct LtPlan {
     int M, N, K;
     bool bias, add;
     cublasLtMatmulDesc_t op = nullptr;
     cublasLtMatrixLayout_t a = nullptr, b = nullptr, c = nullptr;
-    cublasLtMatmulAlgo_t algo;
-    size_t ws = 0;
+    int nalgo = 0, chosen = 0;
+    bool tuned = false;
+    cublasLtMatmulAlgo_t algo[kLtCandidates];
+    size_t ws[kLtCandidates];
 };
 
 struct LtContext {
@@ -217,8 +225,7 @@ namespace {
 LtPlan* lt_plan(LtContext* c, int M, int N, int K, bool bias, bool add, size_t ws_bytes)
 {
     for (LtPlan& p : c->plans)
-        if (p.M == M && p.N == N && p.K == K && p.bias == bias && p.add == add && p.ws <= ws_bytes)
-            return &p;
+        if (p.M == M && p.N == N && p.K == K && p.bias == bias && p.add == add) return &p;
     LtPlan p;
     p.M = M;
     p.N = N;
@@ -245,9 +252,9 @@ LtPlan* lt_plan(LtContext* c, int M, int N, int K, bool bias, bool add, size_t w
     ok = ok && cublasLtMatmulPreferenceCreate(&pref) == CUBLAS_STATUS_SUCCESS &&
          cublasLtMatmulPreferenceSetAttribute(pref, CUBLASLT_MATMUL_PREF_MAX_WORKSPACE_BYTES,
                                               &ws_bytes, sizeof ws_bytes) == CUBLAS_STATUS_SUCCESS;
-    cublasLtMatmulHeuristicResult_t res{};
+    cublasLtMatmulHeuristicResult_t res[kLtCandidates] = {};
     int found = 0;
-    ok = ok && cublasLtMatmulAlgoGetHeuristic(c->h, p.op, p.a, p.b, p.c, p.c, pref, 1, &res,
+    ok = ok && cublasLtMatmulAlgoGetHeuristic(c->h, p.op, p.a, p.b, p.c, p.c, pref, kLtCandidates, res,
                                               &found) == CUBLAS_STATUS_SUCCESS &&
          found > 0;
     if (pref) cublasLtMatmulPreferenceDestroy(pref);
@@ -258,17 +265,29 @@ LtPlan* lt_plan(LtContext* c, int M, int N, int K, bool bias, bool add, size_t w
         cublasLtMatmulDescDestroy(p.op);
         return nullptr;
     }
-    p.algo = res.algo;
-    p.ws = res.workspaceSize;
+    for (int i = 0; i < found; ++i) {
+        p.algo[i] = res[i].algo;
+        p.ws[i] = res[i].workspaceSize;
+    }
+    p.nalgo = found;
+    p.tuned = found <= 1;
     c->plans.push_back(p);
     return &c->plans.back();
+}
+
+bool lt_run(LtContext* c, const LtPlan& p, int i, const __nv_bfloat16* X, const __nv_bfloat16* W,
+            __nv_bfloat16* D, float beta, void* ws, cudaStream_t st)
+{
+    const float alpha = 1.f;
+    return cublasLtMatmul(c->h, p.op, &alpha, W, p.a, X, p.b, &beta, D, p.c, D, p.c, &p.algo[i], ws,
+                          p.ws[i], st) == CUBLAS_STATUS_SUCCESS;
 }
 
 }  // namespace
 
 bool lt_matmul(LtContext* c, const __nv_bfloat16* X, const __nv_bfloat16* W,
                const __nv_bfloat16* bias, __nv_bfloat16* D, bool add, int M, int N, int K,
-               void* ws, size_t ws_bytes, cudaStream_t st)
+               void* ws, size_t ws_bytes, void* scratch, size_t scratch_bytes, cudaStream_t st)
 {
     if (M <= 0) return true;
     LtPlan* p = lt_plan(c, M, N, K, bias != nullptr, add, ws_bytes);
@@ -276,9 +295,36 @@ bool lt_matmul(LtContext* c, const __nv_bfloat16* X, const __nv_bfloat16* W,
     if (bias && cublasLtMatmulDescSetAttribute(p->op, CUBLASLT_MATMUL_DESC_BIAS_POINTER, &bias,
                                                sizeof bias) != CUBLAS_STATUS_SUCCESS)
         return false;
-    const float alpha = 1.f, beta = add ? 1.f : 0.f;
-    return cublasLtMatmul(c->h, p->op, &alpha, W, p->a, X, p->b, &beta, D, p->c, D, p->c, &p->algo,
-                          ws, p->ws, st) == CUBLAS_STATUS_SUCCESS;
+    if (!p->tuned) {
+        // time each candidate (beta = 0) into scratch, or into D when D is
+        // written over anyway; a candidate that fails is skipped
+        __nv_bfloat16* out = static_cast<size_t>(M) * N * 2 <= scratch_bytes
+                                 ? static_cast<__nv_bfloat16*>(scratch)
+                                 : (!add ? D : nullptr);
+        cudaEvent_t e0 = nullptr, e1 = nullptr;
+        if (out && cudaEventCreate(&e0) == cudaSuccess && cudaEventCreate(&e1) == cudaSuccess) {
+            float best = -1.f;
+            for (int i = 0; i < p->nalgo; ++i) {
+                if (!lt_run(c, *p, i, X, W, out, 0.f, ws, st)) continue;  // warm-up
+                cudaEventRecord(e0, st);
+                bool ok = true;
+                for (int r = 0; r < 3 && ok; ++r) ok = lt_run(c, *p, i, X, W, out, 0.f, ws, st);
+                cudaEventRecord(e1, st);
+                float ms = 0.f;
+                if (!ok || cudaEventSynchronize(e1) != cudaSuccess ||
+                    cudaEventElapsedTime(&ms, e0, e1) != cudaSuccess)
+                    continue;
+                if (best < 0.f || ms < best) {
+                    best = ms;
+                    p->chosen = i;
+                }
+            }
+        }
+        if (e0) cudaEventDestroy(e0);
+        if (e1) cudaEventDestroy(e1);
+        p->tuned = true;
+    }
+    return lt_run(c, *p, p->chosen, X, W, D, add ? 1.f : 0.f, ws, st);
 }
 
 }  // namespace statekv

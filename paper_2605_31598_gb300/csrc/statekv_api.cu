@@ -722,7 +722,8 @@ struct BlockBufs {
     size_t h, qkv, q, k, v, attn, gu, act, lt, total;
 };
 
-constexpr size_t kLtWorkspace = 32u << 20;
+constexpr size_t kLtWorkspace = 32u << 20;  // cuBLASLt's own workspace
+constexpr size_t kLtScratch = 32u << 20;    // output of the one-time algorithm timing
 
 BlockBufs block_bufs(const statekv_config& c, const statekv_block_config& b, int streams)
 {
@@ -744,7 +745,7 @@ BlockBufs block_bufs(const statekv_config& c, const statekv_block_config& b, int
     o.attn = take(rows * hq * d * 2);
     o.gu = take(rows * 2 * static_cast<size_t>(b.intermediate) * 2);
     o.act = take(rows * static_cast<size_t>(b.intermediate) * 2);
-    o.lt = take(kLtWorkspace);
+    o.lt = take(kLtWorkspace + kLtScratch);
     o.total = off;
     return o;
 }
@@ -854,7 +855,8 @@ statekv_status statekv_block_frame(statekv_handle* h, const statekv_block_config
                    return lt_matmul(h->lt, static_cast<const __nv_bfloat16*>(X),
                                     static_cast<const __nv_bfloat16*>(Wt),
                                     static_cast<const __nv_bfloat16*>(bias), D, add, rows, N, K,
-                                    ltws, kLtWorkspace, st)
+                                    ltws, kLtWorkspace, static_cast<uint8_t*>(ltws) + kLtWorkspace,
+                                    kLtScratch, st)
                               ? cudaSuccess
                               : cudaErrorNotSupported;
                }) == cudaSuccess;

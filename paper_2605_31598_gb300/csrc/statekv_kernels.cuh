@@ -140,10 +140,12 @@ struct LtContext;
 LtContext* lt_create();
 void lt_destroy(LtContext* c);
 // Row-major D[M][N] = X[M][K] W[N][K]^T (+ bias[N]) (+ D when add), bf16 in and
-// out, fp32 accumulation; false if cuBLASLt has no plan or fails.
+// out, fp32 accumulation; false if cuBLASLt has no plan or fails.  The first
+// call of a shape times cuBLASLt's candidate algorithms (synchronising the
+// stream once) into `scratch` (or into D when it is overwritten anyway).
 bool lt_matmul(LtContext* c, const __nv_bfloat16* X, const __nv_bfloat16* W,
                const __nv_bfloat16* bias, __nv_bfloat16* D, bool add, int M, int N, int K,
-               void* ws, size_t ws_bytes, cudaStream_t st);
+               void* ws, size_t ws_bytes, void* scratch, size_t scratch_bytes, cudaStream_t st);
 
 // One-pass split-K decoding over the cache (decode_kernel.cu): for up to
 // kDecodeRows query rows (new tokens x query heads of a KV head).
