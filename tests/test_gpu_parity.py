@@ -156,3 +156,65 @@ def test_qwen7b_stack_full_size_sampled_units():
     stats = {}
     run_parity(shape, 12, check_frames=[11, 12], units=[(0, 0), (0, 27)], stats=stats)
     print("qwen7b_stack", stats)
+
+
+@pytest.mark.gpu
+def test_streams_at_different_frames_in_one_launch():
+    """One launch whose units see different key ranges: stream 0 runs three
+    frames ahead of stream 1, so the persistent attention kernel walks units
+    with different state sizes (and tile counts) side by side.  Every frame
+    of both streams is checked against the oracle started from the GPU's
+    pre-frame state (outputs within 2e-2, importance within 1e-3)."""
+    import numpy as np
+
+    import oracle
+    from paper_2605_31598_gb300 import StateKV, make_config
+    from paper_2605_31598_gb300.inputs import batch_qkv
+
+    from .parity import IMP_ATOL, IMP_RTOL, OUT_ATOL
+
+    shape = Shape(8, 2, 128, 64, 160, 9, num_layers=2, num_streams=2)
+    S, L, T, Hq, Hkv, d, B = 2, 2, 64, 8, 2, 128, 160
+    eng = StateKV(make_config(shape))
+    lays = {(s, l): oracle.OracleLayer(Hq, Hkv, d, T, B, shape.max_frames) for s in range(S) for l in range(L)}
+    done = [0, 0]
+
+    def run(streams):
+        frames = [done[s] + 1 for s in streams]
+        q, k, v = batch_qkv(shape, frames, streams=streams, layers=range(L), device="cuda")
+        torch.cuda.synchronize()
+        pre = {}
+        for si, s in enumerate(streams):
+            for l in range(L):
+                kk, vv, pp, info = eng.state(s, l)
+                pre[(s, l)] = (info.count, pp.cpu().numpy().astype(np.int64), oracle.as_bf16_bits(kk),
+                               oracle.as_bf16_bits(vv), info.virtual_len)
+        out = torch.full_like(q, float("nan"))
+        imp = torch.full((len(streams), L, Hkv, B + T), float("nan"), device="cuda")
+        assert eng.prefill_frame(q, k, v, out, imp, stream_begin=streams[0],
+                                 stream_count=len(streams)) == 0
+        torch.cuda.synchronize()
+        for si, s in enumerate(streams):
+            for l in range(L):
+                count, ppos, pk, pv, vlen = pre[(s, l)]
+                lay = lays[(s, l)]
+                lay.set_state(np.full(Hkv, count, np.int32), ppos, pk, pv, vlen)
+                o_ref, imp_ref, _ = lay.prefill_frame(*(oracle.as_bf16_bits(x[si, l]) for x in (q, k, v)))
+                err = float(np.abs(out[si, l].float().cpu().numpy() - o_ref).max())
+                assert err <= OUT_ATOL, (s, l, done[s] + 1, err)
+                g = imp[si, l].cpu().numpy().astype(np.float64)
+                for h in range(Hkv):
+                    order = {int(p): i for i, p in enumerate(np.sort(ppos[h, :count]))}
+                    ref = np.array([imp_ref[h, order[int(ppos[h, j])]] for j in range(count)] +
+                                   list(imp_ref[h, B:]))
+                    got = np.concatenate([g[h, :count], g[h, B:]])
+                    assert np.all(np.abs(got - ref) <= IMP_RTOL * np.abs(ref) + IMP_ATOL), (s, l, h)
+        for s in streams:
+            done[s] += 1
+
+    for _ in range(3):
+        run([0])
+    for _ in range(5):
+        run([0, 1])
+    assert done == [8, 5]
+    assert eng.sync() == 0
