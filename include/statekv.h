@@ -74,7 +74,7 @@ typedef struct {
     int32_t max_frames;       /* decode-cache capacity per stream/layer, in frames */
     int32_t causal_in_frame;  /* 1: key t visible to query i iff t <= i (Eq. 5's M_n);
                                  0: every frame key visible (variant) */
-    int32_t host_staging;     /* 1: reserve arena space for statekv_prefill_frame_host */
+    int32_t host_staging;     /* 1: reserve arena space (two frames) for the host-buffer calls */
     float softmax_scale;      /* 0 -> 1 / sqrt(head_dim) (Eq. 5) */
     uint32_t watchdog_ms;     /* bound on every device-side wait; 0 -> 2000 ms */
     int32_t selection;        /* which B tokens the state keeps after each frame:
@@ -301,6 +301,22 @@ statekv_status statekv_decode_step(statekv_handle* h, const statekv_decode_args*
  * must stay valid until the stream is synchronised.  Needs host_staging = 1. */
 statekv_status statekv_prefill_frame_host(statekv_handle* h, const statekv_frame_args* args,
                                           statekv_stream stream);
+
+/* n consecutive frames (Sec. 3.3's per-frame step, n times) from HOST
+ * buffers, with the copies pipelined against the steps: frames[i] holds the
+ * host q/k/v/out (and importance, or null) of frame i, laid out as in
+ * statekv_prefill_frame_host.  Every entry must cover the same streams and
+ * layers, and either every entry or none has an importance buffer.  The
+ * arena's staging area holds two frames; frame i + 1 is copied in on an
+ * internal copy stream while frame i runs on `stream`, and frame i - 1 is
+ * copied out on another.  Ordering: the first copy waits for the work
+ * already enqueued on `stream`, and `stream` waits for the last copy out, so
+ * the results are in the host buffers once `stream` is synchronised.  Host
+ * buffers must stay valid (and the inputs unchanged) until then.  Returns
+ * CACHE_FULL (with no work enqueued) if a covered (stream, layer) cannot take
+ * n more frames.  Needs host_staging = 1. */
+statekv_status statekv_prefill_frames_host(statekv_handle* h, const statekv_frame_args* frames,
+                                           int32_t n, statekv_stream stream);
 
 typedef struct {
     const void* k;            /* bf16 [Hkv][B][d] (device); slot order is arbitrary */

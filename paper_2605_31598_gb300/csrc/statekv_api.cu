@@ -29,7 +29,9 @@ size_t round_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
 struct Layout {
     size_t state_k, state_v, positions, counts, frames, text, cache_k, cache_v, partials;
-    size_t stg_q, stg_k, stg_v, stg_out, stg_imp;
+    struct Staging {
+        size_t q, k, v, out, imp;
+    } stg[2];  // host-buffer calls: two frames, so copies overlap the steps
     size_t total;
 };
 
@@ -92,11 +94,13 @@ Layout make_layout(const statekv_config& c, const Derived& d)
     L.partials = take(std::max(heads * d.MT * static_cast<size_t>(d.P) * 4,
                                heads * kDecodeMaxChunks * kDecodeRows * (static_cast<size_t>(D) + 2) * 4));
     if (c.host_staging) {
-        L.stg_q = take(static_cast<size_t>(d.SL) * T * c.num_q_heads * D * 2);
-        L.stg_k = take(heads * T * D * 2);
-        L.stg_v = take(heads * T * D * 2);
-        L.stg_out = take(static_cast<size_t>(d.SL) * T * c.num_q_heads * D * 2);
-        L.stg_imp = take(heads * static_cast<size_t>(d.P) * 4);
+        for (auto& g : L.stg) {
+            g.q = take(static_cast<size_t>(d.SL) * T * c.num_q_heads * D * 2);
+            g.k = take(heads * T * D * 2);
+            g.v = take(heads * T * D * 2);
+            g.out = take(static_cast<size_t>(d.SL) * T * c.num_q_heads * D * 2);
+            g.imp = take(heads * static_cast<size_t>(d.P) * 4);
+        }
     }
     L.total = off;
     return L;
@@ -160,12 +164,36 @@ struct statekv_handle {
     // attention kernel writes, so it fills SMs the attention grid leaves idle.
     cudaStream_t side = nullptr;
     cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
+    // Pipelined host-buffer frames: copies in and out run on their own
+    // streams; per staging set, "copied in", "step done", "copied out".
+    cudaStream_t cin = nullptr, cout = nullptr;
+    cudaEvent_t ev_start = nullptr, ev_in[2] = {}, ev_comp[2] = {}, ev_out[2] = {};
 
     template <class T>
     T* at(size_t off) const { return reinterpret_cast<T*>(arena + off); }
 };
 
 namespace {
+
+bool create_streams(statekv_handle* h)
+{
+    bool ok = cudaStreamCreateWithFlags(&h->side, cudaStreamNonBlocking) == cudaSuccess &&
+              cudaStreamCreateWithFlags(&h->cin, cudaStreamNonBlocking) == cudaSuccess &&
+              cudaStreamCreateWithFlags(&h->cout, cudaStreamNonBlocking) == cudaSuccess;
+    for (cudaEvent_t* e : {&h->ev_fork, &h->ev_join, &h->ev_start, &h->ev_in[0], &h->ev_in[1],
+                           &h->ev_comp[0], &h->ev_comp[1], &h->ev_out[0], &h->ev_out[1]})
+        ok = ok && cudaEventCreateWithFlags(e, cudaEventDisableTiming) == cudaSuccess;
+    return ok;
+}
+
+void release_streams(statekv_handle* h)
+{
+    for (cudaEvent_t e : {h->ev_fork, h->ev_join, h->ev_start, h->ev_in[0], h->ev_in[1],
+                          h->ev_comp[0], h->ev_comp[1], h->ev_out[0], h->ev_out[1]})
+        if (e) cudaEventDestroy(e);
+    for (cudaStream_t st : {h->side, h->cin, h->cout})
+        if (st) cudaStreamDestroy(st);
+}
 
 statekv_status device_status(int32_t word)
 {
@@ -576,9 +604,7 @@ statekv_status statekv_init(const statekv_config* cfg, void* device_arena, size_
         ok = encode_4d(&h->tm_ck, h->arena + lay.cache_k, dims, strides, box) &&
              encode_4d(&h->tm_cv, h->arena + lay.cache_v, dims, strides, box);
     }
-    ok = ok && cudaStreamCreateWithFlags(&h->side, cudaStreamNonBlocking) == cudaSuccess &&
-         cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming) == cudaSuccess &&
-         cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming) == cudaSuccess;
+    ok = ok && create_streams(h);
     // Empty states and decode caches: zero rows, positions -1.  A key tile that
     // runs past the valid rows of a state or of the cache still reads them;
     // their scores are masked, but P = 0 times a non-finite value row would
@@ -590,9 +616,7 @@ statekv_status statekv_init(const statekv_config* cfg, void* device_arena, size_
          cudaDeviceSynchronize() == cudaSuccess;
     if (!ok) {
         cudaFreeHost(st_host);
-        if (h->ev_fork) cudaEventDestroy(h->ev_fork);
-        if (h->ev_join) cudaEventDestroy(h->ev_join);
-        if (h->side) cudaStreamDestroy(h->side);
+        release_streams(h);
         delete h;
         return STATEKV_ERR_CUDA;
     }
@@ -930,12 +954,17 @@ statekv_status statekv_prefill_frame_host(statekv_handle* h, const statekv_frame
     const size_t qbytes = U * T * c.num_q_heads * D * 2;
     const size_t kvbytes = U * T * c.num_kv_heads * D * 2;
     const size_t impbytes = U * c.num_kv_heads * static_cast<size_t>(h->d.P) * 4;
+    const Layout::Staging& g = h->lay.stg[0];
     statekv_frame_args dev = *args;
-    dev.q = h->arena + h->lay.stg_q;
-    dev.k = h->arena + h->lay.stg_k;
-    dev.v = h->arena + h->lay.stg_v;
-    dev.out = h->arena + h->lay.stg_out;
-    dev.importance = args->importance ? h->at<float>(h->lay.stg_imp) : nullptr;
+    dev.q = h->arena + g.q;
+    dev.k = h->arena + g.k;
+    dev.v = h->arena + g.v;
+    dev.out = h->arena + g.out;
+    dev.importance = args->importance ? h->at<float>(g.imp) : nullptr;
+    // set 0 may still be in use by an earlier pipelined call
+    if (cudaStreamWaitEvent(st, h->ev_comp[0], 0) != cudaSuccess ||
+        cudaStreamWaitEvent(st, h->ev_out[0], 0) != cudaSuccess)
+        return STATEKV_ERR_CUDA;
     if (cudaMemcpyAsync(const_cast<void*>(dev.q), args->q, qbytes, cudaMemcpyHostToDevice, st) !=
             cudaSuccess ||
         cudaMemcpyAsync(const_cast<void*>(dev.k), args->k, kvbytes, cudaMemcpyHostToDevice, st) !=
@@ -950,6 +979,77 @@ statekv_status statekv_prefill_frame_host(statekv_handle* h, const statekv_frame
     if (args->importance &&
         cudaMemcpyAsync(args->importance, dev.importance, impbytes, cudaMemcpyDeviceToHost, st) !=
             cudaSuccess)
+        return STATEKV_ERR_CUDA;
+    return STATEKV_OK;
+}
+
+statekv_status statekv_prefill_frames_host(statekv_handle* h, const statekv_frame_args* frames,
+                                           int32_t n, statekv_stream stream)
+{
+    if (!h || !frames || n < 1) return STATEKV_ERR_INVALID_ARG;
+    const statekv_frame_args& f0 = frames[0];
+    const statekv_status s = check_args(h, &f0, true);
+    if (s != STATEKV_OK) return s;
+    for (int32_t i = 1; i < n; ++i) {
+        const statekv_frame_args& f = frames[i];
+        if (f.stream_begin != f0.stream_begin || f.stream_count != f0.stream_count ||
+            f.layer_begin != f0.layer_begin || f.layer_count != f0.layer_count || !f.q || !f.k ||
+            !f.v || !f.out || (f.importance == nullptr) != (f0.importance == nullptr))
+            return STATEKV_ERR_INVALID_ARG;
+    }
+    const statekv_config& c = h->cfg;
+    for (int sI = f0.stream_begin; sI < f0.stream_begin + f0.stream_count; ++sI)
+        for (int l = f0.layer_begin; l < f0.layer_begin + f0.layer_count; ++l)
+            if (static_cast<long long>(h->frames_host[static_cast<size_t>(sI) * c.num_layers + l]) + n >
+                c.max_frames)
+                return STATEKV_ERR_CACHE_FULL;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    const size_t U = static_cast<size_t>(f0.stream_count) * f0.layer_count;
+    const size_t T = c.tokens_per_frame, D = c.head_dim;
+    const size_t qbytes = U * T * c.num_q_heads * D * 2;
+    const size_t kvbytes = U * T * c.num_kv_heads * D * 2;
+    const size_t impbytes = U * c.num_kv_heads * static_cast<size_t>(h->d.P) * 4;
+    // the copies in start after the work already enqueued on the call's stream
+    if (cudaEventRecord(h->ev_start, st) != cudaSuccess ||
+        cudaStreamWaitEvent(h->cin, h->ev_start, 0) != cudaSuccess)
+        return STATEKV_ERR_CUDA;
+    for (int32_t i = 0; i < n; ++i) {
+        const int b = i & 1;
+        const Layout::Staging& g = h->lay.stg[b];
+        const statekv_frame_args& f = frames[i];
+        statekv_frame_args dev = f;
+        dev.q = h->arena + g.q;
+        dev.k = h->arena + g.k;
+        dev.v = h->arena + g.v;
+        dev.out = h->arena + g.out;
+        dev.importance = f.importance ? h->at<float>(g.imp) : nullptr;
+        // in: once the step that last read this staging set is done
+        if (cudaStreamWaitEvent(h->cin, h->ev_comp[b], 0) != cudaSuccess ||
+            cudaMemcpyAsync(const_cast<void*>(dev.q), f.q, qbytes, cudaMemcpyHostToDevice, h->cin) !=
+                cudaSuccess ||
+            cudaMemcpyAsync(const_cast<void*>(dev.k), f.k, kvbytes, cudaMemcpyHostToDevice, h->cin) !=
+                cudaSuccess ||
+            cudaMemcpyAsync(const_cast<void*>(dev.v), f.v, kvbytes, cudaMemcpyHostToDevice, h->cin) !=
+                cudaSuccess ||
+            cudaEventRecord(h->ev_in[b], h->cin) != cudaSuccess)
+            return STATEKV_ERR_CUDA;
+        // the step: after its inputs landed and the set's previous outputs left
+        if (cudaStreamWaitEvent(st, h->ev_in[b], 0) != cudaSuccess ||
+            cudaStreamWaitEvent(st, h->ev_out[b], 0) != cudaSuccess)
+            return STATEKV_ERR_CUDA;
+        const statekv_status r = run_step(h, dev, st);
+        if (r != STATEKV_OK) return r;
+        if (cudaEventRecord(h->ev_comp[b], st) != cudaSuccess ||
+            cudaStreamWaitEvent(h->cout, h->ev_comp[b], 0) != cudaSuccess ||
+            cudaMemcpyAsync(f.out, dev.out, qbytes, cudaMemcpyDeviceToHost, h->cout) != cudaSuccess ||
+            (f.importance && cudaMemcpyAsync(f.importance, dev.importance, impbytes,
+                                             cudaMemcpyDeviceToHost, h->cout) != cudaSuccess) ||
+            cudaEventRecord(h->ev_out[b], h->cout) != cudaSuccess)
+            return STATEKV_ERR_CUDA;
+    }
+    // later work on the call's stream sees every frame's results
+    if (cudaStreamWaitEvent(st, h->ev_out[0], 0) != cudaSuccess ||
+        cudaStreamWaitEvent(st, h->ev_out[1], 0) != cudaSuccess)
         return STATEKV_ERR_CUDA;
     return STATEKV_OK;
 }
@@ -1042,9 +1142,7 @@ void statekv_destroy(statekv_handle* h)
     }
     cudaFreeHost(const_cast<int32_t*>(h->status_host));
     lt_destroy(h->lt);
-    if (h->ev_fork) cudaEventDestroy(h->ev_fork);
-    if (h->ev_join) cudaEventDestroy(h->ev_join);
-    if (h->side) cudaStreamDestroy(h->side);
+    release_streams(h);
     delete h;
 }
 

@@ -22,7 +22,8 @@ STATUS_NAMES = {
     6: "STATEKV_ERR_ARENA_TOO_SMALL", 7: "STATEKV_ERR_DEVICE_FAULT",
 }
 EXPORTED = ("statekv_arena_bytes", "statekv_init", "statekv_prefill_frame",
-            "statekv_prefill_frame_host", "statekv_full_attention_frame", "statekv_decode_step",
+            "statekv_prefill_frame_host", "statekv_prefill_frames_host",
+            "statekv_full_attention_frame", "statekv_decode_step",
             "statekv_state_view", "statekv_cache_view",
             "statekv_profile_enable", "statekv_profile_read", "statekv_sync",
             "statekv_device_error", "statekv_frame_attention_noalloc",
@@ -111,6 +112,9 @@ def lib() -> ctypes.CDLL:
                 fn = getattr(L, name)
                 fn.argtypes = [ctypes.c_void_p, P(statekv_frame_args), ctypes.c_void_p]
                 fn.restype = st
+            L.statekv_prefill_frames_host.argtypes = [ctypes.c_void_p, P(statekv_frame_args),
+                                                      ctypes.c_int32, ctypes.c_void_p]
+            L.statekv_prefill_frames_host.restype = st
             L.statekv_decode_step.argtypes = [ctypes.c_void_p, P(statekv_decode_args),
                                               ctypes.c_void_p]
             L.statekv_decode_step.restype = st
@@ -201,6 +205,11 @@ def statekv_prefill_frame(handle: int, args: statekv_frame_args, stream: int) ->
 
 def statekv_prefill_frame_host(handle: int, args: statekv_frame_args, stream: int) -> int:
     return lib().statekv_prefill_frame_host(handle, ctypes.byref(args), ctypes.c_void_p(stream))
+
+
+def statekv_prefill_frames_host(handle: int, frames, n: int, stream: int) -> int:
+    """``frames``: a ctypes array of ``n`` statekv_frame_args (host pointers)."""
+    return lib().statekv_prefill_frames_host(handle, frames, n, ctypes.c_void_p(stream))
 
 
 def statekv_full_attention_frame(handle: int, args: statekv_frame_args, stream: int) -> int:
@@ -465,6 +474,21 @@ class StateKV:
         st = (stream or torch.cuda.current_stream()).cuda_stream
         args = self._args(q, k, v, out, importance, stream_begin, sc, layer_begin, lc)
         return statekv_prefill_frame_host(self.handle, args, st)
+
+    def prefill_frames_host(self, frames, *, stream_begin=0, stream_count=None, layer_begin=0,
+                            layer_count=None, stream=None) -> int:
+        """Consecutive frames from pinned host buffers, copies pipelined with the
+        steps: ``frames`` is a sequence of (q, k, v, out, importance-or-None)
+        CPU tensors laid out as for ``prefill_frame_host``.  Returns the C status."""
+        import torch
+
+        sc = self.cfg.num_streams - stream_begin if stream_count is None else stream_count
+        lc = self.cfg.num_layers - layer_begin if layer_count is None else layer_count
+        st = (stream or torch.cuda.current_stream()).cuda_stream
+        arr = (statekv_frame_args * len(frames))()
+        for i, (q, k, v, out, imp) in enumerate(frames):
+            arr[i] = self._args(q, k, v, out, imp, stream_begin, sc, layer_begin, lc)
+        return statekv_prefill_frames_host(self.handle, arr, len(frames), st)
 
     def _arena_view(self, ptr, nbytes, dtype, shape):
         import torch

@@ -96,6 +96,50 @@ def test_host_buffer_entry_point():
     run_parity(Shape(8, 2, 128, 64, 96, 4, num_layers=2), 4, host_api=True)
 
 
+def test_pipelined_host_frames_match_device_calls():
+    """statekv_prefill_frames_host (copies on internal streams, two staging
+    sets) leaves outputs, importance and states bit-identical to one
+    statekv_prefill_frame per frame: two pipelined calls in a row, then a
+    single-frame host call that reuses the first staging set."""
+    shape = Shape(8, 2, 128, 64, 96, 8, num_layers=2, num_streams=2)
+    S, L, H, P = 2, 2, 2, 96 + 64
+    dev = StateKV(make_config(shape))
+    hst = StateKV(make_config(shape, host_staging=True))
+    frames = [batch_qkv(shape, n, streams=range(S), layers=range(L), device="cuda")
+              for n in range(1, 8)]
+    want = []
+    for q, k, v in frames:
+        o = torch.empty_like(q)
+        imp = torch.empty((S, L, H, P), dtype=torch.float32, device="cuda")
+        assert dev.prefill_frame(q, k, v, o, imp) == 0
+        want.append((o, imp))
+    host = [tuple(x.cpu().pin_memory() for x in (q, k, v)) +
+            (torch.empty(q.shape, dtype=torch.bfloat16).pin_memory(),
+             torch.empty((S, L, H, P), dtype=torch.float32).pin_memory())
+            for q, k, v in frames]
+    # refused before any work: mixed importance buffers, too many frames
+    mixed = [host[0], host[1][:4] + (None,)]
+    assert hst.prefill_frames_host(mixed) == 1
+    assert hst.prefill_frames_host(host * 2) == 3  # 14 frames > max_frames = 8
+    torch.cuda.synchronize()
+    assert hst.state(0, 0)[3].frames == 0
+    assert hst.prefill_frames_host(host[:3]) == 0
+    assert hst.prefill_frames_host(host[3:6]) == 0
+    assert hst.prefill_frame_host(*host[6]) == 0
+    torch.cuda.synchronize()
+    for n, (o, imp) in enumerate(want):
+        assert torch.equal(host[n][3].view(torch.int16), o.cpu().view(torch.int16)), f"out, frame {n + 1}"
+        assert torch.equal(host[n][4], imp.cpu()), f"importance, frame {n + 1}"
+    for s_ in range(S):
+        for l_ in range(L):
+            a, b = dev.state(s_, l_), hst.state(s_, l_)
+            assert a[3].frames == b[3].frames == 7 and a[3].count == b[3].count
+            for x, y in zip(a[:3], b[:3]):
+                assert torch.equal(x.view(torch.int16) if x.dtype == torch.bfloat16 else x,
+                                   y.view(torch.int16) if y.dtype == torch.bfloat16 else y)
+    assert dev.sync() == 0 and hst.sync() == 0
+
+
 def test_cache_full_is_refused_without_side_effects():
     shape = Shape(4, 1, 64, 16, 32, 2)
     eng = StateKV(make_config(shape))
