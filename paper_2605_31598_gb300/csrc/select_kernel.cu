@@ -57,26 +57,25 @@ __device__ __forceinline__ int block_exclusive_scan(int x, int* warp_sums, int& 
 }
 
 // For each of 8 pool members (columns col[e], active act[e]): the sum of
-// x[mt * stride + col] over mt < MT, added in mt order.  Eight tiles' loads of
-// all 8 members (64 independent loads) are in flight before any addition, so
-// up to 16 query tiles take two rounds of L2 latency.
+// x[mt * stride + col] over mt < MT, added in mt order.  Four tiles' loads of
+// all 8 members (32 independent loads) are in flight before any addition.
 __device__ __forceinline__ void tiles_sum(const float* x, int MT, int stride, const int (&col)[8],
                                           const bool (&act)[8], float (&s)[8])
 {
 #pragma unroll
     for (int e = 0; e < 8; ++e) s[e] = 0.f;
 #pragma unroll 1
-    for (int mt = 0; mt < MT; mt += 8) {
-        float v[8][8];
+    for (int mt = 0; mt < MT; mt += 4) {
+        float v[4][8];
 #pragma unroll
-        for (int m4 = 0; m4 < 8; ++m4)
+        for (int m4 = 0; m4 < 4; ++m4)
 #pragma unroll
             for (int e = 0; e < 8; ++e)
                 v[m4][e] = (act[e] && mt + m4 < MT)
                                ? __ldg(x + static_cast<size_t>(mt + m4) * stride + col[e])
                                : 0.f;
 #pragma unroll
-        for (int m4 = 0; m4 < 8; ++m4)
+        for (int m4 = 0; m4 < 4; ++m4)
 #pragma unroll
             for (int e = 0; e < 8; ++e)
                 if (mt + m4 < MT) s[e] += v[m4][e];
