@@ -23,7 +23,7 @@
 namespace statekv {
 namespace {
 
-constexpr int kSelThreads = 512;
+constexpr int kSelThreads = 640;
 constexpr int kSelWarps = kSelThreads / 32;
 
 // Exclusive block-wide scan of one int per thread; returns the total.
@@ -82,6 +82,32 @@ __device__ __forceinline__ void tiles_sum(const float* x, int MT, int stride, co
     }
 }
 
+// For 4 adjacent columns c0..c0+3 (16-byte aligned): the sums of
+// x[mt * stride + c] over mt < MT, added in mt order, with up to 12 rows'
+// 16-byte loads in flight at once (one round of L2 latency for up to 12
+// query tiles).
+__device__ __forceinline__ float4 rows_sum4(const float* x, int MT, int stride, int c0)
+{
+    float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 1
+    for (int mt = 0; mt < MT; mt += 12) {
+        float4 v[12];
+#pragma unroll
+        for (int m = 0; m < 12; ++m)
+            v[m] = mt + m < MT ? __ldg(reinterpret_cast<const float4*>(x + static_cast<size_t>(mt + m) * stride + c0))
+                               : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int m = 0; m < 12; ++m)
+            if (mt + m < MT) {
+                s.x += v[m].x;
+                s.y += v[m].y;
+                s.z += v[m].z;
+                s.w += v[m].w;
+            }
+    }
+    return s;
+}
+
 __global__ void __launch_bounds__(kSelThreads)
     state_select_gather(const SelectParams p)
 {
@@ -113,6 +139,42 @@ __global__ void __launch_bounds__(kSelThreads)
     // outside them, so all its loads are independent (the partials come from
     // L2); each member's sum still adds the tiles in order.
     const float* part0 = p.partials + static_cast<size_t>(u) * p.Hkv * p.MT * P;
+    if ((P & 3) == 0) {
+        // Column space, four adjacent columns per thread (16-byte loads): state
+        // slot c < count is member c, frame column B + t is member count + t,
+        // empty slots are skipped.
+        for (int g4 = tid; g4 < (P >> 2); g4 += kSelThreads) {
+            const int c0 = 4 * g4;
+            int ps[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {  // positions first: their loads overlap the sums'
+                const int c = c0 + e;
+                ps[e] = c < count ? pos[c] : L + (c - B);
+            }
+            const float4 s4 = rows_sum4(part, p.MT, P, c0);
+            float4 r4 = s4;
+            if (p.shared) {  // the ranking score: the same sums for every KV head, heads in order
+                r4 = make_float4(0.f, 0.f, 0.f, 0.f);
+                for (int h2 = 0; h2 < p.Hkv; ++h2) {
+                    const float4 t4 = rows_sum4(part0 + static_cast<size_t>(h2) * p.MT * P, p.MT, P, c0);
+                    r4.x += t4.x;
+                    r4.y += t4.y;
+                    r4.z += t4.z;
+                    r4.w += t4.w;
+                }
+            }
+            const float sv[4] = {s4.x, s4.y, s4.z, s4.w}, rv[4] = {r4.x, r4.y, r4.z, r4.w};
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const int c = c0 + e;
+                const int i = c < count ? c : (c >= B && c - B < T) ? count + (c - B) : -1;
+                if (i < 0) continue;
+                key[i] = (static_cast<uint64_t>(__float_as_uint(rv[e])) << 32) |
+                         static_cast<uint32_t>(0xFFFFFFFFu - static_cast<uint32_t>(ps[e]));
+                if (imp_out) imp_out[c] = sv[e];
+            }
+        }
+    } else
     for (int i0 = 0; i0 < n; i0 += 8 * kSelThreads) {
         int col[8], ps[8];
         bool act[8];
