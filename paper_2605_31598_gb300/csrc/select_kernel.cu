@@ -174,36 +174,37 @@ __global__ void __launch_bounds__(kSelThreads)
                 if (imp_out) imp_out[c] = sv[e];
             }
         }
-    } else
-    for (int i0 = 0; i0 < n; i0 += 8 * kSelThreads) {
-        int col[8], ps[8];
-        bool act[8];
-        float s[8], r[8];
+    } else {  // member-wise: up to 8 pool members per thread
+        for (int i0 = 0; i0 < n; i0 += 8 * kSelThreads) {
+            int col[8], ps[8];
+            bool act[8];
+            float s[8], r[8];
 #pragma unroll
-        for (int e = 0; e < 8; ++e) {  // positions first: their loads overlap the sums'
-            const int i = i0 + tid + e * kSelThreads;
-            act[e] = i < n;
-            col[e] = !act[e] ? 0 : i < count ? i : B + (i - count);
-            ps[e] = !act[e] ? 0 : i < count ? pos[i] : L + (i - count);
-            r[e] = 0.f;
-        }
-        tiles_sum(part, p.MT, P, col, act, s);
-        if (p.shared) {  // the ranking score: the same sums for every KV head, heads in order
-            for (int h2 = 0; h2 < p.Hkv; ++h2) {
-                float sh[8];
-                tiles_sum(part0 + static_cast<size_t>(h2) * p.MT * P, p.MT, P, col, act, sh);
-#pragma unroll
-                for (int e = 0; e < 8; ++e) r[e] += sh[e];
+            for (int e = 0; e < 8; ++e) {  // positions first: their loads overlap the sums'
+                const int i = i0 + tid + e * kSelThreads;
+                act[e] = i < n;
+                col[e] = !act[e] ? 0 : i < count ? i : B + (i - count);
+                ps[e] = !act[e] ? 0 : i < count ? pos[i] : L + (i - count);
+                r[e] = 0.f;
             }
-        }
+            tiles_sum(part, p.MT, P, col, act, s);
+            if (p.shared) {  // the ranking score: the same sums for every KV head, heads in order
+                for (int h2 = 0; h2 < p.Hkv; ++h2) {
+                    float sh[8];
+                    tiles_sum(part0 + static_cast<size_t>(h2) * p.MT * P, p.MT, P, col, act, sh);
 #pragma unroll
-        for (int e = 0; e < 8; ++e) {
-            if (!act[e]) continue;
-            const int i = i0 + tid + e * kSelThreads;
-            const float rank = p.shared ? r[e] : s[e];
-            key[i] = (static_cast<uint64_t>(__float_as_uint(rank)) << 32) |
-                     static_cast<uint32_t>(0xFFFFFFFFu - static_cast<uint32_t>(ps[e]));
-            if (imp_out) imp_out[col[e]] = s[e];
+                    for (int e = 0; e < 8; ++e) r[e] += sh[e];
+                }
+            }
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+                if (!act[e]) continue;
+                const int i = i0 + tid + e * kSelThreads;
+                const float rank = p.shared ? r[e] : s[e];
+                key[i] = (static_cast<uint64_t>(__float_as_uint(rank)) << 32) |
+                         static_cast<uint32_t>(0xFFFFFFFFu - static_cast<uint32_t>(ps[e]));
+                if (imp_out) imp_out[col[e]] = s[e];
+            }
         }
     }
     if (imp_out)
