@@ -359,6 +359,16 @@ statekv_status statekv_profile_read(statekv_handle* h, statekv_profile* out);
  * DEVICE_FAULT) if a kernel recorded one. */
 statekv_status statekv_sync(statekv_handle* h);
 
+/* Failure-detection self-test.  Enqueues the frame-attention kernel for one
+ * work unit whose producer first waits on a barrier that nothing completes:
+ * the wait expires after the handle's watchdog (watchdog_ms), the kernel
+ * records DEVICE_TIMEOUT in the status word (site 1) and every warp leaves
+ * through its own bounded wait; no input is read and no copy or MMA is
+ * issued.  The handle's status is sticky afterwards, so the next call (e.g.
+ * statekv_sync) returns STATEKV_ERR_DEVICE_TIMEOUT; use a handle made for
+ * the test.  The GPU context stays usable. */
+statekv_status statekv_watchdog_selftest(statekv_handle* h, statekv_stream stream);
+
 /* The raw device status word (0 = none): low byte 1 = an attention-kernel
  * wait expired (bits 8..15 name the waiting site), 2 = the selection kernel
  * found an inconsistent top-B split.  Read without synchronising. */

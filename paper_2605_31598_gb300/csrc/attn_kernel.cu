@@ -83,8 +83,8 @@ struct AttnLayout {
     static constexpr int kOffBar = kOffStat + 5 * kBM * 4;
     // slot_full[6] slot_empty[6] sa_full[6] sa_read[6] sb_full[2] sb_read[2]
     // p_full[2] pv_done[2] q_full o_full drain a_done a_read stage_full stage_free
-    // o_read
-    static constexpr int kNumBars = 40;
+    // o_read stall
+    static constexpr int kNumBars = 41;
     static constexpr int kOffMisc = kOffBar + kNumBars * 8;
     static constexpr int kBytes = kOffMisc + 16;
     static constexpr int kAlloc = kBytes + 1024;  // room to align the base to 1 KB
@@ -159,6 +159,21 @@ __device__ __forceinline__ bool wait_until(uint64_t* bar, uint32_t parity,
 __device__ __forceinline__ void named_bar_sync(int id, int nthreads)
 {
     asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
+}
+
+// Named barrier that also ANDs a predicate over the participating threads.
+__device__ __forceinline__ bool named_bar_and(int id, int nthreads, bool pred)
+{
+    uint32_t r;
+    asm volatile(
+        "{\n\t.reg .pred p, q;\n\t"
+        "setp.ne.u32 p, %1, 0;\n\t"
+        "bar.red.and.pred q, %2, %3, p;\n\t"
+        "selp.u32 %0, 1, 0, q;\n\t}"
+        : "=r"(r)
+        : "r"(pred ? 1u : 0u), "r"(id), "r"(nthreads)
+        : "memory");
+    return r != 0;
 }
 
 // One MMA group, D[d] (+)= A[a + 8k (+ kGapA when k >= NK/2)] * B_k for k < NK
@@ -348,6 +363,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t* stage_full = bars + 37;  // pass B: the tile's column sums are staged
     uint64_t* stage_free = bars + 38;  // pass B: the reducer warp has read them
     uint64_t* o_read = bars + 39;   // per unit: O has been read out of TMEM
+    uint64_t* stall = bars + 40;    // watchdog self-test: never completed
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + L::kOffMisc);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(sm + L::kOffMisc + 4);
 
@@ -365,7 +381,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int mt = w % p.MT, r = w / p.MT, hkv = r % p.Hkv, u = r / p.Hkv;
         const int tq = static_cast<int>(threadIdx.x) - 128;
         const int qwg = tq >> 7, qrow = tq & 127, qr = mt * kBM + qrow;
-        const bool loads = w < W && tq >= 0 && qwg * 64 < D && qr < rows;
+        const bool loads = p.q != nullptr && w < W && tq >= 0 && qwg * 64 < D && qr < rows;
         const int t = loads ? qr / G : 0, g = loads ? qr - t * G : 0;
         const uint4* src = reinterpret_cast<const uint4*>(
             p.q + ((static_cast<size_t>(loads ? u : 0) * T + t) * p.Hq + (loads ? hkv : 0) * G + g) * D +
@@ -399,6 +415,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_init(o_read, 256);
         mbar_init(drain, 2);   // one commit per MMA issuer
         mbar_init(a_done, 2);
+        mbar_init(stall, 1);
         *abort_flag = 0;
         fence_mbar_init();
     }
@@ -434,6 +451,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                 for (int sl = 0; sl < kSlots; ++sl) last_use[sl] = -1;
                 bool ok = true;
+                if (p.selftest_stall && !wait_until(stall, 0, globaltimer() + p.watchdog_ns)) {
+                    fail(1);
+                    ok = false;
+                }
                 int n = 0;  // global item
                 for (int w = w0; ok && w < W; w += wstep) {
                     const WorkUnit x = work_unit(p, w);
@@ -784,11 +805,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             }
             if (it0 >= x.nt) mbar_arrive(a_read);  // a warpgroup without pass-A tiles
-            if (!ok) break;
+            if (ok) {
+                stat[(wg * 2 + 0) * kBM + row] = m;
+                stat[(wg * 2 + 1) * kBM + row] = l;
+            }
+            // Both warpgroups reach this barrier even after an expired wait (the
+            // other may have no pass-A tile left to wait on), and leave together
+            // if either timed out, so neither is stranded at the barrier below.
+            if (!named_bar_and(1, 256, ok)) {
+                ok = false;
+                break;
+            }
             site = 11;
-            stat[(wg * 2 + 0) * kBM + row] = m;
-            stat[(wg * 2 + 1) * kBM + row] = l;
-            named_bar_sync(1, 256);
             float nlse;  // -log2-sum-exp of this row (scaled); -inf for padding rows
             {
                 const float m0 = stat[0 * kBM + row], l0 = stat[1 * kBM + row];

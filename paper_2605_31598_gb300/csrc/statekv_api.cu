@@ -1054,6 +1054,34 @@ statekv_status statekv_prefill_frames_host(statekv_handle* h, const statekv_fram
     return STATEKV_OK;
 }
 
+statekv_status statekv_watchdog_selftest(statekv_handle* h, statekv_stream stream)
+{
+    if (!h) return STATEKV_ERR_INVALID_ARG;
+    const statekv_config& c = h->cfg;
+    // One work unit (stream 0, layer 0) whose producer first waits on a barrier
+    // that nothing completes: no input is read, no copy or MMA is issued, and
+    // every role of the CTA leaves through its bounded waits.
+    AttnParams pa{};
+    pa.counts = h->at<int32_t>(h->lay.counts);
+    pa.status = h->status_dev;
+    pa.units = UnitRange{0, 0, 1, c.num_layers};
+    pa.T = c.tokens_per_frame;
+    pa.Hq = c.num_q_heads;
+    pa.Hkv = c.num_kv_heads;
+    pa.G = h->d.G;
+    pa.B = c.state_capacity;
+    pa.P = h->d.P;
+    pa.MT = h->d.MT;
+    pa.causal = c.causal_in_frame;
+    pa.count_mul = 1;
+    pa.scale_log2 = h->d.scale * 1.4426950408889634f;
+    pa.watchdog_ns = 1000000ull * (c.watchdog_ms ? c.watchdog_ms : 2000u);
+    pa.selftest_stall = 1;
+    const cudaError_t e = launch_attn(c.head_dim, h->tm_sk, h->tm_sv, h->tm_sk, h->tm_sv, pa, 1,
+                                      reinterpret_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? STATEKV_OK : STATEKV_ERR_CUDA;
+}
+
 statekv_status statekv_state_view(const statekv_handle* h, int32_t stream, int32_t layer,
                                   statekv_state_info* out)
 {

@@ -17,7 +17,8 @@ namespace statekv {
 
 // Device error codes written to the status word (0 = no error).  The low
 // byte is the kind; an attention-kernel timeout carries the waiting site in
-// bits 8..15 (the first expired wait of the CTA): 2 producer (free slot),
+// bits 8..15 (the first expired wait of the CTA): 1 the watchdog self-test's
+// barrier (see AttnParams::selftest_stall), 2 producer (free slot),
 // 4..9 MMA issuer X (4 Q ready, 5 K tile landed, 6 score buffer free, 7 P
 // written, 8 V tile landed, 9 pass A done and read; +16 for issuer Y),
 // 10..12 and 14 softmax warpgroup 0 (10 Q K^T in pass A, 11 pass-B scores
@@ -56,6 +57,10 @@ struct AttnParams {
     int count_mul;            // 1: counts are state sizes; T: counts are frame counters
     float scale_log2;         // softmax scale * log2(e)
     unsigned long long watchdog_ns;
+    // Watchdog self-test: 1 makes the producer wait first on a barrier that
+    // nothing completes, so its bounded wait expires and the CTA aborts
+    // through the regular timeout path (no copy or MMA is issued).
+    int selftest_stall;
 };
 
 struct SelectParams {

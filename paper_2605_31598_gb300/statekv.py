@@ -26,7 +26,7 @@ EXPORTED = ("statekv_arena_bytes", "statekv_init", "statekv_prefill_frame",
             "statekv_full_attention_frame", "statekv_decode_step",
             "statekv_state_view", "statekv_cache_view",
             "statekv_profile_enable", "statekv_profile_read", "statekv_sync",
-            "statekv_device_error", "statekv_frame_attention_noalloc",
+            "statekv_device_error", "statekv_watchdog_selftest", "statekv_frame_attention_noalloc",
             "statekv_scores_workspace_bytes", "statekv_full_attention_scores",
             "statekv_topb_mask", "statekv_concentration_sums", "statekv_state_metrics",
             "statekv_block_workspace_bytes", "statekv_block_frame",
@@ -115,6 +115,8 @@ def lib() -> ctypes.CDLL:
             L.statekv_prefill_frames_host.argtypes = [ctypes.c_void_p, P(statekv_frame_args),
                                                       ctypes.c_int32, ctypes.c_void_p]
             L.statekv_prefill_frames_host.restype = st
+            L.statekv_watchdog_selftest.argtypes = [ctypes.c_void_p, ctypes.c_void_p]
+            L.statekv_watchdog_selftest.restype = st
             L.statekv_decode_step.argtypes = [ctypes.c_void_p, P(statekv_decode_args),
                                               ctypes.c_void_p]
             L.statekv_decode_step.restype = st
@@ -536,3 +538,12 @@ class StateKV:
     def device_error(self) -> int:
         """Raw device status word (0 = none); see statekv_device_error."""
         return statekv_device_error(self.handle)
+
+    def watchdog_selftest(self, stream=None) -> int:
+        """Enqueue the failure-detection self-test (statekv_watchdog_selftest):
+        the attention kernel's bounded wait on a barrier nothing completes
+        expires, and the handle reports DEVICE_TIMEOUT from then on."""
+        import torch
+
+        st = (stream or torch.cuda.current_stream()).cuda_stream
+        return lib().statekv_watchdog_selftest(self.handle, ctypes.c_void_p(st))

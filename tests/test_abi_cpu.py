@@ -99,6 +99,7 @@ def test_null_arguments_rejected(lib):
     assert lib.statekv_init(ctypes.byref(_cfg()), None, 1 << 30, ctypes.byref(h)) == 1
     assert lib.statekv_prefill_frame(None, None, None) == 1
     assert lib.statekv_prefill_frames_host(None, None, 0, None) == 1
+    assert lib.statekv_watchdog_selftest(None, None) == 1
     assert lib.statekv_state_view(None, 0, 0, None) == 1
     assert lib.statekv_cache_view(None, 0, 0, None) == 1
     lib.statekv_destroy(None)
