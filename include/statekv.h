@@ -361,8 +361,9 @@ statekv_status statekv_sync(statekv_handle* h);
 
 /* Failure-detection self-test.  Enqueues the frame-attention kernel for one
  * work unit whose producer first waits on a barrier that nothing completes:
- * the wait expires after the handle's watchdog (watchdog_ms), the kernel
- * records DEVICE_TIMEOUT in the status word (site 1) and every warp leaves
+ * the wait expires after half the handle's watchdog (watchdog_ms), before
+ * any other wait can, the kernel records DEVICE_TIMEOUT in the status word
+ * (site 1) and every warp leaves
  * through its own bounded wait; no input is read and no copy or MMA is
  * issued.  The handle's status is sticky afterwards, so the next call (e.g.
  * statekv_sync) returns STATEKV_ERR_DEVICE_TIMEOUT; use a handle made for
