@@ -513,6 +513,8 @@ def run_curve(args, local):
     device = torch.device("cuda", local)
     torch.cuda.set_device(device)
     shape = WORKLOADS[args.workload]
+    if args.capacity is not None:  # the paper's wall-time sweep varies the state capacity
+        shape = dataclasses.replace(shape, state_capacity=args.capacity)
     S, L, T, B = shape.num_streams, shape.num_layers, shape.tokens_per_frame, shape.state_capacity
     N = args.frames or shape.max_frames
     shape = dataclasses.replace(shape, max_frames=max(N, shape.max_frames))
@@ -566,6 +568,7 @@ def run_curve(args, local):
 
     line = {
         "curve": WORKLOAD_TEXT[args.workload],
+        "state_capacity": B,
         "frames": N,
         "streams": S,
         "layers": L,
@@ -855,6 +858,8 @@ def main():
                     help="per-frame cost vs frame index, StateKV next to exact full attention")
     ap.add_argument("--frames", type=int, default=0, help="--curve: frames to run (default: "
                     "the workload's video length)")
+    ap.add_argument("--capacity", type=int, default=None,
+                    help="--curve: state capacity B in tokens (default: the workload's)")
     ap.add_argument("--decode", action="store_true",
                     help="decoding over the detailed cache after --frames video frames")
     ap.add_argument("--prompt", type=int, default=64, help="--decode: prompt tokens")
