@@ -72,14 +72,61 @@ def test_yarn_frequencies():
     np.testing.assert_array_equal(f1, plain)  # factor 1: plain RoPE
     assert m1 == 1.0
     f, m = ob.rope_frequencies(d, theta, s, L)
-    assert m == pytest.approx(0.1 * np.log(s) + 1.0)
     r = L * plain / (2 * np.pi)  # trained context over wavelength
     np.testing.assert_allclose(f[r < 1.0], plain[r < 1.0] / s)   # long wavelengths: interpolated
     np.testing.assert_allclose(f[r > 32.0], plain[r > 32.0])     # short ones: kept
-    mid = (r > 1.0) & (r < 32.0)
-    assert mid.any()
-    g = (r[mid] - 1.0) / 31.0
-    np.testing.assert_allclose(f[mid], (1 - g) * plain[mid] / s + g * plain[mid])
+    assert ((r > 1.0) & (r < 32.0)).any()
+
+
+def test_yarn_mid_ramp_frequency_hand_value():
+    """YaRN's blend at a hand-chosen ramp point (d 4, theta 1e4, s 4).
+
+    Pair 0 has frequency 1 (wavelength 2 pi) and pair 1 frequency
+    1e4^(-1/2) = 0.01 (wavelength 200 pi).  With a trained context of
+    L = 1750 pi, pair 1 sees r = L / (200 pi) = 8.75, a quarter of the way up
+    the ramp from r = 1 to r = 32: gamma = (8.75 - 1) / 31 = 0.25, so its
+    frequency is 0.75 * 0.01 / 4 + 0.25 * 0.01 = 0.004375 (the blend's weights
+    swapped would give 0.008125).  Pair 0 sees r = 875 > 32 and keeps
+    frequency 1.  The q/k factor is 0.1 ln 4 + 1 = 1.138629436111989.
+    """
+    f, m = ob.rope_frequencies(4, 1e4, 4.0, 1750 * np.pi)
+    np.testing.assert_allclose(f, [1.0, 0.004375], rtol=1e-12)
+    assert m == pytest.approx(1.138629436111989, rel=1e-14)
+    # just below the ramp (r = 0.5 for pair 1): fully interpolated, 0.01 / 4
+    f, _ = ob.rope_frequencies(4, 1e4, 4.0, 100 * np.pi)
+    np.testing.assert_allclose(f, [1.0, 0.0025], rtol=1e-12)
+
+
+def test_yarn_factor_scales_both_q_and_k():
+    """The attention factor multiplies q and k alike, so the scale of a q.k
+    logit grows by (0.1 ln s + 1)^2 = 1.2964769927807063 at s = 4 (a factor
+    applied to one of them only would give 1.1386); and the attention of the
+    step consumes the scaled q and k.  Checked at position 0, where the rotation is the
+    identity for every frequency, against the same layer without scaling."""
+    rng = np.random.default_rng(11)
+    hidden, inter, n_q, n_kv, d, T = 64, 32, 1, 1, 64, 2
+    w = _weights(rng, hidden, inter, n_q, n_kv, d)
+    x = ob.round_bf16(rng.standard_normal((T, hidden)))
+    plain = ob.OracleBlock(n_q, n_kv, d, T, 8, 2, [w], theta=1e4)
+    yarn = ob.OracleBlock(n_q, n_kv, d, T, 8, 2, [w], theta=1e4, yarn_factor=4.0,
+                          original_max=64)
+    _, a = plain.layer_frame(0, x)
+    _, b = yarn.layer_frame(0, x)
+    q0a, k0a, q0b, k0b = a["q"][0, 0], a["k"][0, 0], b["q"][0, 0], b["k"][0, 0]
+    # each side carries the factor once (bf16 rounding: a few parts in 1e3)
+    np.testing.assert_allclose(np.dot(q0b, q0a) / np.dot(q0a, q0a), 1.138629436111989, rtol=8e-3)
+    np.testing.assert_allclose(np.dot(k0b, k0a) / np.dot(k0a, k0a), 1.138629436111989, rtol=8e-3)
+    # so the logit scale, |q| |k|, grows by the square
+    np.testing.assert_allclose(np.linalg.norm(q0b) * np.linalg.norm(k0b) /
+                               (np.linalg.norm(q0a) * np.linalg.norm(k0a)), 1.2964769927807063,
+                               rtol=8e-3)
+    # the step attends with them: key 0's importance is 1 (query 0 sees only
+    # it) plus its softmax weight for query 1
+    q1, k0, k1 = b["q"][1, 0], b["k"][0, 0], b["k"][1, 0]
+    z = np.array([np.dot(q1, k0), np.dot(q1, k1)]) / np.sqrt(d)
+    w0 = 1.0 / (1.0 + np.exp(z[1] - z[0]))
+    np.testing.assert_allclose(b["imp"][0, 8], 1.0 + w0, rtol=1e-12)
+    np.testing.assert_allclose(b["imp"][0, 9], 1.0 - w0, rtol=1e-12)
 
 
 def _weights(rng, hidden, inter, n_q, n_kv, d, zero_out=False):
