@@ -18,7 +18,6 @@ import hashlib
 import json
 import math
 import os
-import re
 import statistics
 import subprocess
 import sys
@@ -42,7 +41,18 @@ WORKLOAD_TEXT = {
     "toy": "toy layer: 4 q / 1 kv heads, head_dim 64, 16 tokens/frame, state capacity 32",
 }
 KERNEL_SOURCE = os.path.join(ROOT, "paper_2605_31598_gb300", "csrc", "attn_kernel.cu")
-TRAFFIC_FILE = os.path.join(ROOT, "profiles", "frame_attn_qwen7b_stack.md")
+# DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) of one attention
+# launch, from one ncu capture per workload, keyed by the workload and the
+# first 16 hex digits of the sha256 of the attention-kernel source it was taken
+# on.  A workload or kernel source with no capture reports null.
+K1_DRAM_BYTES = {
+    ("qwen7b_stack", "a7a9ed44211fd1b8"): 199170304,
+}
+
+
+FLATNESS_MIN_FRAMES = 64
+# --curve generates inputs in chunks of at most this many bytes
+CURVE_CHUNK_BYTES = 24e9
 
 
 def log(*a):
@@ -71,17 +81,10 @@ def kernel_source_hash():
         return hashlib.sha256(f.read()).hexdigest()[:16]
 
 
-def recorded_traffic():
-    """DRAM bytes per attention launch from the committed ncu summary, or None
-    if the summary is missing or was taken on a different kernel source."""
-    if not os.path.exists(TRAFFIC_FILE):
-        return None
-    txt = open(TRAFFIC_FILE).read()
-    m = re.search(r"dram_bytes_per_full_launch:\s*([0-9.eE+]+)", txt)
-    h = re.search(r"kernel_source_sha256_16:\s*([0-9a-f]+)", txt)
-    if not m or not h or h.group(1) != kernel_source_hash():
-        return None
-    return float(m.group(1))
+def recorded_traffic(workload):
+    """DRAM bytes per attention launch captured for this workload on the
+    current kernel source, or None."""
+    return K1_DRAM_BYTES.get((workload, kernel_source_hash()))
 
 
 class ClockSampler:
@@ -116,11 +119,11 @@ class ClockSampler:
             except subprocess.TimeoutExpired:
                 self.proc.kill()
 
-    def summary(self, t0, t1):
+    def summary(self, t0, t1, pad=0.3):
         if not self.samples:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no nvidia-smi samples"],
                     "samples": 0}
-        win = [s for (t, s) in self.samples if t0 - 0.3 <= t <= t1 + 0.3]
+        win = [s for (t, s) in self.samples if t0 - pad <= t <= t1 + pad]
         if not win:  # timed region shorter than the sampling period: nearest samples
             mid = 0.5 * (t0 + t1)
             win = [min(self.samples, key=lambda x: abs(x[0] - mid))[1]]
@@ -134,6 +137,15 @@ class ClockSampler:
                 "samples": len(win),
                 "power_w_max": max((float(s[2]) for s in win
                                     if s[2].replace(".", "").isdigit()), default=None)}
+
+
+def gpu_sampler(device):
+    """A clock sampler on the GPU behind ``device`` (by UUID when torch knows it)."""
+    import torch
+
+    props = torch.cuda.get_device_properties(device)
+    gpu_id = f"GPU-{props.uuid}" if getattr(props, "uuid", None) else str(device.index or 0)
+    return ClockSampler(gpu_id)
 
 
 def dist_setup():
@@ -310,9 +322,7 @@ def run_ours(args, world, rank, local):
         step(n)
     torch.cuda.synchronize()
 
-    props = torch.cuda.get_device_properties(device)
-    gpu_id = f"GPU-{props.uuid}" if getattr(props, "uuid", None) else str(local)
-    sampler = ClockSampler(gpu_id)
+    sampler = gpu_sampler(device)
     time.sleep(0.3)
     st = torch.cuda.current_stream()
     starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
@@ -343,7 +353,7 @@ def run_ours(args, world, rank, local):
     k1_avg_s = k1_ms / max(k1_launches, 1) * 1e-3
     flops = S * L * attn_flops(shape, B)
     achieved = flops / k1_avg_s / 1e12
-    traffic = recorded_traffic()
+    traffic = recorded_traffic(args.workload)
     a_launches, a_ms = prof[0]
     s_launches, s_ms = prof[2]
     d = shape.head_dim
@@ -373,10 +383,15 @@ def run_ours(args, world, rank, local):
     slope = sum((x - mx) * (y - my) for x, y in zip(idx, per_step)) / var if var > 0 else 0.0
     early = sorted(per_step[:32])
     late = sorted(per_step[n // 2:])
+    # a per-100-frame slope needs a window of comparable length to mean anything
     flatness = {"frames": f"{first}..{first + n - 1}",
-                "slope_pct_per_100_frames": 100.0 * 100.0 * slope / my if my > 0 else None,
+                "slope_pct_per_100_frames": (100.0 * 100.0 * slope / my
+                                             if my > 0 and n >= FLATNESS_MIN_FRAMES else None),
                 "p50_first32_us": 1e3 * early[len(early) // 2],
                 "p50_last_half_us": 1e3 * late[len(late) // 2]}
+    if n < FLATNESS_MIN_FRAMES:
+        flatness["note"] = (f"slope omitted: {n} timed frames (< {FLATNESS_MIN_FRAMES}); "
+                            "bench.py --curve measures the per-frame cost over whole videos")
     line = {
         "metric": METRIC,
         "value": value,
@@ -497,11 +512,15 @@ def run_curve(args, local):
     self-attention (Sec. 4.1's comparison, App. B's protocol: given the
     preceding cache, process one more frame).
 
-    Every frame 1..N runs statekv_prefill_frame (timed with CUDA events; the
-    frame's inputs are generated beforehand, outside the timed region).  At
-    sample frames statekv_full_attention_frame first runs on the same handle,
-    over the decode cache that the earlier frames filled, and is timed the
-    same way.  Prints one JSON line.
+    The frames' inputs are generated in chunks that fit in HBM, outside any
+    timed region; the frames of a chunk then run back to back, each
+    statekv_prefill_frame bracketed by CUDA events, so the GPU stays busy and
+    the clocks sampled meanwhile are those of the timed work.  At sample
+    frames statekv_full_attention_frame first runs on the same handle, over
+    the decode cache that the earlier frames filled (twice; the second run is
+    timed).  nvidia-smi clocks are sampled throughout; every 32-frame bin and
+    every sample frame reports the median SM clock of the samples taken while
+    it ran (the nearest sample when none fell inside).  Prints one JSON line.
     """
     import torch
 
@@ -516,39 +535,66 @@ def run_curve(args, local):
     if args.capacity is not None:  # the paper's wall-time sweep varies the state capacity
         shape = dataclasses.replace(shape, state_capacity=args.capacity)
     S, L, T, B = shape.num_streams, shape.num_layers, shape.tokens_per_frame, shape.state_capacity
+    Hq, Hkv, d = shape.num_q_heads, shape.num_kv_heads, shape.head_dim
     N = args.frames or shape.max_frames
     shape = dataclasses.replace(shape, max_frames=max(N, shape.max_frames))
     samples = sorted({n for n in (1, 2, 4, 8, 16, 32, 64, 96, 128, 192, 256, 384, 512, 640, 768,
                                   896, 1024) if n <= N} | {N})
+    frame_bytes = S * L * T * (Hq + 2 * Hkv) * d * 2
+    chunk = max(1, min(N, int(CURVE_CHUNK_BYTES // frame_bytes)))
     eng = StateKV(make_config(shape))
     st = torch.cuda.current_stream()
     out = None
-    step_ms, full_ms = [], {}
-    log(f"[curve] {args.workload}: {N} frames, full attention at {samples}")
-    for n in range(1, N + 1):
-        q, k, v = batch_qkv(shape, n, streams=range(S), layers=range(L), seed=args.seed,
-                            device=device)
+    step_ms, full_ms, wall = [0.0] * N, {}, [(0.0, 0.0)] * N
+    full_wall = {}
+    log(f"[curve] {args.workload}: {N} frames in chunks of {chunk}, full attention at {samples}")
+    sampler = gpu_sampler(device)
+    time.sleep(0.3)
+    t_all0 = time.time()
+    ev = lambda: torch.cuda.Event(enable_timing=True)
+    for c0 in range(1, N + 1, chunk):
+        c1 = min(N, c0 + chunk - 1)
+        frames = [batch_qkv(shape, n, streams=range(S), layers=range(L), seed=args.seed,
+                            device=device) for n in range(c0, c1 + 1)]
         if out is None:
-            out = torch.empty_like(q)
+            out = torch.empty_like(frames[0][0])
         torch.cuda.synchronize()
-        if n in samples:
-            for rep in range(2):  # second run timed: code and TMA descriptors warm
-                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-                e0.record(st)
-                rc = eng.full_attention_frame(q, k, v, out)
-                e1.record(st)
-                if rc != 0:
-                    raise RuntimeError(f"statekv_full_attention_frame returned {rc} at frame {n}")
-            torch.cuda.synchronize()
-            full_ms[n] = e0.elapsed_time(e1)
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record(st)
-        rc = eng.prefill_frame(q, k, v, out)
-        e1.record(st)
-        if rc != 0:
-            raise RuntimeError(f"statekv_prefill_frame returned {rc} at frame {n}")
+        base = ev()
+        marks = []
+        t0 = time.time()
+        base.record(st)
+        for n in range(c0, c1 + 1):
+            q, k, v = frames[n - c0]
+            fm = None
+            if n in samples:
+                for rep in range(2):  # second run timed: code and TMA descriptors warm
+                    f0, f1 = ev(), ev()
+                    f0.record(st)
+                    rc = eng.full_attention_frame(q, k, v, out)
+                    f1.record(st)
+                    if rc != 0:
+                        raise RuntimeError(f"statekv_full_attention_frame returned {rc} at frame {n}")
+                fm = (f0, f1)
+            e0, e1 = ev(), ev()
+            e0.record(st)
+            rc = eng.prefill_frame(q, k, v, out)
+            e1.record(st)
+            if rc != 0:
+                raise RuntimeError(f"statekv_prefill_frame returned {rc} at frame {n}")
+            marks.append((n, e0, e1, fm))
         torch.cuda.synchronize()
-        step_ms.append(e0.elapsed_time(e1))
+        for n, e0, e1, fm in marks:
+            step_ms[n - 1] = e0.elapsed_time(e1)
+            # wall-clock window of the frame: the chunk's start plus its GPU offset
+            wall[n - 1] = (t0 + 1e-3 * base.elapsed_time(e0), t0 + 1e-3 * base.elapsed_time(e1))
+            if fm is not None:
+                full_ms[n] = fm[0].elapsed_time(fm[1])
+                full_wall[n] = (t0 + 1e-3 * base.elapsed_time(fm[0]),
+                                t0 + 1e-3 * base.elapsed_time(fm[1]))
+        del frames, marks
+    t_all1 = time.time()
+    time.sleep(0.3)
+    sampler.stop()
     assert eng.sync() == 0
     fill = math.ceil(B / T) if B > 0 else 0
     post = step_ms[fill + 1:]  # frames whose pool exceeds B
@@ -559,6 +605,7 @@ def run_curve(args, local):
     var = sum((x - mx) ** 2 for x in idx)
     slope = sum((x - mx) * (y - my) for x, y in zip(idx, post)) / var if var > 0 else 0.0
     p50 = lambda xs: sorted(xs)[len(xs) // 2]
+    clk = lambda w: sampler.summary(w[0], w[1], pad=0.0)["sm_mhz"]
 
     def pairs(n):  # visible (query, key) pairs per query head
         return T * (n - 1) * T + T * (T + 1) / 2
@@ -566,14 +613,23 @@ def run_curve(args, local):
     def pairs_statekv(n):
         return T * min(B, (n - 1) * T) + T * (T + 1) / 2
 
+    bins = []
+    for b0 in range(1, N + 1, 32):
+        b1 = min(N, b0 + 31)
+        bins.append({"frames": f"{b0}..{b1}",
+                     "p50_us": 1e3 * p50(step_ms[b0 - 1:b1]),
+                     "sm_mhz": clk((wall[b0 - 1][0], wall[b1 - 1][1]))})
     line = {
         "curve": WORKLOAD_TEXT[args.workload],
         "state_capacity": B,
         "frames": N,
         "streams": S,
         "layers": L,
+        "input_chunk_frames": chunk,
         "statekv_step_us_at": {str(n): 1e3 * step_ms[n - 1] for n in samples},
+        "statekv_sm_mhz_at": {str(n): clk(wall[n - 1]) for n in samples},
         "full_attention_us_at": {str(n): 1e3 * full_ms[n] for n in samples},
+        "full_attention_sm_mhz_at": {str(n): clk(full_wall[n]) for n in samples},
         "full_over_statekv_flops_at": {str(n): pairs(n) / pairs_statekv(n) for n in samples},
         "statekv_flatness": {
             "frames": f"{first}..{first + m - 1}",
@@ -582,8 +638,12 @@ def run_curve(args, local):
             "slope_pct_per_100_frames": 100.0 * 100.0 * slope / my if my > 0 else None,
             "p50_all_us": 1e3 * p50(post),
         },
+        "statekv_bins_of_32": bins,
+        "clocks": sampler.summary(t_all0, t_all1),
         "note": "full attention = the attention call alone (the decode-cache append it also "
-                "needs is the same as StateKV's and not included); StateKV = the whole step",
+                "needs is the same as StateKV's and not included); StateKV = the whole step; "
+                "sm_mhz = median nvidia-smi SM clock while the frames ran (nearest sample "
+                "when none fell inside)",
     }
     print(json.dumps(line), flush=True)
 
@@ -624,24 +684,33 @@ def run_decode(args, local):
         return mk(Hq), mk(Hkv), mk(Hkv)
 
     st = torch.cuda.current_stream()
+    sampler = gpu_sampler(device)
+    time.sleep(0.3)
 
-    def timed(n):
-        q, k, v = tokens(n)
-        o = torch.empty_like(q)
+    def timed(batch):
+        """Runs decode steps back to back (inputs made beforehand), each
+        bracketed by CUDA events; returns their times in ms and the wall
+        window of the run."""
+        outs = [torch.empty_like(q) for q, _, _ in batch]
         torch.cuda.synchronize()
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record(st)
-        rc = eng.decode_step(q, k, v, o)
-        e1.record(st)
-        if rc != 0:
-            raise RuntimeError(f"statekv_decode_step returned {rc}")
+        evs = []
+        t0 = time.time()
+        for (q, k, v), o in zip(batch, outs):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(st)
+            rc = eng.decode_step(q, k, v, o)
+            e1.record(st)
+            if rc != 0:
+                raise RuntimeError(f"statekv_decode_step returned {rc}")
+            evs.append((e0, e1))
         torch.cuda.synchronize()
-        return e0.elapsed_time(e1)
+        return [a.elapsed_time(b) for a, b in evs], (t0, time.time())
 
-    prompt_ms = timed(args.prompt)
-    for _ in range(3):  # warm-up single-token steps
-        timed(1)
-    tok_ms = sorted(timed(1) for _ in range(steps))
+    (prompt_ms,), _ = timed([tokens(args.prompt)])
+    timed([tokens(1) for _ in range(3)])  # warm-up single-token steps
+    tok, win = timed([tokens(1) for _ in range(steps)])
+    tok_ms = sorted(tok)
+    sampler.stop()
     assert eng.sync() == 0
     rows = N * T + args.prompt + 3 + steps // 2
     cache_bytes = S * L * Hkv * rows * d * 2 * 2  # K and V read once per token
@@ -655,6 +724,8 @@ def run_decode(args, local):
         "token_p50_us": 1e3 * p50,
         "tokens_per_s": 1e3 / p50,
         "kv_read_gbs_at_p50": cache_bytes / (p50 * 1e-3) / 1e9,
+        "kv_read_frac_of_hbm_at_p50": cache_bytes / (p50 * 1e-3) / 1e9 / peaks()[0],
+        "clocks": sampler.summary(*win),
         "note": "one call = every (stream, layer); single tokens (<= 16 query rows per KV head) "
                 "run the one-pass split-K decode kernel, which reads each K and V row once; the "
                 "prompt runs the two-pass attention kernel",
@@ -786,13 +857,18 @@ def run_block(args, local):
         if eng.block_frame(bc, warr, xs[n], y, ws) != 0:
             raise RuntimeError(f"statekv_block_frame failed at frame {n + 1}")
     torch.cuda.synchronize()
+    sampler = gpu_sampler(device)
+    time.sleep(0.3)
     eng.profile(True)
+    t0 = time.time()
     for i in range(steps):
         starts[i].record(st)
         if eng.block_frame(bc, warr, xs[fill + args.warmup + i], y, ws) != 0:
             raise RuntimeError("statekv_block_frame failed")
         ends[i].record(st)
     torch.cuda.synchronize()
+    t1 = time.time()
+    sampler.stop()
     prof = eng.profile_read()
     eng.profile(False)
     assert eng.sync() == 0
@@ -819,6 +895,7 @@ def run_block(args, local):
         "gemm_weight_read_frac_of_hbm": weight_bytes / (per(3) * 1e-3) / 1e9 / hbm,
         "gemm_tflops": gemm_flops / (per(3) * 1e-3) / 1e12,
         "attention_tflops": attn_flops / (per(1) * 1e-3) / 1e12,
+        "clocks": sampler.summary(t0, t1),
         "note": "layers run in sequence (layer l+1 reads layer l's output); at one stream the "
                 "projections read every weight once per frame for 196 rows, so they are "
                 "bound by HBM bandwidth, not by the tensor cores",

@@ -388,7 +388,12 @@ statekv_status statekv_device_error(const statekv_handle* h, int32_t* code);
  * allocates nothing.  Its first call on a device looks up the arrays' device
  * addresses; make that first call before any stream capture.  Calls share the
  * scratch: calls that overlap on the GPU race.  The call synchronises `stream`
- * before it returns and reports its own DEVICE_TIMEOUT.
+ * before it returns and reports its own DEVICE_TIMEOUT, so `stream` must not
+ * be under capture (STATEKV_ERR_INVALID_ARG, nothing enqueued); while another
+ * component captures, pass a cudaStreamNonBlocking stream, since a blocking
+ * stream (the legacy default stream among them) synchronises implicitly with
+ * the capturing one and so invalidates that capture.  T above 4096, more than
+ * 64 KV heads or G * T above 2^31 - 1 also return STATEKV_ERR_UNSUPPORTED.
  *   cfg           num_q_heads, num_kv_heads, head_dim, tokens_per_frame,
  *                 state_capacity (B), causal_in_frame, softmax_scale,
  *                 watchdog_ms are used; the rest is ignored

@@ -959,7 +959,17 @@ __global__ void __launch_bounds__(kThreads, 1)
 constexpr int kLaunchRegs = 168;
 static_assert(128 * 96 + 256 * 200 <= kThreads * kLaunchRegs, "register split");
 
-int g_num_sms = 0;  // SMs of the device, read once by attn_prepare
+// SMs of each device, read by attn_prepare with that device current; the
+// persistent grid of a launch is sized for the device current at the launch.
+constexpr int kMaxDevices = 64;
+int g_num_sms[kMaxDevices] = {};
+
+int current_device_sms()
+{
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return 1;
+    return g_num_sms[dev] > 0 ? g_num_sms[dev] : 1;
+}
 
 template <int D>
 cudaError_t prepare_one()
@@ -968,10 +978,12 @@ cudaError_t prepare_one()
     cudaError_t e = cudaFuncGetAttributes(&fa, frame_attn_lse_importance<D>);
     if (e != cudaSuccess) return e;
     if (fa.numRegs < kLaunchRegs) return cudaErrorInvalidConfiguration;
-    int dev = 0;
+    int dev = 0, sms = 0;
     if ((e = cudaGetDevice(&dev)) != cudaSuccess ||
-        (e = cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
+        (e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
         return e;
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    g_num_sms[dev] = sms;
     return cudaFuncSetAttribute(frame_attn_lse_importance<D>,
                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 AttnLayout<D>::kAlloc);
@@ -987,7 +999,7 @@ cudaError_t launch_one(const CUtensorMap& tm_sk, const CUtensorMap& tm_sv, const
     const long long W = static_cast<long long>(p.MT) * p.Hkv * U;
     if (W <= 0) return cudaSuccess;
     if (W > 0x7FFFFFFFll) return cudaErrorInvalidValue;
-    const int sms = g_num_sms > 0 ? g_num_sms : 1;
+    const int sms = current_device_sms();
     const int grid = static_cast<int>(W < sms ? W : sms);
     frame_attn_lse_importance<D><<<grid, kThreads, AttnLayout<D>::kAlloc, st>>>(tm_sk, tm_sv, tm_fk,
                                                                               tm_fv, p);
@@ -996,7 +1008,7 @@ cudaError_t launch_one(const CUtensorMap& tm_sk, const CUtensorMap& tm_sv, const
 
 }  // namespace
 
-int device_sm_count() { return g_num_sms > 0 ? g_num_sms : 1; }
+int device_sm_count() { return current_device_sms(); }
 
 size_t attn_smem_bytes(int D)
 {

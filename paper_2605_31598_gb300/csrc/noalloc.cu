@@ -19,12 +19,15 @@
 // contents: the counts and the status word are rewritten at the start of
 // each call, and the kernels write every partial they later read.  Calls that
 // overlap on the GPU (different streams or threads, no ordering) race on the
-// scratch.  Each call synchronises its stream before returning.
+// scratch.  Each call synchronises its stream before returning, so the stream
+// must not be under capture (refused), and a caller that runs while another
+// component captures should pass a cudaStreamNonBlocking stream: a blocking
+// stream, the legacy default stream among them, synchronises implicitly with
+// the capturing stream, which invalidates that capture.
 #include "../../include/statekv.h"
 #include "statekv_kernels.cuh"
 
 #include <cuda.h>
-#include <cudaTypedefs.h>
 #include <cuda_runtime.h>
 
 #include <cmath>
@@ -101,33 +104,16 @@ __global__ void noalloc_importance(const float* __restrict__ partials, float* __
     }
 }
 
-PFN_cuTensorMapEncodeTiled_v12000 noalloc_encode_fn()
-{
-    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-    static std::once_flag once;
-    std::call_once(once, [] {
-        void* p = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000,
-                                             cudaEnableDefault, &q) == cudaSuccess &&
-            q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
-    });
-    return fn;
-}
-
+// The frame's K or V ([T][Hkv][D]: boxes of one head x 128 tokens) or the
+// state's ([Hkv][B][D]: boxes of 128 slots of one head), as the handle path
+// maps them for one (stream, layer).
 bool noalloc_map(CUtensorMap* m, const void* base, cuuint64_t d0, cuuint64_t d1, cuuint64_t d2,
                  cuuint32_t b1, cuuint32_t b2)
 {
-    auto fn = noalloc_encode_fn();
-    if (!fn) return false;
     const cuuint64_t dims[4] = {d0, d1, d2, 1};
     const cuuint64_t strides[3] = {d0 * 2, d0 * d1 * 2, d0 * d1 * d2 * 2};
     const cuuint32_t box[4] = {64, b1, b2, 1};
-    const cuuint32_t es[4] = {1, 1, 1, 1};
-    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box,
-              es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+    return encode_4d(m, base, dims, strides, box);
 }
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
@@ -155,16 +141,26 @@ extern "C" statekv_status statekv_frame_attention_noalloc(
         return STATEKV_ERR_INVALID_ARG;
     if (D != 64 && D != 128) return STATEKV_ERR_UNSUPPORTED;
     const int G = Hq / Hkv;
-    const int MT = (G * T + kBM - 1) / kBM;
+    // sizes beyond what the kernels or the fixed scratch take are refused
+    // before anything is computed from them in int
+    if (T > kMaxFrameTokens || Hkv > kNoAllocMaxKV ||
+        static_cast<long long>(G) * T > 0x7FFFFFFFll)
+        return STATEKV_ERR_UNSUPPORTED;
+    const long long MT = (static_cast<long long>(G) * T + kBM - 1) / kBM;
     const long long P = static_cast<long long>(B) + T;
-    // sizes beyond the fixed scratch are refused
-    if (Hkv > kNoAllocMaxKV || static_cast<long long>(Hkv) * MT * P >
-                                   static_cast<long long>(kNoAllocMaxPartials))
+    if (static_cast<long long>(Hkv) * MT * P > static_cast<long long>(kNoAllocMaxPartials))
         return STATEKV_ERR_UNSUPPORTED;
 
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    // The call waits for its own work (below), which a stream being captured
+    // cannot do; refuse such a stream before enqueueing anything.
+    cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(st, &cap) != cudaSuccess || cap != cudaStreamCaptureStatusNone) {
+        cudaGetLastError();  // a refused query leaves no sticky error behind
+        return STATEKV_ERR_INVALID_ARG;
+    }
     ScratchAddrs s;
     if (scratch_for_current_device(&s) != cudaSuccess) return STATEKV_ERR_CUDA;
-    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
 
     CUtensorMap tm_sk{}, tm_sv{}, tm_fk{}, tm_fv{};
     if (!noalloc_map(&tm_fk, k, D, Hkv, T, 1, kBN) || !noalloc_map(&tm_fv, v, D, Hkv, T, 1, kBN))
@@ -189,7 +185,7 @@ extern "C" statekv_status statekv_frame_attention_noalloc(
     p.G = G;
     p.B = B;
     p.P = static_cast<int>(P);
-    p.MT = MT;
+    p.MT = static_cast<int>(MT);
     p.causal = cfg->causal_in_frame;
     p.count_mul = 1;
     const float scale =
@@ -198,7 +194,7 @@ extern "C" statekv_status statekv_frame_attention_noalloc(
     p.watchdog_ns = 1000000ull * (cfg->watchdog_ms ? cfg->watchdog_ms : 2000u);
     if (launch_attn(D, tm_sk, tm_sv, tm_fk, tm_fv, p, 1, st) != cudaSuccess) return STATEKV_ERR_CUDA;
     noalloc_importance<<<(Hkv * static_cast<int>(P) + 255) / 256, 256, 0, st>>>(
-        s.partials, importance, Hkv, MT, static_cast<int>(P), B, state_count);
+        s.partials, importance, Hkv, static_cast<int>(MT), static_cast<int>(P), B, state_count);
     if (cudaGetLastError() != cudaSuccess) return STATEKV_ERR_CUDA;
     // The call completes before it returns, so it can report its own device
     // status (an expired wait leaves out / importance unspecified).

@@ -106,7 +106,18 @@ Layout make_layout(const statekv_config& c, const Derived& d)
     return L;
 }
 
-PFN_cuTensorMapEncodeTiled_v12000 encode_fn()
+bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+struct ProfRec {
+    cudaEvent_t a, b;
+    int kind;
+};
+
+}  // namespace
+
+namespace statekv {
+
+static PFN_cuTensorMapEncodeTiled_v12000 encode_fn()
 {
     static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
     static std::once_flag once;
@@ -121,8 +132,8 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn()
     return fn;
 }
 
-// 4-D bf16 tensor map with a (64, b1, b2, 1) box and 128-byte swizzle; OOB
-// elements read as zero.
+bool tma_encode_available() { return encode_fn() != nullptr; }
+
 bool encode_4d(CUtensorMap* m, const void* base, const cuuint64_t dims[4],
                const cuuint64_t strides_bytes[3], const cuuint32_t box[4])
 {
@@ -135,14 +146,7 @@ bool encode_4d(CUtensorMap* m, const void* base, const cuuint64_t dims[4],
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
-
-struct ProfRec {
-    cudaEvent_t a, b;
-    int kind;
-};
-
-}  // namespace
+}  // namespace statekv
 
 struct statekv_handle {
     statekv_config cfg;
@@ -549,7 +553,7 @@ statekv_status statekv_init(const statekv_config* cfg, void* device_arena, size_
     if (!out || !device_arena || !aligned(device_arena, kAlign)) return STATEKV_ERR_INVALID_ARG;
     const Layout lay = make_layout(*cfg, d);
     if (arena_bytes < lay.total) return STATEKV_ERR_ARENA_TOO_SMALL;
-    if (!encode_fn()) return STATEKV_ERR_CUDA;
+    if (!tma_encode_available()) return STATEKV_ERR_CUDA;
 
     statekv_handle* h = new (std::nothrow) statekv_handle();
     if (!h) return STATEKV_ERR_CUDA;

@@ -190,8 +190,17 @@ constexpr int kMaxPool = 24576;
 constexpr int kMaxFrameTokens = 4096;
 size_t select_smem_bytes(int P, int T);
 
+// Every TMA descriptor of the library: a 4-D bf16 tensor map (dims and byte
+// strides innermost first) with a (64, b1, b2, 1) box, 128-byte swizzle and
+// zero fill out of bounds -- the layout the attention kernel's shared-memory
+// descriptors assume.  False when the driver entry point is missing or the
+// driver rejects the map.
+bool encode_4d(CUtensorMap* m, const void* base, const cuuint64_t dims[4],
+               const cuuint64_t strides_bytes[3], const cuuint32_t box[4]);
+bool tma_encode_available();
+
 cudaError_t attn_prepare(int D);
-int device_sm_count();  // SMs of the device (read by attn_prepare)
+int device_sm_count();  // SMs of the current device (read by attn_prepare)
 cudaError_t select_prepare();
 cudaError_t launch_attn(int D, const CUtensorMap& tm_sk, const CUtensorMap& tm_sv,
                         const CUtensorMap& tm_fk, const CUtensorMap& tm_fv, const AttnParams& p,

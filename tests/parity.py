@@ -16,6 +16,9 @@ two results are compared:
 """
 from __future__ import annotations
 
+import os
+from concurrent.futures import ThreadPoolExecutor
+
 import numpy as np
 import torch
 
@@ -31,6 +34,23 @@ BAND = 1e-3
 
 def _bits(t):
     return oracle.as_bf16_bits(t)
+
+
+def _oracle_frames(lays, pre, units, q, k, v):
+    """The oracle's frame for every unit, teacher-forced from the GPU's
+    pre-frame state ``pre[unit]``; units run on host threads side by side
+    (the C loops run outside the Python lock)."""
+    bits = {u: (_bits(q[u[0], u[1]]), _bits(k[u[0], u[1]]), _bits(v[u[0], u[1]])) for u in units}
+
+    def one(u):
+        count, ppos, pk, pv, vlen = pre[u]
+        lay = lays[u]
+        lay.set_state(np.full(lay.n_kv, count, np.int32), ppos, pk, pv, vlen)
+        return lay.prefill_frame(*bits[u])
+
+    workers = max(1, min(len(units), os.cpu_count() or 1))
+    with ThreadPoolExecutor(max_workers=workers) as ex:
+        return dict(zip(units, ex.map(one, units)))
 
 
 def run_parity(shape, nframes, *, kind=None, seed=0, check_frames=None, causal=True,
@@ -104,13 +124,11 @@ def run_parity(shape, nframes, *, kind=None, seed=0, check_frames=None, causal=T
             hist_v[u].append(_bits(v[s, l]))
         if not checking:
             continue
+        refs = _oracle_frames(lays, pre, units, q, k, v)
         for u in units:
             s, l = u
             count, ppos, pk, pv, vlen = pre[u]
-            lay = lays[u]
-            lay.set_state(np.full(Hkv, count, np.int32), ppos, pk, pv, vlen)
-            o_ref, imp_ref, kept_ref = lay.prefill_frame(_bits(q[s, l]), _bits(k[s, l]),
-                                                         _bits(v[s, l]))
+            o_ref, imp_ref, kept_ref = refs[u]
             o_gpu = out[s, l].float().cpu().numpy()
             err = float(np.abs(o_gpu - o_ref).max())
             stats["max_out_err"] = max(stats["max_out_err"], err)
@@ -177,3 +195,70 @@ def run_parity(shape, nframes, *, kind=None, seed=0, check_frames=None, causal=T
             assert np.array_equal(_bits(cv[:, :Ln]), allv.transpose(1, 0, 2)), f"frame {n}: cache V"
     assert eng.sync() == 0
     return eng
+
+
+def run_free_running(shape, nframes, *, kind=None, seed=0, stats=None):
+    """Free-running parity of one (stream, layer): the oracle keeps its own
+    state from frame 1 on and is never reset to the GPU's.
+
+    Until the first near-tie at the selection boundary both sides must hold
+    the same state (as position sets) after every frame, with outputs and
+    importance within the tolerances above.  A frame is a near-tie when the
+    B-th and (B+1)-th best oracle scores are within 2e-3 of each other
+    (relative): each may move by the 1e-3 importance tolerance, so either
+    decision is correct there and the two runs may part.  The run stops after
+    that frame.  Returns the number of frames compared and the frame of the
+    first near-tie (None when there was none).
+    """
+    T, Hq, Hkv, d, B = (shape.tokens_per_frame, shape.num_q_heads, shape.num_kv_heads,
+                        shape.head_dim, shape.state_capacity)
+    assert shape.num_streams == 1 and shape.num_layers == 1
+    eng = StateKV(make_config(shape))
+    lay = oracle.OracleLayer(Hq, Hkv, d, T, B, shape.max_frames)
+    stats = stats if stats is not None else {}
+    tie_frame = None
+    n = 0
+    for n in range(1, nframes + 1):
+        q, k, v = batch_qkv(shape, n, streams=[0], layers=[0], seed=seed, device="cuda", kind=kind)
+        torch.cuda.synchronize()
+        _, _, gpre, ginfo = eng.state(0, 0)
+        gpre = gpre.cpu().numpy().astype(np.int64)
+        count = int(ginfo.count)
+        opre = [lay.state_positions(h) for h in range(Hkv)]
+        for h in range(Hkv):
+            assert sorted(gpre[h, :count].tolist()) == opre[h].tolist(), \
+                f"frame {n} head {h}: states parted before a near-tie"
+        out = torch.full_like(q, float("nan"))
+        imp = torch.full((1, 1, Hkv, B + T), float("nan"), device="cuda")
+        assert eng.prefill_frame(q, k, v, out, imp) == 0
+        o_ref, imp_ref, kept_ref = lay.prefill_frame(_bits(q[0, 0]), _bits(k[0, 0]), _bits(v[0, 0]))
+        torch.cuda.synchronize()
+        err = float(np.abs(out[0, 0].float().cpu().numpy() - o_ref).max())
+        assert err <= OUT_ATOL, f"frame {n}: max |dO| = {err}"
+        g_imp = imp[0, 0].cpu().numpy().astype(np.float64)
+        _, _, gpost, _ = eng.state(0, 0)
+        gpost = gpost.cpu().numpy()
+        near_tie = False
+        for h in range(Hkv):
+            col = {int(p): i for i, p in enumerate(opre[h])}
+            o_cols = np.zeros(B + T)
+            for j in range(count):
+                o_cols[j] = imp_ref[h, col[int(gpre[h, j])]]
+            o_cols[B:] = imp_ref[h, B:]
+            sel = np.r_[0:count, B:B + T]
+            assert np.all(np.abs(g_imp[h, sel] - o_cols[sel]) <= IMP_RTOL * np.abs(o_cols[sel]) + IMP_ATOL), \
+                f"frame {n} head {h}: importance"
+            scores = np.sort(np.concatenate([imp_ref[h, :count], imp_ref[h, B:]]))[::-1]
+            if B > 0 and len(scores) > B:
+                tau = scores[B - 1]
+                near_tie |= bool(scores[B - 1] - scores[B] <= 2 * BAND * tau)
+        if near_tie:
+            tie_frame = n
+            break
+        for h in range(Hkv):
+            gset = sorted(int(x) for x in gpost[h] if x >= 0)
+            assert gset == lay.state_positions(h).tolist(), f"frame {n} head {h}: kept sets differ"
+    assert eng.sync() == 0
+    stats["frames"] = n
+    stats["first_near_tie"] = tie_frame
+    return n, tie_frame

@@ -13,7 +13,7 @@ import torch
 from paper_2605_31598_gb300 import StateKV, make_config
 from paper_2605_31598_gb300.inputs import WORKLOADS, Shape, batch_qkv
 
-from .parity import run_parity
+from .parity import run_free_running, run_parity
 
 pytestmark = pytest.mark.gpu
 
@@ -200,6 +200,62 @@ def test_qwen7b_stack_full_size_sampled_units():
     stats = {}
     run_parity(shape, 12, check_frames=[11, 12], units=[(0, 0), (0, 27)], stats=stats)
     print("qwen7b_stack", stats)
+
+
+def test_qwen7b_stack_late_frames():
+    """The 28-layer 7B stack carried to frame 256, the last frame of its
+    workload (positions up to 50,175; 245 frames of state churn after the
+    state fills), in the benchmark's one-call-per-frame launch: frames 128
+    and 256 compared in full on three of the 28 layers."""
+    stats = {}
+    run_parity(WORKLOADS["qwen7b_stack"], 256, check_frames=[128, 256],
+               units=[(0, 0), (0, 13), (0, 27)], stats=stats)
+    print("qwen7b_stack late", stats)
+
+
+def test_qwen72b_stack_first_evictions():
+    """The 80-layer 72B-shaped stack (64 q / 8 kv heads, B 4096: 33 state key
+    tiles per unit, a 4292-member pool) in its one-launch-per-frame
+    configuration: frame 21 (the first whose pool exceeds B) and frame 24
+    compared in full on three of the 80 layers.  The decode cache is sized
+    for 24 frames; the launch does not depend on it."""
+    shape = dataclasses.replace(WORKLOADS["qwen72b_stack"], max_frames=24)
+    stats = {}
+    run_parity(shape, 24, check_frames=[21, 24], units=[(0, 0), (0, 41), (0, 79)], stats=stats)
+    print("qwen72b_stack", stats)
+
+
+def test_qwen7b_8streams_late_frame():
+    """Eight concurrent 7B streams (28 layers each, 224 units per launch)
+    carried to frame 1024, the end of the streaming workload (virtual
+    positions up to 200,703): frames 512 and 1024 compared in full on one
+    layer of each of two streams."""
+    stats = {}
+    run_parity(WORKLOADS["qwen7b_8streams"], 1024, check_frames=[512, 1024],
+               units=[(2, 5), (6, 27)], stats=stats)
+    print("qwen7b_8streams late", stats)
+
+
+FREE_RUNNING = {
+    # the toy layer over 32 frames: its first near-tie comes at frame 13
+    "toy": (dataclasses.replace(WORKLOADS["toy"], max_frames=32), None),
+    # one KV head of 4 query heads, d 128, T 64, B 128, unit-variance Q/K:
+    # first near-tie at frame 8
+    "peaked_g4_t64": (Shape(4, 1, 128, 64, 128, 32), "peaked"),
+}
+
+
+@pytest.mark.parametrize("name", sorted(FREE_RUNNING))
+def test_free_running_until_first_near_tie(name):
+    """The GPU and the oracle each keep their own state from frame 1 (no
+    teacher forcing): the kept position sets must agree after every frame
+    until the first frame whose selection boundary is a near-tie."""
+    shape, kind = FREE_RUNNING[name]
+    stats = {}
+    n, tie = run_free_running(shape, shape.max_frames, kind=kind, stats=stats)
+    print("free running", name, stats)
+    first_eviction = shape.state_capacity // shape.tokens_per_frame + 1
+    assert n >= first_eviction + 2  # several evicting frames matched exactly
 
 
 @pytest.mark.gpu
