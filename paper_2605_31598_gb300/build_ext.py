@@ -2,9 +2,8 @@
 
 Each translation unit compiles in parallel into ``_build/``; the objects link
 into ``paper_2605_31598_gb300/libstatekv.so`` with the CUDA runtime linked
-statically and cuBLASLt (used only by the transformer-block entry point)
-linked from the toolkit's lib64 by rpath, so the library loads on a machine
-without a GPU driver (it needs one only when a call reaches the device).
+statically and no other library, so it loads on a machine without a GPU
+driver (it needs one only when a call reaches the device).
 """
 from __future__ import annotations
 
@@ -20,7 +19,7 @@ CSRC = os.path.join(PKG, "csrc")
 OUT = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libstatekv.so")
 SOURCES = ["attn_kernel.cu", "select_kernel.cu", "diag_kernel.cu", "block_kernel.cu", "decode_kernel.cu",
-           "statekv_api.cu", "noalloc.cu"]
+           "gemm_kernel.cu", "statekv_api.cu", "noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
          "--expt-relaxed-constexpr", "-I", os.path.join(ROOT, "include")]
@@ -70,10 +69,7 @@ def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
         list(ex.map(run, jobs))
     if force or jobs or not _newer(LIB, objs):
         tmp = LIB + ".tmp.%d" % os.getpid()
-        # cuBLASLt (the block's projection GEMMs) from the toolkit next to nvcc
-        cuda_lib = os.path.join(os.path.dirname(os.path.dirname(nvcc)), "lib64")
-        run([nvcc, *ARCH, "-shared", "-o", tmp, *objs, "-L", cuda_lib, "-lcublasLt",
-             "-Xlinker", "-rpath," + cuda_lib])
+        run([nvcc, *ARCH, "-shared", "-o", tmp, *objs])
         os.replace(tmp, LIB)
     return LIB
 

@@ -287,6 +287,7 @@ struct WorkUnit {
     int nft;    // frame key tiles the tile's last row can see
     int nt;     // nst + nft
     int rot;    // first state tile (see state_tile)
+    int full_state;  // state tiles [0, full_state) hold 128 valid keys wherever they start
 };
 
 __device__ __forceinline__ WorkUnit work_unit(const AttnParams& p, int w)
@@ -308,6 +309,10 @@ __device__ __forceinline__ WorkUnit work_unit(const AttnParams& p, int w)
     // a different one (a fixed rotation) so they do not all request the same
     // L2 lines at the same moment.  Frame tiles keep their order.
     x.rot = x.nst > 0 ? (x.mt * 3) % x.nst : 0;
+    // with a rotation the ragged state tile (the last one, if count % 128 != 0)
+    // can come at any position; only when every state tile is whole is the
+    // check skipped for all of them
+    x.full_state = (x.count % kBN == 0) ? x.nst : 0;
     return x;
 }
 
@@ -856,19 +861,22 @@ __global__ void __launch_bounds__(kThreads, 1)
                 ok = __all_sync(0xffffffffu, wait_until(&sb_full[b], (g >> 1) & 1, deadline));
                 if (!ok) break;
                 tc_fence_after();
-                int lim4[4];  // keys [0, lim) of this tile are visible to each row
-                if (j < x.nst) {
-                    const int lim = min(kBN, x.count - state_tile(x, j) * kBN);
+                int lim4[4] = {kBN, kBN, kBN, kBN};  // keys [0, lim) of this tile are visible to each row
+                bool full = true;
+                if (j >= x.full_state) {  // the last state tile or a frame tile
+                    if (j < x.nst) {
+                        const int lim = min(kBN, x.count - state_tile(x, j) * kBN);
 #pragma unroll
-                    for (int q4 = 0; q4 < 4; ++q4) lim4[q4] = lim;
-                } else {
-                    const int f0 = (j - x.nst) * kBN;
+                        for (int q4 = 0; q4 < 4; ++q4) lim4[q4] = lim;
+                    } else {
+                        const int f0 = (j - x.nst) * kBN;
 #pragma unroll
-                    for (int q4 = 0; q4 < 4; ++q4)
-                        lim4[q4] = min(kBN, (p.causal ? min(T, tq4[q4] + 1) : T) - f0);
+                        for (int q4 = 0; q4 < 4; ++q4)
+                            lim4[q4] = min(kBN, (p.causal ? min(T, tq4[q4] + 1) : T) - f0);
+                    }
+                    const int lmin = min(min(lim4[0], lim4[1]), min(lim4[2], lim4[3]));
+                    full = lmin >= c0 + 64;
                 }
-                const int lmin = min(min(lim4[0], lim4[1]), min(lim4[2], lim4[3]));
-                const bool full = lmin >= c0 + 64;
                 float v[2][32];
 #pragma unroll
                 for (int h = 0; h < 2; ++h) tmem_ld_16x256b_x8((b ? tSh1 : tSh0) + ((16u * h) << 16), v[h]);
@@ -889,12 +897,20 @@ __global__ void __launch_bounds__(kThreads, 1)
                             upk(fma2(pk(v[h][i], v[h][i + 1]), cc, pk(nk, nk)), x0, x1);
                             v[h][i] = ex2(x0);
                             v[h][i + 1] = ex2(x1);
-                            if (!full) {
+                        }
+                if (!full) {  // a ragged tile: keys at or past a row's limit get zero weight
+#pragma unroll
+                    for (int h = 0; h < 2; ++h)
+#pragma unroll
+                        for (int r = 0; r < 8; ++r)
+#pragma unroll
+                            for (int k2 = 0; k2 < 2; ++k2) {
+                                const int i = 4 * r + 2 * k2;
                                 const int col = c0 + 8 * r + cq, lim = lim4[2 * h + k2];
                                 v[h][i] = col < lim ? v[h][i] : 0.f;
                                 v[h][i + 1] = col + 1 < lim ? v[h][i + 1] : 0.f;
                             }
-                        }
+                }
                 // the P buffer is free once the P V of tile g - 2 has read it
                 if (b == 0 && g >= 2)
                     ok = __all_sync(0xffffffffu, wait_until(&pv_done[0], ((g - 2) >> 1) & 1, deadline));

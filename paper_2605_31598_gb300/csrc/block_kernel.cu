@@ -9,16 +9,10 @@
 //                layout.  Angles p * theta_k are formed and reduced modulo
 //                2 pi in fp64 (p reaches 2^20 and more), then sin/cos in fp32.
 //   silu_mul     a = SiLU(gate) * up                       (fp32, one rounding)
-//   projections  plain bf16 GEMMs on cuBLASLt (fp32 accumulation): the QKV
-//                projection with its bias in the epilogue, the output and
-//                down projections accumulating into the residual stream.
+// The projection GEMMs themselves run on the tensor cores (gemm_kernel.cu).
 // Rows are tokens (stream-major, then token): one CTA per row for the norm and
 // the rotation, 8 elements per thread for SiLU * up; 16-byte accesses where
 // the layout allows.
-#include <cublasLt.h>
-
-#include <vector>
-
 #include "statekv_kernels.cuh"
 
 namespace statekv {
@@ -170,161 +164,6 @@ cudaError_t launch_silu_mul(const __nv_bfloat16* gu, __nv_bfloat16* a, long long
     silu_mul_kernel<<<static_cast<unsigned>((total + 255) / 256), 256, 0, st>>>(
         gu, a, static_cast<int>(rows), I);
     return cudaGetLastError();
-}
-
-// ------------------------------------------------------------------ GEMMs
-// cuBLASLt's first heuristic choice is not always its fastest for the block's
-// shapes (196 rows per stream against thousands of output features), so the
-// first call of each shape times up to kLtCandidates of its candidates on the
-// call's own operands and keeps the fastest.
-constexpr int kLtCandidates = 8;
-
-struct LtPlan {
-    int M, N, K;
-    bool bias, add;
-    cublasLtMatmulDesc_t op = nullptr;
-    cublasLtMatrixLayout_t a = nullptr, b = nullptr, c = nullptr;
-    int nalgo = 0, chosen = 0;
-    bool tuned = false;
-    cublasLtMatmulAlgo_t algo[kLtCandidates];
-    size_t ws[kLtCandidates];
-};
-
-struct LtContext {
-    cublasLtHandle_t h = nullptr;
-    std::vector<LtPlan> plans;
-};
-
-LtContext* lt_create()
-{
-    LtContext* c = new LtContext;
-    if (cublasLtCreate(&c->h) != CUBLAS_STATUS_SUCCESS) {
-        delete c;
-        return nullptr;
-    }
-    return c;
-}
-
-void lt_destroy(LtContext* c)
-{
-    if (!c) return;
-    for (LtPlan& p : c->plans) {
-        cublasLtMatrixLayoutDestroy(p.a);
-        cublasLtMatrixLayoutDestroy(p.b);
-        cublasLtMatrixLayoutDestroy(p.c);
-        cublasLtMatmulDescDestroy(p.op);
-    }
-    cublasLtDestroy(c->h);
-    delete c;
-}
-
-namespace {
-
-// Row-major D[M][N] = X[M][K] W[N][K]^T: in cuBLASLt's column-major terms
-// D^T (N x M) = op_T(W as K x N) * X^T (K x M).
-LtPlan* lt_plan(LtContext* c, int M, int N, int K, bool bias, bool add, size_t ws_bytes)
-{
-    for (LtPlan& p : c->plans)
-        if (p.M == M && p.N == N && p.K == K && p.bias == bias && p.add == add) return &p;
-    LtPlan p;
-    p.M = M;
-    p.N = N;
-    p.K = K;
-    p.bias = bias;
-    p.add = add;
-    bool ok = cublasLtMatmulDescCreate(&p.op, CUBLAS_COMPUTE_32F, CUDA_R_32F) == CUBLAS_STATUS_SUCCESS;
-    const cublasOperation_t ta = CUBLAS_OP_T, tb = CUBLAS_OP_N;
-    ok = ok &&
-         cublasLtMatmulDescSetAttribute(p.op, CUBLASLT_MATMUL_DESC_TRANSA, &ta, sizeof ta) ==
-             CUBLAS_STATUS_SUCCESS &&
-         cublasLtMatmulDescSetAttribute(p.op, CUBLASLT_MATMUL_DESC_TRANSB, &tb, sizeof tb) ==
-             CUBLAS_STATUS_SUCCESS;
-    if (ok && bias) {
-        const cublasLtEpilogue_t ep = CUBLASLT_EPILOGUE_BIAS;
-        ok = cublasLtMatmulDescSetAttribute(p.op, CUBLASLT_MATMUL_DESC_EPILOGUE, &ep, sizeof ep) ==
-             CUBLAS_STATUS_SUCCESS;
-    }
-    ok = ok &&
-         cublasLtMatrixLayoutCreate(&p.a, CUDA_R_16BF, K, N, K) == CUBLAS_STATUS_SUCCESS &&
-         cublasLtMatrixLayoutCreate(&p.b, CUDA_R_16BF, K, M, K) == CUBLAS_STATUS_SUCCESS &&
-         cublasLtMatrixLayoutCreate(&p.c, CUDA_R_16BF, N, M, N) == CUBLAS_STATUS_SUCCESS;
-    cublasLtMatmulPreference_t pref = nullptr;
-    ok = ok && cublasLtMatmulPreferenceCreate(&pref) == CUBLAS_STATUS_SUCCESS &&
-         cublasLtMatmulPreferenceSetAttribute(pref, CUBLASLT_MATMUL_PREF_MAX_WORKSPACE_BYTES,
-                                              &ws_bytes, sizeof ws_bytes) == CUBLAS_STATUS_SUCCESS;
-    cublasLtMatmulHeuristicResult_t res[kLtCandidates] = {};
-    int found = 0;
-    ok = ok && cublasLtMatmulAlgoGetHeuristic(c->h, p.op, p.a, p.b, p.c, p.c, pref, kLtCandidates, res,
-                                              &found) == CUBLAS_STATUS_SUCCESS &&
-         found > 0;
-    if (pref) cublasLtMatmulPreferenceDestroy(pref);
-    if (!ok) {
-        cublasLtMatrixLayoutDestroy(p.a);
-        cublasLtMatrixLayoutDestroy(p.b);
-        cublasLtMatrixLayoutDestroy(p.c);
-        cublasLtMatmulDescDestroy(p.op);
-        return nullptr;
-    }
-    for (int i = 0; i < found; ++i) {
-        p.algo[i] = res[i].algo;
-        p.ws[i] = res[i].workspaceSize;
-    }
-    p.nalgo = found;
-    p.tuned = found <= 1;
-    c->plans.push_back(p);
-    return &c->plans.back();
-}
-
-bool lt_run(LtContext* c, const LtPlan& p, int i, const __nv_bfloat16* X, const __nv_bfloat16* W,
-            __nv_bfloat16* D, float beta, void* ws, cudaStream_t st)
-{
-    const float alpha = 1.f;
-    return cublasLtMatmul(c->h, p.op, &alpha, W, p.a, X, p.b, &beta, D, p.c, D, p.c, &p.algo[i], ws,
-                          p.ws[i], st) == CUBLAS_STATUS_SUCCESS;
-}
-
-}  // namespace
-
-bool lt_matmul(LtContext* c, const __nv_bfloat16* X, const __nv_bfloat16* W,
-               const __nv_bfloat16* bias, __nv_bfloat16* D, bool add, int M, int N, int K,
-               void* ws, size_t ws_bytes, void* scratch, size_t scratch_bytes, cudaStream_t st)
-{
-    if (M <= 0) return true;
-    LtPlan* p = lt_plan(c, M, N, K, bias != nullptr, add, ws_bytes);
-    if (!p) return false;
-    if (bias && cublasLtMatmulDescSetAttribute(p->op, CUBLASLT_MATMUL_DESC_BIAS_POINTER, &bias,
-                                               sizeof bias) != CUBLAS_STATUS_SUCCESS)
-        return false;
-    if (!p->tuned) {
-        // time each candidate (beta = 0) into scratch, or into D when D is
-        // written over anyway; a candidate that fails is skipped
-        __nv_bfloat16* out = static_cast<size_t>(M) * N * 2 <= scratch_bytes
-                                 ? static_cast<__nv_bfloat16*>(scratch)
-                                 : (!add ? D : nullptr);
-        cudaEvent_t e0 = nullptr, e1 = nullptr;
-        if (out && cudaEventCreate(&e0) == cudaSuccess && cudaEventCreate(&e1) == cudaSuccess) {
-            float best = -1.f;
-            for (int i = 0; i < p->nalgo; ++i) {
-                if (!lt_run(c, *p, i, X, W, out, 0.f, ws, st)) continue;  // warm-up
-                cudaEventRecord(e0, st);
-                bool ok = true;
-                for (int r = 0; r < 3 && ok; ++r) ok = lt_run(c, *p, i, X, W, out, 0.f, ws, st);
-                cudaEventRecord(e1, st);
-                float ms = 0.f;
-                if (!ok || cudaEventSynchronize(e1) != cudaSuccess ||
-                    cudaEventElapsedTime(&ms, e0, e1) != cudaSuccess)
-                    continue;
-                if (best < 0.f || ms < best) {
-                    best = ms;
-                    p->chosen = i;
-                }
-            }
-        }
-        if (e0) cudaEventDestroy(e0);
-        if (e1) cudaEventDestroy(e1);
-        p->tuned = true;
-    }
-    return lt_run(c, *p, p->chosen, X, W, D, add ? 1.f : 0.f, ws, st);
 }
 
 }  // namespace statekv

@@ -162,7 +162,6 @@ struct statekv_handle {
     bool prof_on;
     size_t prof_used;
     std::vector<ProfRec> prof;
-    LtContext* lt = nullptr;   // cuBLASLt, created by the first block call
     // The decode-cache append runs on a side stream forked from the call's
     // stream and joined before the selection: it depends on nothing the
     // attention kernel writes, so it fills SMs the attention grid leaves idle.
@@ -202,7 +201,9 @@ void release_streams(statekv_handle* h)
 statekv_status device_status(int32_t word)
 {
     if (word == 0) return STATEKV_OK;
-    return (word & 0xFF) == DEV_TIMEOUT_ATTN ? STATEKV_ERR_DEVICE_TIMEOUT : STATEKV_ERR_DEVICE_FAULT;
+    const int kind = word & 0xFF;
+    return kind == DEV_TIMEOUT_ATTN || kind == DEV_TIMEOUT_GEMM ? STATEKV_ERR_DEVICE_TIMEOUT
+                                                                : STATEKV_ERR_DEVICE_FAULT;
 }
 
 statekv_status check_args(const statekv_handle* h, const statekv_frame_args* a, bool host)
@@ -587,6 +588,7 @@ statekv_status statekv_init(const statekv_config* cfg, void* device_arena, size_
 
     const int D = cfg->head_dim, B = cfg->state_capacity, Hkv = cfg->num_kv_heads;
     bool ok = attn_prepare(D) == cudaSuccess && select_prepare() == cudaSuccess &&
+              gemm_prepare() == cudaSuccess &&
               decode_prepare() == cudaSuccess;
     if (ok && B > 0) {
         const cuuint64_t dims[4] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(B),
@@ -747,11 +749,28 @@ namespace {
 
 // Workspace carve-up of one block call (all offsets 256-byte aligned).
 struct BlockBufs {
-    size_t h, qkv, q, k, v, attn, gu, act, lt, total;
+    size_t h, qkv, q, k, v, attn, gu, act, gemm_part, gemm_cnt, total;
 };
 
-constexpr size_t kLtWorkspace = 32u << 20;  // cuBLASLt's own workspace
-constexpr size_t kLtScratch = 32u << 20;    // output of the one-time algorithm timing
+// split-K tile counters: one region per projection GEMM of a block call (a
+// split plan has fewer tiles than SMs), zeroed at the start of the call
+constexpr int kGemmCounterRegion = 256;
+
+// The four projection GEMMs of a layer at `rows` rows: (N, K) of QKV, O,
+// gate/up and down.
+void block_gemm_shapes(const statekv_config& c, const statekv_block_config& b, int (&nk)[4][2])
+{
+    const int d = c.head_dim, hq = c.num_q_heads, hkv = c.num_kv_heads;
+    const int H = b.hidden, I = b.intermediate;
+    nk[0][0] = (hq + 2 * hkv) * d;
+    nk[0][1] = H;
+    nk[1][0] = H;
+    nk[1][1] = hq * d;
+    nk[2][0] = 2 * I;
+    nk[2][1] = H;
+    nk[3][0] = H;
+    nk[3][1] = I;
+}
 
 BlockBufs block_bufs(const statekv_config& c, const statekv_block_config& b, int streams)
 {
@@ -773,7 +792,13 @@ BlockBufs block_bufs(const statekv_config& c, const statekv_block_config& b, int
     o.attn = take(rows * hq * d * 2);
     o.gu = take(rows * 2 * static_cast<size_t>(b.intermediate) * 2);
     o.act = take(rows * static_cast<size_t>(b.intermediate) * 2);
-    o.lt = take(kLtWorkspace + kLtScratch);
+    // split-K partials of the largest split GEMM, and their tile counters
+    int nk[4][2];
+    block_gemm_shapes(c, b, nk);
+    size_t part = 0;
+    for (auto& g : nk) part = std::max(part, gemm_plan(static_cast<int>(rows), g[0], g[1], device_sm_count()).partial_bytes);
+    o.gemm_part = take(part);
+    o.gemm_cnt = take(static_cast<size_t>(4) * c.num_layers * kGemmCounterRegion * 4);
     o.total = off;
     return o;
 }
@@ -837,7 +862,6 @@ statekv_status statekv_block_frame(statekv_handle* h, const statekv_block_config
     probe.out = buf(bb.attn);
     const statekv_status s = check_args(h, &probe, false);
     if (s != STATEKV_OK) return s;
-    if (!h->lt && !(h->lt = lt_create())) return STATEKV_ERR_CUDA;
 
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     const int T = c.tokens_per_frame, d = c.head_dim, Hq = c.num_q_heads, Hkv = c.num_kv_heads;
@@ -876,18 +900,44 @@ statekv_status statekv_block_frame(statekv_handle* h, const statekv_block_config
         }
         if (b.yarn_factor > 1.f) rp.scale = static_cast<float>(0.1 * std::log(b.yarn_factor) + 1.0);
     }
-    void* ltws = ws + bb.lt;
+    const int sms = device_sm_count();
+    int* gemm_cnt = reinterpret_cast<int*>(ws + bb.gemm_cnt);
+    if (cudaMemsetAsync(gemm_cnt, 0, static_cast<size_t>(4) * layer_count * kGemmCounterRegion * 4, st) !=
+        cudaSuccess)
+        return STATEKV_ERR_CUDA;
+    int gemm_seq = 0;  // the call's projection GEMMs in order: each has its own counters
+    // D[rows][N] = X[rows][K] W[N][K]^T (+ bias) (+ D), on the tensor cores
     auto gemm = [&](const void* X, const void* Wt, const void* bias, __nv_bfloat16* D, bool add,
                     int N, int K) {
-        return timed(h, 3, st, [&] {
-                   return lt_matmul(h->lt, static_cast<const __nv_bfloat16*>(X),
-                                    static_cast<const __nv_bfloat16*>(Wt),
-                                    static_cast<const __nv_bfloat16*>(bias), D, add, rows, N, K,
-                                    ltws, kLtWorkspace, static_cast<uint8_t*>(ltws) + kLtWorkspace,
-                                    kLtScratch, st)
-                              ? cudaSuccess
-                              : cudaErrorNotSupported;
-               }) == cudaSuccess;
+        const GemmPlan g = gemm_plan(rows, N, K, sms);
+        if (g.counters > kGemmCounterRegion) return false;
+        int* counters = gemm_cnt + static_cast<size_t>(gemm_seq++) * kGemmCounterRegion;
+        CUtensorMap tx, tw;
+        const cuuint64_t dx[4] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(rows), 1, 1};
+        const cuuint64_t dw[4] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(N), 1, 1};
+        const cuuint64_t sx[3] = {static_cast<cuuint64_t>(K) * 2, static_cast<cuuint64_t>(K) * rows * 2,
+                                  static_cast<cuuint64_t>(K) * rows * 2};
+        const cuuint64_t sw[3] = {static_cast<cuuint64_t>(K) * 2, static_cast<cuuint64_t>(K) * N * 2,
+                                  static_cast<cuuint64_t>(K) * N * 2};
+        const cuuint32_t box[4] = {static_cast<cuuint32_t>(kGemmBK), static_cast<cuuint32_t>(kGemmBM), 1, 1};
+        if (!encode_4d(&tx, X, dx, sx, box) || !encode_4d(&tw, Wt, dw, sw, box)) return false;
+        GemmParams gp{};
+        gp.M = rows;
+        gp.N = N;
+        gp.K = K;
+        gp.n_tiles = g.n_tiles;
+        gp.k_steps = g.k_steps;
+        gp.kps = g.kps;
+        gp.splits = g.splits;
+        gp.units = g.units;
+        gp.bias = static_cast<const __nv_bfloat16*>(bias);
+        gp.D = D;
+        gp.add = add ? 1 : 0;
+        gp.partials = reinterpret_cast<float*>(ws + bb.gemm_part);
+        gp.counters = counters;
+        gp.status = h->status_dev;
+        gp.watchdog_ns = 1000000ull * (c.watchdog_ms ? c.watchdog_ms : 2000u);
+        return timed(h, 3, st, [&] { return launch_gemm(tx, tw, gp, sms, st); }) == cudaSuccess;
     };
     for (int l = layer_begin; l < layer_begin + layer_count; ++l) {
         const statekv_block_weights& w = weights[l];
@@ -896,8 +946,7 @@ statekv_status statekv_block_frame(statekv_handle* h, const statekv_block_config
                                       buf(bb.h), rows, H, st);
             }) != cudaSuccess)
             return STATEKV_ERR_CUDA;
-        if (!gemm(buf(bb.h), w.w_qkv, w.b_qkv, buf(bb.qkv), false, W, H))
-            return STATEKV_ERR_UNSUPPORTED;
+        if (!gemm(buf(bb.h), w.w_qkv, w.b_qkv, buf(bb.qkv), false, W, H)) return STATEKV_ERR_CUDA;
         rp.layer = l;
         if (timed(h, 4, st, [&] { return launch_qkv_rope(rp, st); }) != cudaSuccess)
             return STATEKV_ERR_CUDA;
@@ -906,18 +955,17 @@ statekv_status statekv_block_frame(statekv_handle* h, const statekv_block_config
         a.layer_count = 1;
         const statekv_status r = run_step(h, a, st);
         if (r != STATEKV_OK) return r;
-        if (!gemm(buf(bb.attn), w.w_o, nullptr, x, true, H, Hq * d)) return STATEKV_ERR_UNSUPPORTED;
+        if (!gemm(buf(bb.attn), w.w_o, nullptr, x, true, H, Hq * d)) return STATEKV_ERR_CUDA;
         if (timed(h, 4, st, [&] {
                 return launch_rmsnorm(x, static_cast<const __nv_bfloat16*>(w.norm_mlp), b.rms_eps,
                                       buf(bb.h), rows, H, st);
             }) != cudaSuccess)
             return STATEKV_ERR_CUDA;
-        if (!gemm(buf(bb.h), w.w_gate_up, nullptr, buf(bb.gu), false, 2 * I, H))
-            return STATEKV_ERR_UNSUPPORTED;
+        if (!gemm(buf(bb.h), w.w_gate_up, nullptr, buf(bb.gu), false, 2 * I, H)) return STATEKV_ERR_CUDA;
         if (timed(h, 4, st, [&] { return launch_silu_mul(buf(bb.gu), buf(bb.act), rows, I, st); }) !=
             cudaSuccess)
             return STATEKV_ERR_CUDA;
-        if (!gemm(buf(bb.act), w.w_down, nullptr, x, true, H, I)) return STATEKV_ERR_UNSUPPORTED;
+        if (!gemm(buf(bb.act), w.w_down, nullptr, x, true, H, I)) return STATEKV_ERR_CUDA;
     }
     return STATEKV_OK;
 }
@@ -1173,7 +1221,6 @@ void statekv_destroy(statekv_handle* h)
         cudaEventDestroy(r.b);
     }
     cudaFreeHost(const_cast<int32_t*>(h->status_host));
-    lt_destroy(h->lt);
     release_streams(h);
     delete h;
 }

@@ -28,6 +28,8 @@ enum DeviceError : int32_t {
     DEV_OK = 0,
     DEV_TIMEOUT_ATTN = 1,
     DEV_BAD_SELECT = 2,  // the top-B selection admitted more tokens than free slots
+    DEV_TIMEOUT_GEMM = 3,  // a projection-GEMM wait expired (bits 8..15: 2 producer,
+                           // 3 MMA issuer stage, 4 MMA issuer accumulator, 5 epilogue)
 };
 
 // Tile sizes of the attention kernel: 128 query rows x 128 keys per MMA tile.
@@ -141,16 +143,34 @@ cudaError_t launch_rmsnorm(const __nv_bfloat16* x, const __nv_bfloat16* g, float
 cudaError_t launch_qkv_rope(const RopeParams& p, cudaStream_t st);
 cudaError_t launch_silu_mul(const __nv_bfloat16* gu, __nv_bfloat16* a, long long rows, int I,
                             cudaStream_t st);
-struct LtContext;
-LtContext* lt_create();
-void lt_destroy(LtContext* c);
-// Row-major D[M][N] = X[M][K] W[N][K]^T (+ bias[N]) (+ D when add), bf16 in and
-// out, fp32 accumulation; false if cuBLASLt has no plan or fails.  The first
-// call of a shape times cuBLASLt's candidate algorithms (synchronising the
-// stream once) into `scratch` (or into D when it is overwritten anyway).
-bool lt_matmul(LtContext* c, const __nv_bfloat16* X, const __nv_bfloat16* W,
-               const __nv_bfloat16* bias, __nv_bfloat16* D, bool add, int M, int N, int K,
-               void* ws, size_t ws_bytes, void* scratch, size_t scratch_bytes, cudaStream_t st);
+// Projection GEMMs of the block (gemm_kernel.cu): D[M][N] = X[M][K] W[N][K]^T
+// (+ bias[N]) (+ D when add), bf16, fp32 accumulation on tcgen05.  A unit is
+// a 128-column tile of W for a pair of 128-row tiles of X over kps 64-wide K
+// steps; splits > 1 writes fp32 partials [units][2][128][128] and, in a
+// cooperative launch, every split of a tile waits for its siblings
+// (counters[tile], zero on entry, left at `splits`) and adds its share of the
+// tile's rows over all splits in split order.
+constexpr int kGemmBM = 128, kGemmBN = 128, kGemmBK = 64;
+struct GemmPlan {
+    int n_tiles, m_pairs, k_steps, kps, splits, units, counters;
+    size_t partial_bytes;
+};
+GemmPlan gemm_plan(int M, int N, int K, int sms);
+struct GemmParams {
+    int M, N, K;
+    int n_tiles, k_steps, kps, splits, units;
+    const __nv_bfloat16* bias;  // nullable [N]
+    __nv_bfloat16* D;           // [M][N]
+    int add;                    // 1: D += X W^T
+    float* partials;            // splits > 1: [units][2][128][128]
+    int* counters;              // splits > 1: [n_tiles * m_pairs], zero on entry, used once
+    int32_t* status;
+    unsigned long long watchdog_ns;
+};
+cudaError_t gemm_prepare();
+cudaError_t launch_gemm(const CUtensorMap& tm_x, const CUtensorMap& tm_w, const GemmParams& p,
+                        int sms, cudaStream_t st);
+
 
 // One-pass split-K decoding over the cache (decode_kernel.cu): for up to
 // kDecodeRows query rows (new tokens x query heads of a KV head).

@@ -154,3 +154,18 @@ def test_block_qwen7b_geometry_two_layers():
     stats = {}
     worst = run_block_parity(shape, BLOCKS["qwen7b"], 3, check_frames=[1, 3], stats=stats)
     print("7B block worst |dx|", worst, stats)
+
+
+@pytest.mark.gpu
+def test_block_ragged_widths_many_streams():
+    """Widths that are not multiples of the GEMM tiles (hidden 136, MLP 200:
+    ragged 128-column tiles and a ragged last 64-wide K step) and 20 streams
+    (320 rows: two 256-row pairs, the second only partly filled), so the
+    projections take several row pairs and split K."""
+    from paper_2605_31598_gb300.inputs import BlockShape
+
+    _need_gpu()
+    shape = Shape(4, 2, 64, 16, 32, 3, num_layers=1, num_streams=20)
+    stats = {}
+    worst = run_block_parity(shape, BlockShape(136, 200, weight_std=0.08), 3, stats=stats)
+    print("ragged block worst |dx|", worst, stats)
