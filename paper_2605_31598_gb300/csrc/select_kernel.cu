@@ -51,9 +51,7 @@ __device__ __forceinline__ int block_exclusive_scan(int x, int* warp_sums, int& 
     }
     __syncthreads();
     excl = warp_sums[warp] + incl - x;
-    const int total = warp_sums[kSelWarps];
-    __syncthreads();
-    return total;
+    return warp_sums[kSelWarps];  // warp_sums is not written again before the caller's next barrier
 }
 
 // For each of 8 pool members (columns col[e], active act[e]): the sum of
@@ -116,10 +114,11 @@ __global__ void __launch_bounds__(kSelThreads)
     uint64_t* key = reinterpret_cast<uint64_t*>(smem_raw);            // [P]
     int* free_slot = reinterpret_cast<int*>(key + P);                  // [T]
     int* adm_tok = free_slot + T;                                      // [T]
-    __shared__ unsigned hist[256];
+    __shared__ unsigned hist2[2][256];  // pass p counts into hist2[p & 1]; the other is cleared meanwhile
     __shared__ int warp_sums[kSelWarps + 1];
     __shared__ unsigned long long sh_prefix, sh_mask;
-    __shared__ int sh_k, sh_done;
+    __shared__ int sh_k, sh_done, sh_shift;
+    __shared__ unsigned long long warp_and[kSelWarps], warp_or[kSelWarps];
 
     const int hkv = blockIdx.x, u = blockIdx.y;
     const int ua = p.units.unit_abs(u);
@@ -139,6 +138,8 @@ __global__ void __launch_bounds__(kSelThreads)
     // outside them, so all its loads are independent (the partials come from
     // L2); each member's sum still adds the tiles in order.
     const float* part0 = p.partials + static_cast<size_t>(u) * p.Hkv * p.MT * P;
+    // bits every selection key shares: the radix select starts below them
+    unsigned long long kand = ~0ull, kor = 0ull;
     if ((P & 3) == 0) {
         // Column space, four adjacent columns per thread (16-byte loads): state
         // slot c < count is member c, frame column B + t is member count + t,
@@ -169,8 +170,11 @@ __global__ void __launch_bounds__(kSelThreads)
                 const int c = c0 + e;
                 const int i = c < count ? c : (c >= B && c - B < T) ? count + (c - B) : -1;
                 if (i < 0) continue;
-                key[i] = (static_cast<uint64_t>(__float_as_uint(rv[e])) << 32) |
-                         static_cast<uint32_t>(0xFFFFFFFFu - static_cast<uint32_t>(ps[e]));
+                const uint64_t kk = (static_cast<uint64_t>(__float_as_uint(rv[e])) << 32) |
+                                    static_cast<uint32_t>(0xFFFFFFFFu - static_cast<uint32_t>(ps[e]));
+                key[i] = kk;
+                kand &= kk;
+                kor |= kk;
                 if (imp_out) imp_out[c] = sv[e];
             }
         }
@@ -201,8 +205,11 @@ __global__ void __launch_bounds__(kSelThreads)
                 if (!act[e]) continue;
                 const int i = i0 + tid + e * kSelThreads;
                 const float rank = p.shared ? r[e] : s[e];
-                key[i] = (static_cast<uint64_t>(__float_as_uint(rank)) << 32) |
-                         static_cast<uint32_t>(0xFFFFFFFFu - static_cast<uint32_t>(ps[e]));
+                const uint64_t kk = (static_cast<uint64_t>(__float_as_uint(rank)) << 32) |
+                                    static_cast<uint32_t>(0xFFFFFFFFu - static_cast<uint32_t>(ps[e]));
+                key[i] = kk;
+                kand &= kk;
+                kor |= kk;
                 if (imp_out) imp_out[col[e]] = s[e];
             }
         }
@@ -217,14 +224,41 @@ __global__ void __launch_bounds__(kSelThreads)
     // 2. top-B selection: kept(i) <=> (key[i] & mask) >= prefix
     unsigned long long prefix = 0, mask = 0;
     if (n > B) {
+        {   // block-wide AND and OR of the keys: digits above the highest bit in
+            // which two keys differ hold one value for every key, so the radix
+            // passes start at the digit holding that bit
+            const uint32_t ah = __reduce_and_sync(0xffffffffu, static_cast<uint32_t>(kand >> 32));
+            const uint32_t al = __reduce_and_sync(0xffffffffu, static_cast<uint32_t>(kand));
+            const uint32_t oh = __reduce_or_sync(0xffffffffu, static_cast<uint32_t>(kor >> 32));
+            const uint32_t ol = __reduce_or_sync(0xffffffffu, static_cast<uint32_t>(kor));
+            if (lane == 0) {
+                warp_and[tid >> 5] = (static_cast<unsigned long long>(ah) << 32) | al;
+                warp_or[tid >> 5] = (static_cast<unsigned long long>(oh) << 32) | ol;
+            }
+        }
+        __syncthreads();
         if (tid == 0) {
+            unsigned long long a = ~0ull, o = 0ull;
+            for (int w = 0; w < kSelWarps; ++w) {
+                a &= warp_and[w];
+                o |= warp_or[w];
+            }
+            const unsigned long long diff = a ^ o;  // bits in which some keys differ
+            const int hb = diff ? 63 - __clzll(static_cast<long long>(diff)) : 0;
+            const int shift0 = (hb / 8) * 8;
+            const unsigned long long above = shift0 >= 56 ? 0ull : ~((1ull << (shift0 + 8)) - 1);
+            sh_shift = shift0;
+            sh_prefix = o & above;  // = a & above
+            sh_mask = above;
             sh_k = B;
             sh_done = 0;
         }
+        for (int i = tid; i < 512; i += kSelThreads) hist2[i >> 8][i & 255] = 0;
         __syncthreads();
-        for (int shift = 56; shift >= 0; shift -= 8) {
-            for (int i = tid; i < 256; i += kSelThreads) hist[i] = 0;
-            __syncthreads();
+        prefix = sh_prefix;
+        mask = sh_mask;
+        for (int shift = sh_shift, pass = 0; shift >= 0; shift -= 8, ++pass) {
+            unsigned* hist = hist2[pass & 1];
             for (int i0 = 0; i0 < n; i0 += kSelThreads) {
                 const int i = i0 + tid;
                 int digit = -1;
@@ -233,7 +267,9 @@ __global__ void __launch_bounds__(kSelThreads)
                 if (digit >= 0 && lane == __ffs(peers) - 1) atomicAdd(&hist[digit], __popc(peers));
             }
             __syncthreads();
-            if (tid < 32) {
+            if (tid >= 32) {  // the next pass's histogram, while warp 0 reads this one
+                for (int i = tid - 32; i < 256; i += kSelThreads - 32) hist2[(pass + 1) & 1][i] = 0;
+            } else {
                 // lane owns digits 255 - 8*lane - j, j = 0..7 (descending)
                 unsigned c[8], local = 0;
 #pragma unroll
