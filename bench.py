@@ -46,7 +46,9 @@ KERNEL_SOURCE = os.path.join(ROOT, "paper_2605_31598_gb300", "csrc", "attn_kerne
 # first 16 hex digits of the sha256 of the attention-kernel source it was taken
 # on.  A workload or kernel source with no capture reports null.
 K1_DRAM_BYTES = {
-    ("qwen7b_stack", "a7a9ed44211fd1b8"): 199170304,
+    ("qwen7b_stack", "c61b81053cfe3200"): 198420480,
+    ("qwen72b_stack", "c61b81053cfe3200"): 2044000000,    # ncu's printed 1.66 GB + 384.00 MB
+    ("qwen7b_8streams", "c61b81053cfe3200"): 1733380000,  # ncu's printed 1.35 GB + 383.38 MB
 }
 
 
