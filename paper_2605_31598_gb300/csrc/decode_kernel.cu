@@ -11,34 +11,68 @@
 // padded to 16) keeps the instruction count far below the memory time.
 //
 //   decode_partial   grid (chunks, KV heads, units), 4 warps.  A warp takes 32
-//                    keys at a time: their K and V rows (256 B each) arrive by
-//                    coalesced 16-byte asynchronous copies, two steps ahead,
-//                    into the warp's three-stage shared memory (rows padded to D + 8 so
-//                    fragment loads hit distinct banks), then S = Q K^T, the
-//                    running max / sum per row, P in bf16, O += P V.  The 4
-//                    warps' (max, sum, O) merge into the chunk's partial.
+//                    keys at a time: their K and V rows arrive as TMA tensor
+//                    copies (boxes of 64 columns x 32 keys of the cache's 4-D
+//                    map, 128-byte swizzle), two steps ahead, into the warp's
+//                    three-stage ring, each stage behind an mbarrier; fragment
+//                    loads undo the swizzle, so they hit distinct banks.  Then
+//                    S = Q K^T, the running max / sum per row, P in bf16,
+//                    O += P V.  The 4 warps' (max, sum, O) merge into the
+//                    chunk's partial.  Every wait is bounded by the watchdog.
 //   decode_combine   one CTA per (unit, KV head): the chunks' partials merge
 //                    (rescaled to the overall max) into O / sum, written as bf16.
+#include "sm103_ptx.cuh"
 #include "statekv_kernels.cuh"
 
 namespace statekv {
 namespace {
 
+using namespace ptx;
+
 constexpr int kDecThreads = 128;
 constexpr int kDecWarps = kDecThreads / 32;
-constexpr int kDecKeys = 32;  // keys per warp step
+constexpr int kDecKeys = kDecodeKeyBox;  // keys per warp step (one TMA box)
 constexpr int kDecStages = 3; // steps a warp has in flight or in use
 
 template <int D>
 struct DecLayout {
-    static constexpr int kRow = D + 8;                       // padded row (bf16)
-    static constexpr int kMat = kDecKeys * kRow * 2;         // bytes of 32 rows
+    // a 32-key tile of K (or V): D / 64 blocks of 32 rows x 128 bytes (64
+    // columns), each in the TMA's 128-byte swizzle (1 KB atoms of 8 rows)
+    static constexpr int kBlock = kDecKeys * 128;
+    static constexpr int kMat = (D / 64) * kBlock;
     static constexpr int kStage = 2 * kMat;                  // K and V
     static constexpr int kWarp = kDecStages * kStage;
-    static constexpr int kBytes = kDecWarps * kWarp;
-    static_assert(kDecWarps * kDecodeRows * D * 4 + 2 * kDecWarps * kDecodeRows * 4 <= kBytes,
+    static constexpr int kOffBar = kDecWarps * kWarp;        // full[warp][stage]
+    static constexpr int kBytes = kOffBar + kDecWarps * kDecStages * 8;
+    static constexpr int kAlloc = kBytes + 1024;             // room to align the base to 1 KB
+    static_assert(kDecWarps * kDecodeRows * D * 4 + 2 * kDecWarps * kDecodeRows * 4 <= kOffBar,
                   "merge area fits");
+    static_assert(kBlock % 1024 == 0, "swizzle atoms stay aligned");
 };
+
+// Byte offset of element (row, col) of a swizzled 32-key tile.
+__device__ __forceinline__ uint32_t sw_off(int row, int col)
+{
+    const int blk = col >> 6, cc = col & 63;
+    return blk * (kDecKeys * 128) + row * 128 + ((((cc >> 3) ^ (row & 7))) << 4) + ((cc & 7) << 1);
+}
+
+__device__ __forceinline__ unsigned long long dec_timer()
+{
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+__device__ __forceinline__ bool dec_wait(uint64_t* bar, uint32_t parity, unsigned long long deadline)
+{
+    for (;;) {
+#pragma unroll 1
+        for (int i = 0; i < 64; ++i)
+            if (mbar_try_wait(bar, parity)) return true;
+        if (dec_timer() > deadline) return false;
+    }
+}
 
 __device__ __forceinline__ float ex2(float x)
 {
@@ -64,21 +98,15 @@ __device__ __forceinline__ void mma16816(float (&d)[4], const uint32_t (&a)[4], 
         : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
 
-__device__ __forceinline__ void cp_async16(void* smem, const void* gmem)
-{
-    const uint32_t sa = static_cast<uint32_t>(__cvta_generic_to_shared(smem));
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(sa), "l"(gmem) : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
-
 template <int D>
-__global__ void __launch_bounds__(kDecThreads) decode_partial(const DecodeParams p)
+__global__ void __launch_bounds__(kDecThreads)
+    decode_partial(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
+                   const DecodeParams p)
 {
     using L = DecLayout<D>;
-    constexpr int KS = L::kRow;
-    extern __shared__ __align__(16) uint8_t dsm[];
+    extern __shared__ uint8_t dsm_raw[];
+    uint8_t* dsm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(dsm_raw) + 1023) &
+                                              ~static_cast<uintptr_t>(1023));
     const int chunk = blockIdx.x, hkv = blockIdx.y, u = blockIdx.z;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int g = lane >> 2, tig = lane & 3;  // fragment row group and column pair
@@ -88,9 +116,15 @@ __global__ void __launch_bounds__(kDecThreads) decode_partial(const DecodeParams
     const int len = len0 + p.n;
     const int R = p.n * p.G;
     const int k0 = chunk * p.ck, k1 = min(len, k0 + p.ck);
-    const __nv_bfloat16* Kh = p.cache_k + head * p.cap * D;
-    const __nv_bfloat16* Vh = p.cache_v + head * p.cap * D;
     uint8_t* wsm = dsm + warp * L::kWarp;
+    uint64_t* full = reinterpret_cast<uint64_t*>(dsm + L::kOffBar) + warp * kDecStages;
+    if (lane == 0) {
+        for (int s2 = 0; s2 < kDecStages; ++s2) mbar_init(&full[s2], 1);
+        fence_mbar_init();
+    }
+    __syncwarp();
+    const unsigned long long deadline = dec_timer() + p.watchdog_ns;
+    bool ok = true;
 
     // Q as A fragments: row r = token r / G, head hkv G + r % G (rows >= R are 0)
     uint32_t qa[D / 16][4];
@@ -109,19 +143,20 @@ __global__ void __launch_bounds__(kDecThreads) decode_partial(const DecodeParams
             qa[ks][3] = pack_bf16(qval(g + 8, c + 8), qval(g + 8, c + 9));
         }
     }
-    // the 32 K and V rows from key `base` into stage st (rows past the cache
-    // capacity read its last row; their scores are masked)
+    // the 32 K and V rows from key `base` into stage st, by one lane (rows past
+    // the cache capacity read as zero; their scores are masked)
     auto load_step = [&](int base, int st) {
-        __nv_bfloat16* ks = reinterpret_cast<__nv_bfloat16*>(wsm + st * L::kStage);
-        __nv_bfloat16* vs = reinterpret_cast<__nv_bfloat16*>(wsm + st * L::kStage + L::kMat);
+        if (lane == 0) {
+            uint8_t* ks = wsm + st * L::kStage;
+            uint8_t* vs = ks + L::kMat;
+            fence_proxy_async_smem();  // the warp's earlier reads of this stage come first
+            mbar_arrive_expect_tx(&full[st], 2 * L::kMat);
 #pragma unroll
-        for (int i = 0; i < kDecKeys * D / 8 / 32; ++i) {
-            const int cidx = lane + 32 * i, row = cidx / (D / 8), c16 = cidx % (D / 8);
-            const long long key = min(static_cast<long long>(base + row), p.cap - 1);
-            cp_async16(ks + row * KS + c16 * 8, Kh + key * D + c16 * 8);
-            cp_async16(vs + row * KS + c16 * 8, Vh + key * D + c16 * 8);
+            for (int hb = 0; hb < D / 64; ++hb) {
+                tma_load_4d(ks + hb * L::kBlock, &tm_k, &full[st], hb * 64, base, hkv, ua);
+                tma_load_4d(vs + hb * L::kBlock, &tm_v, &full[st], hb * 64, base, hkv, ua);
+            }
         }
-        cp_async_commit();
     };
 
     const float c = p.scale_log2;
@@ -135,23 +170,21 @@ __global__ void __launch_bounds__(kDecThreads) decode_partial(const DecodeParams
     const int stride = kDecWarps * kDecKeys;
     const int base0 = k0 + warp * kDecKeys;
     const int nsteps = base0 < k1 ? (k1 - base0 + stride - 1) / stride : 0;
-    // kDecStages - 1 steps ahead; a step without copies still commits a
-    // (empty) group so that the wait count below stays uniform
+    // kDecStages - 1 steps ahead
 #pragma unroll
-    for (int s0 = 0; s0 < kDecStages - 1; ++s0) {
+    for (int s0 = 0; s0 < kDecStages - 1; ++s0)
         if (s0 < nsteps) load_step(base0 + s0 * stride, s0);
-        else cp_async_commit();
-    }
-    for (int step = 0; step < nsteps; ++step) {
+    int step = 0;
+    for (; step < nsteps; ++step) {
         const int base = base0 + step * stride;
         const int st = step % kDecStages;
         const int pre = step + kDecStages - 1;
+        // the stage `pre` lands in was read by step - 1, which this warp finished
         if (pre < nsteps) load_step(base0 + pre * stride, pre % kDecStages);
-        else cp_async_commit();
-        cp_async_wait<kDecStages - 1>();  // this step's group has landed
-        __syncwarp();
-        const __nv_bfloat16* ks = reinterpret_cast<const __nv_bfloat16*>(wsm + st * L::kStage);
-        const __nv_bfloat16* vs = reinterpret_cast<const __nv_bfloat16*>(wsm + st * L::kStage + L::kMat);
+        ok = __all_sync(0xffffffffu, dec_wait(&full[st], (step / kDecStages) & 1, deadline));
+        if (!ok) break;
+        const uint8_t* ks = wsm + st * L::kStage;
+        const uint8_t* vs = ks + L::kMat;
         // S = Q K^T: 4 key tiles of 8
         float sc[4][4];
 #pragma unroll
@@ -160,9 +193,9 @@ __global__ void __launch_bounds__(kDecThreads) decode_partial(const DecodeParams
             for (int e = 0; e < 4; ++e) sc[nt][e] = 0.f;
 #pragma unroll
             for (int kst = 0; kst < D / 16; ++kst) {
-                const __nv_bfloat16* kr = ks + (nt * 8 + g) * KS + kst * 16 + 2 * tig;
-                mma16816(sc[nt], qa[kst], *reinterpret_cast<const uint32_t*>(kr),
-                         *reinterpret_cast<const uint32_t*>(kr + 8));
+                const int kr = nt * 8 + g, kc = kst * 16 + 2 * tig;
+                mma16816(sc[nt], qa[kst], *reinterpret_cast<const uint32_t*>(ks + sw_off(kr, kc)),
+                         *reinterpret_cast<const uint32_t*>(ks + sw_off(kr, kc + 8)));
             }
         }
         // masks, running max / sum of rows g (h = 0) and g + 8 (h = 1)
@@ -213,22 +246,29 @@ __global__ void __launch_bounds__(kDecThreads) decode_partial(const DecodeParams
                                     pack_bf16(sc[2 * j][2], sc[2 * j][3]),
                                     pack_bf16(sc[2 * j + 1][0], sc[2 * j + 1][1]),
                                     pack_bf16(sc[2 * j + 1][2], sc[2 * j + 1][3])};
-            const __nv_bfloat16* v0 = vs + (16 * j + 2 * tig) * KS + g;
+            const int vr0 = 16 * j + 2 * tig;
 #pragma unroll
             for (int nd = 0; nd < D / 8; ++nd) {
-                const __nv_bfloat16* vr = v0 + nd * 8;
+                const int vc = nd * 8 + g;
+                auto vat = [&](int r) { return *reinterpret_cast<const __nv_bfloat16*>(vs + sw_off(r, vc)); };
                 __nv_bfloat162 b0, b1;
-                b0.x = vr[0];
-                b0.y = vr[KS];
-                b1.x = vr[8 * KS];
-                b1.y = vr[9 * KS];
+                b0.x = vat(vr0);
+                b0.y = vat(vr0 + 1);
+                b1.x = vat(vr0 + 8);
+                b1.y = vat(vr0 + 9);
                 mma16816(o[nd], pa, *reinterpret_cast<const uint32_t*>(&b0),
                          *reinterpret_cast<const uint32_t*>(&b1));
             }
         }
         __syncwarp();  // the stage is refilled kDecStages - 1 steps later
     }
-    cp_async_wait<0>();
+    if (!ok) {
+        if (lane == 0) *reinterpret_cast<volatile int32_t*>(p.status) = DEV_TIMEOUT_DECODE;
+        // let the copies already issued land before the shared memory is reused
+        if (lane == 0)
+            for (int s2 = step; s2 < min(nsteps, step + kDecStages); ++s2)
+                dec_wait(&full[s2 % kDecStages], (s2 / kDecStages) & 1, dec_timer() + p.watchdog_ns);
+    }
     __syncthreads();
 
     // merge the 4 warps into the chunk's partial (reusing the staging memory)
@@ -302,15 +342,16 @@ __global__ void __launch_bounds__(256) decode_combine(const DecodeParams p)
 
 }  // namespace
 
-cudaError_t launch_decode(const DecodeParams& p, int D, int U, cudaStream_t st)
+cudaError_t launch_decode(const CUtensorMap& tm_k, const CUtensorMap& tm_v, const DecodeParams& p, int D,
+                          int U, cudaStream_t st)
 {
     if (U <= 0) return cudaSuccess;
     const dim3 g1(p.nchunk, p.Hkv, U), g2(p.Hkv, U);
     if (D == 64) {
-        decode_partial<64><<<g1, kDecThreads, DecLayout<64>::kBytes, st>>>(p);
+        decode_partial<64><<<g1, kDecThreads, DecLayout<64>::kAlloc, st>>>(tm_k, tm_v, p);
         decode_combine<64><<<g2, 256, 0, st>>>(p);
     } else {
-        decode_partial<128><<<g1, kDecThreads, DecLayout<128>::kBytes, st>>>(p);
+        decode_partial<128><<<g1, kDecThreads, DecLayout<128>::kAlloc, st>>>(tm_k, tm_v, p);
         decode_combine<128><<<g2, 256, 0, st>>>(p);
     }
     return cudaGetLastError();
@@ -319,10 +360,10 @@ cudaError_t launch_decode(const DecodeParams& p, int D, int U, cudaStream_t st)
 cudaError_t decode_prepare()
 {
     cudaError_t e = cudaFuncSetAttribute(decode_partial<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         DecLayout<64>::kBytes);
+                                         DecLayout<64>::kAlloc);
     if (e != cudaSuccess) return e;
     return cudaFuncSetAttribute(decode_partial<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                DecLayout<128>::kBytes);
+                                DecLayout<128>::kAlloc);
 }
 
 }  // namespace statekv

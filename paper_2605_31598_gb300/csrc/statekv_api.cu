@@ -156,7 +156,8 @@ struct statekv_handle {
     std::vector<int32_t> frames_host;  // [S*L]
     std::vector<int32_t> text_host;    // [S*L]: tokens appended by statekv_decode_step
     CUtensorMap tm_sk, tm_sv;  // state rows, [S*L][Hkv][B][D]
-    CUtensorMap tm_ck, tm_cv;  // decode-cache rows, [S*L][Hkv][cap][D]
+    CUtensorMap tm_ck, tm_cv;  // decode-cache rows, [S*L][Hkv][cap][D], boxes of 128 keys
+    CUtensorMap tm_dk, tm_dv;  // the same with boxes of kDecodeKeyBox keys (decode kernel)
     volatile int32_t* status_host;
     int32_t* status_dev;
     bool prof_on;
@@ -202,8 +203,9 @@ statekv_status device_status(int32_t word)
 {
     if (word == 0) return STATEKV_OK;
     const int kind = word & 0xFF;
-    return kind == DEV_TIMEOUT_ATTN || kind == DEV_TIMEOUT_GEMM ? STATEKV_ERR_DEVICE_TIMEOUT
-                                                                : STATEKV_ERR_DEVICE_FAULT;
+    return kind == DEV_TIMEOUT_ATTN || kind == DEV_TIMEOUT_GEMM || kind == DEV_TIMEOUT_DECODE
+               ? STATEKV_ERR_DEVICE_TIMEOUT
+               : STATEKV_ERR_DEVICE_FAULT;
 }
 
 statekv_status check_args(const statekv_handle* h, const statekv_frame_args* a, bool host)
@@ -479,8 +481,10 @@ statekv_status run_decode(statekv_handle* h, const statekv_decode_args& a, cudaS
         dp.T = T;
         dp.cap = d.cap;
         dp.scale_log2 = d.scale * 1.4426950408889634f;
+        dp.status = h->status_dev;
+        dp.watchdog_ns = 1000000ull * (c.watchdog_ms ? c.watchdog_ms : 2000u);
         if (timed(h, 0, st, [&] { return launch_append(ap, st); }) != cudaSuccess ||
-            timed(h, 1, st, [&] { return launch_decode(dp, D, U, st); }) != cudaSuccess ||
+            timed(h, 1, st, [&] { return launch_decode(h->tm_dk, h->tm_dv, dp, D, U, st); }) != cudaSuccess ||
             launch_advance(text, ur, U, Hkv, n, st) != cudaSuccess)
             return STATEKV_ERR_CUDA;
         for (int s = a.stream_begin; s < a.stream_begin + a.stream_count; ++s)
@@ -570,6 +574,8 @@ statekv_status statekv_init(const statekv_config* cfg, void* device_arena, size_
     std::memset(&h->tm_sv, 0, sizeof(CUtensorMap));
     std::memset(&h->tm_ck, 0, sizeof(CUtensorMap));
     std::memset(&h->tm_cv, 0, sizeof(CUtensorMap));
+    std::memset(&h->tm_dk, 0, sizeof(CUtensorMap));
+    std::memset(&h->tm_dv, 0, sizeof(CUtensorMap));
 
     void* st_host = nullptr;
     if (cudaHostAlloc(&st_host, 64, cudaHostAllocMapped) != cudaSuccess) {
@@ -607,8 +613,11 @@ statekv_status statekv_init(const statekv_config* cfg, void* device_arena, size_
                                        static_cast<cuuint64_t>(d.cap) * D * 2,
                                        static_cast<cuuint64_t>(Hkv) * d.cap * D * 2};
         const cuuint32_t box[4] = {64, static_cast<cuuint32_t>(kBN), 1, 1};
+        const cuuint32_t dbox[4] = {64, static_cast<cuuint32_t>(kDecodeKeyBox), 1, 1};
         ok = encode_4d(&h->tm_ck, h->arena + lay.cache_k, dims, strides, box) &&
-             encode_4d(&h->tm_cv, h->arena + lay.cache_v, dims, strides, box);
+             encode_4d(&h->tm_cv, h->arena + lay.cache_v, dims, strides, box) &&
+             encode_4d(&h->tm_dk, h->arena + lay.cache_k, dims, strides, dbox) &&
+             encode_4d(&h->tm_dv, h->arena + lay.cache_v, dims, strides, dbox);
     }
     ok = ok && create_streams(h);
     // Empty states and decode caches: zero rows, positions -1.  A key tile that

@@ -30,6 +30,7 @@ enum DeviceError : int32_t {
     DEV_BAD_SELECT = 2,  // the top-B selection admitted more tokens than free slots
     DEV_TIMEOUT_GEMM = 3,  // a projection-GEMM wait expired (bits 8..15: 2 producer,
                            // 3 MMA issuer stage, 4 MMA issuer accumulator, 5 epilogue)
+    DEV_TIMEOUT_DECODE = 4,  // a decode kernel's wait for its K/V copies expired
 };
 
 // Tile sizes of the attention kernel: 128 query rows x 128 keys per MMA tile.
@@ -190,8 +191,14 @@ struct DecodeParams {
     long long cap;
     int ck, nchunk;             // keys per chunk (a multiple of 256), chunks
     float scale_log2;
+    int32_t* status;
+    unsigned long long watchdog_ns;
 };
-cudaError_t launch_decode(const DecodeParams& p, int D, int U, cudaStream_t st);
+// tm_k / tm_v: the decode caches as 4-D maps [S*L][Hkv][cap][D] with boxes of
+// 64 columns x 32 keys (kDecodeKeyBox), 128-byte swizzle
+constexpr int kDecodeKeyBox = 32;
+cudaError_t launch_decode(const CUtensorMap& tm_k, const CUtensorMap& tm_v, const DecodeParams& p, int D,
+                          int U, cudaStream_t st);
 cudaError_t decode_prepare();  // once, before the first launch_decode
 
 // Recency-window state update (the baseline): the frame's tokens enter ring
