@@ -372,8 +372,24 @@ statekv_status statekv_watchdog_selftest(statekv_handle* h, statekv_stream strea
 
 /* The raw device status word (0 = none): low byte 1 = an attention-kernel
  * wait expired (bits 8..15 name the waiting site), 2 = the selection kernel
- * found an inconsistent top-B split.  Read without synchronising. */
+ * found an inconsistent top-B split, 3 = a projection-GEMM wait expired,
+ * 4 = a decode-kernel wait expired, 5 / 6 = a debug build's bounds check or
+ * guard band failed (see statekv_debug_check).  Read without synchronising. */
 statekv_status statekv_device_error(const statekv_handle* h, int32_t* code);
+
+/* Debug builds (the library compiled with STATEKV_DEBUG_CHECKS=1, e.g.
+ * build_ext.build(debug=True) -> libstatekv_debug.so) put a 256-byte guard band
+ * after every arena region, filled with 0xA5 at init, and check indices before
+ * the state, cache and importance writes; a failed check records a bounds
+ * fault in the status word and skips the access (no trap).  This call
+ * enqueues a comparison of every guard byte with its fill on `stream`; an
+ * overwritten band records a canary fault.  Either fault is reported, like any
+ * device fault, as STATEKV_ERR_DEVICE_FAULT by the next call that reads the
+ * status (statekv_sync), with the kind in statekv_device_error's low byte
+ * (5 bounds, 6 canary) and the site or band in bits 8..15.  A release build
+ * returns STATEKV_ERR_UNSUPPORTED and enqueues nothing.  These are the
+ * sanitizer substitutes of the implementation; the paper has no counterpart. */
+statekv_status statekv_debug_check(statekv_handle* h, statekv_stream stream);
 
 /* Frame attention with importance (steps a1 and a2) for ONE (stream, layer)
  * against a caller-given state, for callers that cannot allocate device

@@ -18,6 +18,10 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 OUT = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libstatekv.so")
+# the debug build: bounds checks that record a fault in the status word, and
+# guard bands around the arena's regions (STATEKV_DEBUG_CHECKS=1)
+OUT_DEBUG = os.path.join(PKG, "_build_debug")
+LIB_DEBUG = os.path.join(PKG, "libstatekv_debug.so")
 SOURCES = ["attn_kernel.cu", "select_kernel.cu", "diag_kernel.cu", "block_kernel.cu", "decode_kernel.cu",
            "gemm_kernel.cu", "statekv_api.cu", "noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
@@ -45,15 +49,19 @@ def _headers():
     return hs
 
 
-def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
-    """Compile and link; returns the library path.  Rebuilds only what changed."""
+def build(force: bool = False, verbose: bool = False, extra_flags=(), debug: bool = False) -> str:
+    """Compile and link; returns the library path.  Rebuilds only what changed.
+    ``debug`` builds ``libstatekv_debug.so`` with STATEKV_DEBUG_CHECKS=1."""
     nvcc = _nvcc()
-    os.makedirs(OUT, exist_ok=True)
+    out_dir, lib_path = (OUT_DEBUG, LIB_DEBUG) if debug else (OUT, LIB)
+    if debug:
+        extra_flags = tuple(extra_flags) + ("-DSTATEKV_DEBUG_CHECKS=1",)
+    os.makedirs(out_dir, exist_ok=True)
     headers = _headers()
     objs, jobs = [], []
     for src in SOURCES:
         spath = os.path.join(CSRC, src)
-        obj = os.path.join(OUT, src.replace(".cu", ".o"))
+        obj = os.path.join(out_dir, src.replace(".cu", ".o"))
         objs.append(obj)
         if force or not _newer(obj, [spath] + headers):
             jobs.append([nvcc, *ARCH, *FLAGS, *extra_flags, "-c", spath, "-o", obj])
@@ -67,11 +75,11 @@ def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
 
     with cf.ThreadPoolExecutor(max_workers=len(SOURCES)) as ex:
         list(ex.map(run, jobs))
-    if force or jobs or not _newer(LIB, objs):
-        tmp = LIB + ".tmp.%d" % os.getpid()
+    if force or jobs or not _newer(lib_path, objs):
+        tmp = lib_path + ".tmp.%d" % os.getpid()
         run([nvcc, *ARCH, "-shared", "-o", tmp, *objs])
-        os.replace(tmp, LIB)
-    return LIB
+        os.replace(tmp, lib_path)
+    return lib_path
 
 
 if __name__ == "__main__":

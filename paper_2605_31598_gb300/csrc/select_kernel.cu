@@ -132,6 +132,9 @@ __global__ void __launch_bounds__(kSelThreads)
     float* imp_out =
         p.importance ? p.importance + (static_cast<size_t>(u) * p.Hkv + hkv) * P : nullptr;
     const int n = count + T;
+    // the counters come from the arena: a state larger than B or a negative frame
+    // count would index past the pool (uniform across the CTA)
+    if (!SKV_CHECK(count >= 0 && count <= B && nf >= 0, p.status, 1)) return;
 
     // 1. importance (fixed-order sum over query tiles) and selection keys.  A
     // thread takes up to 8 pool members at once and walks the query tiles
@@ -351,11 +354,13 @@ __global__ void __launch_bounds__(kSelThreads)
         const int r = w % (npairs * chunks);
         const int i = r / chunks, ch = r % chunks;
         const int t = adm_tok[i], s = free_slot[i];
+        if (!SKV_CHECK(t >= 0 && t < T && s >= 0 && s < B, p.status, 2)) continue;
         const __nv_bfloat16* src = (which ? vsrc : ksrc) + t * src_stride + ch * 8;
         __nv_bfloat16* dst = (which ? vdst : kdst) + static_cast<size_t>(s) * D + ch * 8;
         *reinterpret_cast<uint4*>(dst) = *reinterpret_cast<const uint4*>(src);
     }
-    for (int i = tid; i < npairs; i += kSelThreads) pos[free_slot[i]] = L + adm_tok[i];
+    for (int i = tid; i < npairs; i += kSelThreads)
+        if (SKV_CHECK(free_slot[i] >= 0 && free_slot[i] < B, p.status, 3)) pos[free_slot[i]] = L + adm_tok[i];
     if (tid == 0) {
         p.counts[head] = min(B, count + T);
         p.frames[head] = nf + 1;
@@ -384,11 +389,27 @@ __global__ void __launch_bounds__(256) decode_cache_append(const AppendParams p)
                                    static_cast<size_t>(rr) * 8;
         __nv_bfloat16* dst = (which ? p.cache_v : p.cache_k) +
                              (head * p.cap + row) * p.D + ch * 8;
+        if (!SKV_CHECK(row >= 0 && row < p.cap, p.status, 4)) continue;
         *reinterpret_cast<uint4*>(dst) = *reinterpret_cast<const uint4*>(src);
     }
 }
 
+// one CTA of kGuardBytes threads per guard band
+__global__ void canary_check(const uint8_t* arena, const GuardList g, int32_t* status)
+{
+    const int b = blockIdx.x;
+    if (b < g.n && arena[g.off[b] + threadIdx.x] != kGuardFill)
+        *reinterpret_cast<volatile int32_t*>(status) = DEV_CANARY | (b << 8);
+}
+
 }  // namespace
+
+cudaError_t launch_canary_check(const uint8_t* arena, const GuardList& g, int32_t* status, cudaStream_t st)
+{
+    if (g.n <= 0) return cudaSuccess;
+    canary_check<<<g.n, kGuardBytes, 0, st>>>(arena, g, status);
+    return cudaGetLastError();
+}
 
 size_t select_smem_bytes(int P, int T)
 {

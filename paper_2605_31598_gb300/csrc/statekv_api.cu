@@ -27,11 +27,16 @@ constexpr int kProfPairs = 3 * 4096;
 
 size_t round_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
+// Debug builds put a guard band of kGuardBytes after every arena region,
+// filled with kGuardFill at init and compared by statekv_debug_check.
+constexpr size_t kGuard = STATEKV_DEBUG_CHECKS ? kGuardBytes : 0;
+
 struct Layout {
     size_t state_k, state_v, positions, counts, frames, text, cache_k, cache_v, partials;
     struct Staging {
         size_t q, k, v, out, imp;
     } stg[2];  // host-buffer calls: two frames, so copies overlap the steps
+    GuardList guards;
     size_t total;
 };
 
@@ -79,6 +84,10 @@ Layout make_layout(const statekv_config& c, const Derived& d)
     auto take = [&](size_t bytes) {
         const size_t at = off;
         off += round_up(bytes);
+        if (kGuard > 0 && L.guards.n < kMaxGuards) {
+            L.guards.off[L.guards.n++] = off;
+            off += kGuard;
+        }
         return at;
     };
     L.state_k = take(heads * B * D * 2);
@@ -285,6 +294,7 @@ statekv_status run_step(statekv_handle* h, const statekv_frame_args& a, cudaStre
     ap.D = D;
     ap.row_mul = T;
     ap.cap = d.cap;
+    ap.status = h->status_dev;
     // append on the side stream; it reads the frame counters, so the join
     // comes before the selection kernel advances them
     if (cudaEventRecord(h->ev_fork, st) != cudaSuccess ||
@@ -437,6 +447,7 @@ statekv_status run_decode(statekv_handle* h, const statekv_decode_args& a, cudaS
     ap.D = D;
     ap.row_mul = T;
     ap.cap = d.cap;
+    ap.status = h->status_dev;
     if (n * d.G <= kDecodeRows) {
         // A few rows: the new tokens' K/V go into the cache first, then the
         // one-pass split-K kernel reads every key once from the cache.
@@ -627,8 +638,10 @@ statekv_status statekv_init(const statekv_config* cfg, void* device_arena, size_
     ok = ok && cudaMemset(h->arena + lay.state_k, 0, lay.positions - lay.state_k) == cudaSuccess &&
          cudaMemset(h->arena + lay.positions, 0xFF, lay.counts - lay.positions) == cudaSuccess &&
          cudaMemset(h->arena + lay.counts, 0, lay.cache_k - lay.counts) == cudaSuccess &&
-         cudaMemset(h->arena + lay.cache_k, 0, lay.partials - lay.cache_k) == cudaSuccess &&
-         cudaDeviceSynchronize() == cudaSuccess;
+         cudaMemset(h->arena + lay.cache_k, 0, lay.partials - lay.cache_k) == cudaSuccess;
+    for (int i = 0; ok && i < lay.guards.n; ++i)  // debug builds: the guard bands, after the fills above
+        ok = cudaMemset(h->arena + lay.guards.off[i], kGuardFill, kGuard) == cudaSuccess;
+    ok = ok && cudaDeviceSynchronize() == cudaSuccess;
     if (!ok) {
         cudaFreeHost(st_host);
         release_streams(h);
@@ -645,6 +658,17 @@ statekv_status statekv_prefill_frame(statekv_handle* h, const statekv_frame_args
     const statekv_status s = check_args(h, args, false);
     if (s != STATEKV_OK) return s;
     return run_step(h, *args, reinterpret_cast<cudaStream_t>(stream));
+}
+
+statekv_status statekv_debug_check(statekv_handle* h, statekv_stream stream)
+{
+    if (!h) return STATEKV_ERR_INVALID_ARG;
+    if (!STATEKV_DEBUG_CHECKS) return STATEKV_ERR_UNSUPPORTED;
+    if (*h->status_host != 0) return device_status(*h->status_host);
+    return launch_canary_check(h->arena, h->lay.guards, h->status_dev,
+                               reinterpret_cast<cudaStream_t>(stream)) == cudaSuccess
+               ? STATEKV_OK
+               : STATEKV_ERR_CUDA;
 }
 
 statekv_status statekv_full_attention_frame(statekv_handle* h, const statekv_frame_args* args,

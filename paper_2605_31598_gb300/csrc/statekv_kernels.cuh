@@ -31,7 +31,30 @@ enum DeviceError : int32_t {
     DEV_TIMEOUT_GEMM = 3,  // a projection-GEMM wait expired (bits 8..15: 2 producer,
                            // 3 MMA issuer stage, 4 MMA issuer accumulator, 5 epilogue)
     DEV_TIMEOUT_DECODE = 4,  // a decode kernel's wait for its K/V copies expired
+    DEV_BOUNDS = 5,          // debug builds: an index failed its bounds check (bits 8..15: site)
+    DEV_CANARY = 6,          // debug builds: an arena guard band was overwritten (bits 8..15: band)
 };
+
+// Debug builds (STATEKV_DEBUG_CHECKS=1) check indices before the accesses
+// marked with SKV_CHECK: a failed check records DEV_BOUNDS with its site in
+// the status word (unless a failure is already recorded) and the access is
+// skipped; no trap.
+// Release builds compile every check to `true`.
+#ifndef STATEKV_DEBUG_CHECKS
+#define STATEKV_DEBUG_CHECKS 0
+#endif
+#if STATEKV_DEBUG_CHECKS
+__device__ __forceinline__ bool skv_check(bool ok, int32_t* status, int site)
+{
+    // the status word may live in mapped host memory: a plain store, no atomic
+    if (!ok && status && *reinterpret_cast<volatile int32_t*>(status) == 0)
+        *reinterpret_cast<volatile int32_t*>(status) = DEV_BOUNDS | (site << 8);
+    return ok;
+}
+#define SKV_CHECK(cond, status, site) (::statekv::skv_check((cond), (status), (site)))
+#else
+#define SKV_CHECK(cond, status, site) true
+#endif
 
 // Tile sizes of the attention kernel: 128 query rows x 128 keys per MMA tile.
 constexpr int kBM = 128;
@@ -93,6 +116,7 @@ struct AppendParams {
     int U, T, Hkv, D;
     int row_mul;                // first row = frames * row_mul + row_add
     long long cap;
+    int32_t* status;            // debug builds: bounds-check failures
 };
 
 struct RecencyParams {
@@ -234,5 +258,17 @@ cudaError_t launch_attn(int D, const CUtensorMap& tm_sk, const CUtensorMap& tm_s
                         int U, cudaStream_t st);
 cudaError_t launch_select(const SelectParams& p, int U, cudaStream_t st);
 cudaError_t launch_append(const AppendParams& p, cudaStream_t st);
+
+// Debug builds: compares every byte of up to kMaxGuards 256-byte guard bands
+// of the arena with the fill pattern kGuardFill; a mismatch records
+// DEV_CANARY with the band's index.
+constexpr int kMaxGuards = 24;
+constexpr int kGuardBytes = 256;
+constexpr unsigned char kGuardFill = 0xA5;
+struct GuardList {
+    unsigned long long off[kMaxGuards];
+    int n;
+};
+cudaError_t launch_canary_check(const uint8_t* arena, const GuardList& g, int32_t* status, cudaStream_t st);
 
 }  // namespace statekv

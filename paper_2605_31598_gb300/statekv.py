@@ -13,7 +13,10 @@ import os
 import threading
 
 PKG = os.path.dirname(os.path.abspath(__file__))
-LIB_PATH = os.path.join(PKG, "libstatekv.so")
+# STATEKV_DEBUG=1 in the environment (before the first call) loads the debug
+# build (bounds checks and arena guard bands; build_ext.build(debug=True))
+LIB_PATH = os.path.join(PKG, "libstatekv_debug.so" if os.environ.get("STATEKV_DEBUG") == "1"
+                        else "libstatekv.so")
 
 STATEKV_OK = 0
 STATUS_NAMES = {
@@ -27,6 +30,7 @@ EXPORTED = ("statekv_arena_bytes", "statekv_init", "statekv_prefill_frame",
             "statekv_state_view", "statekv_cache_view",
             "statekv_profile_enable", "statekv_profile_read", "statekv_sync",
             "statekv_device_error", "statekv_watchdog_selftest", "statekv_frame_attention_noalloc",
+            "statekv_debug_check",
             "statekv_scores_workspace_bytes", "statekv_full_attention_scores",
             "statekv_topb_mask", "statekv_concentration_sums", "statekv_state_metrics",
             "statekv_block_workspace_bytes", "statekv_block_frame",
@@ -115,6 +119,8 @@ def lib() -> ctypes.CDLL:
             L.statekv_prefill_frames_host.argtypes = [ctypes.c_void_p, P(statekv_frame_args),
                                                       ctypes.c_int32, ctypes.c_void_p]
             L.statekv_prefill_frames_host.restype = st
+            L.statekv_debug_check.argtypes = [ctypes.c_void_p, ctypes.c_void_p]
+            L.statekv_debug_check.restype = st
             L.statekv_watchdog_selftest.argtypes = [ctypes.c_void_p, ctypes.c_void_p]
             L.statekv_watchdog_selftest.restype = st
             L.statekv_decode_step.argtypes = [ctypes.c_void_p, P(statekv_decode_args),
@@ -538,6 +544,14 @@ class StateKV:
     def device_error(self) -> int:
         """Raw device status word (0 = none); see statekv_device_error."""
         return statekv_device_error(self.handle)
+
+    def debug_check(self, stream=None) -> int:
+        """Enqueue the guard-band comparison of a debug build
+        (statekv_debug_check); STATEKV_ERR_UNSUPPORTED from a release build."""
+        import torch
+
+        st = (stream or torch.cuda.current_stream()).cuda_stream
+        return lib().statekv_debug_check(self.handle, ctypes.c_void_p(st))
 
     def watchdog_selftest(self, stream=None) -> int:
         """Enqueue the failure-detection self-test (statekv_watchdog_selftest):
