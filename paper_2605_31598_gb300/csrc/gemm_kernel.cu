@@ -420,6 +420,234 @@ __global__ void __launch_bounds__(kGThreads, 1)
     if (warp == 1) tmem_dealloc(tbase, 512);
 }
 
+
+// ---------------------------------------------------------------- thin GEMM
+// M <= 256 rows.  The roles swap: W is the A operand (128 of its rows per
+// instruction, two row blocks per unit) and the whole of X, Mp rows, the B
+// operand (N = Mp), so each 64-wide K step loads two 16 KB W tiles and one
+// X tile of Mp x 128 B, and both accumulators (TMEM columns [0, Mp) and
+// [256, 256 + Mp)) share the X tile.  One unit per CTA: nothing waits on
+// another CTA.
+constexpr int kTTileW = 128 * kGemmBK * 2;  // 16 KB: 128 rows of W x 64 K
+constexpr int kTMaxStages = 8;
+constexpr int kTBarBytes = 256;             // barriers, TMEM slot, abort flag
+constexpr int kTSmemMax = 232448;
+
+__host__ __device__ constexpr int thin_stage_bytes(int Mp) { return 2 * kTTileW + Mp * kGemmBK * 2; }
+
+__device__ __forceinline__ float silu_times(float g, float u) { return g / (1.f + expf(-g)) * u; }
+
+__global__ void __launch_bounds__(kGThreads, 1)
+    gemm_thin_tc(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_w,
+                 const ThinParams p)
+{
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+    const int S = p.stages;
+    const int stage_bytes = thin_stage_bytes(p.Mp);
+    uint64_t* bars = reinterpret_cast<uint64_t*>(sm + S * stage_bytes);
+    uint64_t* full = bars;            // stage loaded
+    uint64_t* empty = bars + S;       // stage read by its MMAs
+    uint64_t* acc_full = bars + 2 * S;
+    uint64_t* drain = acc_full + 1;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+    const int tile = blockIdx.x / p.splits, split = blockIdx.x - tile * p.splits;
+    const int ks0 = split * p.kps, ks1 = min(p.k_steps, ks0 + p.kps);
+    // W row blocks of the unit and the rows of each that are outputs
+    int wb0, wb1, nv0, nv1;
+    if (p.paired_I > 0) {
+        wb0 = 128 * tile;
+        wb1 = p.paired_I + 128 * tile;
+        nv0 = nv1 = min(128, p.paired_I - 128 * tile);
+    } else {
+        wb0 = 256 * tile;
+        wb1 = wb0 + 128;
+        nv0 = min(128, p.Nw - wb0);
+        nv1 = max(0, min(128, p.Nw - wb1));
+    }
+    const bool two = nv1 > 0;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < S; ++i) {
+            mbar_init(&full[i], 1);
+            mbar_init(&empty[i], 1);
+        }
+        mbar_init(acc_full, 1);
+        mbar_init(drain, 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (warp == 1) {
+        tmem_alloc(tmem_slot, 512);
+        tmem_relinquish();
+    }
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tbase = *tmem_slot;
+    const unsigned long long deadline = g_globaltimer() + p.watchdog_ns;
+    auto fail = [&](int site) {
+        if (atomicExch(const_cast<int*>(abort_flag), 1) == 0)
+            *reinterpret_cast<volatile int32_t*>(p.status) = DEV_TIMEOUT_GEMM | (site << 8);
+    };
+    // the next kernel may start launching (it waits for this one's completion
+    // before touching what this one writes)
+    pdl_launch_dependents();
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ TMA producer
+        if (lane == 0) {
+            tma_prefetch_desc(&tm_x);
+            tma_prefetch_desc(&tm_w);
+            const uint32_t tx = (two ? 2 : 1) * kTTileW + p.Mp * kGemmBK * 2;
+            // The weights do not depend on the previous kernel of the stream:
+            // the first ring's worth of W tiles is requested before waiting
+            // for it (a no-op unless launched programmatically), X after.
+            const int pre = min(S, ks1 - ks0);
+            for (int n = 0; n < pre; ++n) {
+                uint8_t* base = sm + n * stage_bytes;
+                mbar_arrive_expect_tx(&full[n], tx);
+                const int kc = (ks0 + n) * kGemmBK;
+                tma_load_4d(base, &tm_w, &full[n], kc, wb0, 0, 0);
+                if (two) tma_load_4d(base + kTTileW, &tm_w, &full[n], kc, wb1, 0, 0);
+            }
+            pdl_wait();
+            for (int n = 0; n < pre; ++n)
+                tma_load_4d(sm + n * stage_bytes + 2 * kTTileW, &tm_x, &full[n], (ks0 + n) * kGemmBK, 0, 0, 0);
+            int n = pre;
+            for (int ks = ks0 + pre; ks < ks1; ++ks, ++n) {
+                if (*abort_flag) break;
+                const int s = n % S, use = n / S;
+                if (use >= 1 && !g_wait(&empty[s], (use - 1) & 1, deadline)) {
+                    fail(6);
+                    break;
+                }
+                uint8_t* base = sm + s * stage_bytes;
+                mbar_arrive_expect_tx(&full[s], tx);
+                const int kc = ks * kGemmBK;
+                tma_load_4d(base, &tm_w, &full[s], kc, wb0, 0, 0);
+                if (two) tma_load_4d(base + kTTileW, &tm_w, &full[s], kc, wb1, 0, 0);
+                tma_load_4d(base + 2 * kTTileW, &tm_x, &full[s], kc, 0, 0, 0);
+            }
+            // let every copy land before the CTA's memory goes away: the last
+            // use of stage s is the largest use issued for it
+            const unsigned long long dl = g_globaltimer() + p.watchdog_ns;
+            for (int s = 0; s < S && s < n; ++s) g_wait(&full[s], ((n - 1 - s) / S) & 1, dl);
+        }
+        __syncwarp();
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            const uint32_t id = idesc_bf16_f32(128, p.Mp, false, false);
+            const uint32_t s0 = smem_addr(sm);
+            bool ok = true;
+            int n = 0;
+            for (int ks = ks0; ks < ks1; ++ks, ++n) {
+                const int s = n % S;
+                if (!(ok = g_wait(&full[s], (n / S) & 1, deadline))) break;
+                tc_fence_after();
+                const uint32_t sa = s0 + s * stage_bytes;
+                const uint64_t da0 = sdesc_sw128(sa, 16, 1024);
+                const uint64_t da1 = sdesc_sw128(sa + kTTileW, 16, 1024);
+                const uint64_t dx = sdesc_sw128(sa + 2 * kTTileW, 16, 1024);
+#pragma unroll
+                for (int kk = 0; kk < kGemmBK / 16; ++kk) {
+                    const uint32_t acc = (ks > ks0 || kk > 0) ? 1u : 0u;
+                    umma_bf16(tbase, da0 + 2 * kk, dx + 2 * kk, id, acc);
+                    if (two) umma_bf16(tbase + 256, da1 + 2 * kk, dx + 2 * kk, id, acc);
+                }
+                umma_commit(&empty[s]);
+            }
+            if (ok) umma_commit(acc_full);
+            else fail(7);
+            umma_commit(drain);
+            g_wait(drain, 0, g_globaltimer() + p.watchdog_ns);
+        }
+        __syncwarp();
+    } else {
+        // ------------------------------------------------------------ epilogue (warps 2..5)
+        // Thread = W row (TMEM lane); each 32-column TMEM load holds 32 rows of
+        // X for it.  The values go to shared memory as one output row per X
+        // row (the stage ring is free once the last MMA has completed), then
+        // one lane per warp copies whole rows out with bulk stores: a few
+        // large writes per row instead of one 128-byte store per warp and X
+        // row, which left the kernel's completion waiting long after its
+        // last instruction.
+        const int quad = warp & 3;
+        const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
+        const int r = quad * 32 + lane;
+        const int chunks = (p.M + 31) / 32;
+        const bool ok = __all_sync(0xffffffffu, g_wait(acc_full, 0, deadline));
+        if (ok) {
+            tc_fence_after();
+            if (p.act) {
+                __nv_bfloat16* stage = reinterpret_cast<__nv_bfloat16*>(sm);  // [M][128]
+#pragma unroll 1
+                for (int c = 0; c < chunks; ++c) {
+                    float g[32], u[32];
+                    tmem_ld32(tbase + lane_off + 32 * c, g);
+                    tmem_ld32(tbase + lane_off + 256 + 32 * c, u);
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) {
+                        const int t = 32 * c + j;
+                        if (t < p.M) {
+                            // gate and up are rounded to bf16 first, as when
+                            // they are stored between kernels
+                            const float gb = __bfloat162float(__float2bfloat16_rn(g[j]));
+                            const float ub = __bfloat162float(__float2bfloat16_rn(u[j]));
+                            stage[t * 128 + r] = __float2bfloat16_rn(silu_times(gb, ub));
+                        }
+                    }
+                }
+                fence_proxy_async_smem();
+                epi_bar();
+                if (lane == 0) {
+                    const uint32_t bytes = static_cast<uint32_t>(nv0) * 2;
+                    for (int t = quad; t < p.M; t += 4)
+                        bulk_store(p.act + static_cast<size_t>(t) * p.paired_I + 128 * tile, stage + t * 128, bytes);
+                    bulk_commit();
+                    bulk_wait();
+                }
+            } else {
+                float* stage = reinterpret_cast<float*>(sm);  // [M][128]
+                for (int b = 0; b < (two ? 2 : 1); ++b) {
+#pragma unroll 1
+                    for (int c = 0; c < chunks; ++c) {
+                        float v[32];
+                        tmem_ld32(tbase + lane_off + 256 * b + 32 * c, v);
+                        tmem_ld_wait();
+#pragma unroll
+                        for (int j = 0; j < 32; ++j) {
+                            const int t = 32 * c + j;
+                            if (t < p.M) stage[t * 128 + r] = v[j];
+                        }
+                    }
+                    fence_proxy_async_smem();
+                    epi_bar();
+                    if (lane == 0) {
+                        const uint32_t bytes = static_cast<uint32_t>(b ? nv1 : nv0) * 4;
+                        float* dst = p.partials + static_cast<size_t>(split) * p.M * p.Nw + (b ? wb1 : wb0);
+                        for (int t = quad; t < p.M; t += 4)
+                            bulk_store(dst + static_cast<size_t>(t) * p.Nw, stage + t * 128, bytes);
+                        bulk_commit();
+                        bulk_wait();  // the stage is rewritten for the next block
+                    }
+                    epi_bar();
+                }
+            }
+        } else {
+            fail(8);
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) tmem_dealloc(tbase, 512);
+}
+
 }  // namespace
 
 GemmPlan gemm_plan(int M, int N, int K, int sms)
@@ -463,6 +691,57 @@ cudaError_t launch_gemm(const CUtensorMap& tm_x, const CUtensorMap& tm_w, const 
     void* args[] = {&a, &b, &q};
     return cudaLaunchCooperativeKernel(reinterpret_cast<const void*>(gemm_bf16_tc), dim3(grid),
                                        dim3(kGThreads), args, kGAlloc, st);
+}
+
+ThinPlan thin_plan(int M, int Nw, int K, int sms, int paired_I)
+{
+    ThinPlan g{};
+    g.Mp = (M + 15) / 16 * 16;
+    g.tiles = paired_I > 0 ? (paired_I + 127) / 128 : (Nw + 255) / 256;
+    g.k_steps = (K + kGemmBK - 1) / kGemmBK;
+    // split K while the tiles alone leave SMs idle, into as many ranges as
+    // keep every unit in one wave
+    int splits = g.tiles >= sms ? 1 : sms / g.tiles;
+    splits = splits < 1 ? 1 : (splits > g.k_steps ? g.k_steps : splits);
+    g.kps = (g.k_steps + splits - 1) / splits;
+    g.splits = (g.k_steps + g.kps - 1) / g.kps;
+    g.units = g.tiles * g.splits;
+    const int sb = thin_stage_bytes(g.Mp);
+    g.stages = (kTSmemMax - 1024 - kTBarBytes) / sb;
+    g.stages = g.stages > kTMaxStages ? kTMaxStages : g.stages;
+    g.smem = static_cast<size_t>(g.stages) * sb + kTBarBytes + 1024;
+    g.partial_bytes = (paired_I > 0 && g.splits == 1) ? 0 : static_cast<size_t>(g.splits) * M * Nw * 4;
+    return g;
+}
+
+cudaError_t thin_prepare()
+{
+    return cudaFuncSetAttribute(gemm_thin_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, kTSmemMax);
+}
+
+cudaError_t launch_thin_gemm(const CUtensorMap& tm_x, const CUtensorMap& tm_w, const ThinParams& p,
+                             size_t smem, cudaStream_t st)
+{
+    const int units = (p.paired_I > 0 ? (p.paired_I + 127) / 128 : (p.Nw + 255) / 256) * p.splits;
+    if (units <= 0) return cudaSuccess;
+    if (p.M < 1 || p.M > kThinMaxRows || p.Mp != (p.M + 15) / 16 * 16 || p.stages < 2 ||
+        p.stages > kTMaxStages || (p.act && (p.paired_I <= 0 || p.splits != 1)) || (!p.act && !p.partials) ||
+        (p.paired_I > 0 ? (p.paired_I & 7) : (p.Nw & 3)) != 0 ||
+        static_cast<size_t>(p.M) * 128 * 4 > static_cast<size_t>(p.stages) * thin_stage_bytes(p.Mp) ||
+        smem > static_cast<size_t>(kTSmemMax) ||
+        static_cast<size_t>(p.stages) * thin_stage_bytes(p.Mp) + kTBarBytes + 1024 > smem)
+        return cudaErrorInvalidValue;
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3(units);
+    cfg.blockDim = dim3(kGThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, gemm_thin_tc, tm_x, tm_w, p);
 }
 
 }  // namespace statekv

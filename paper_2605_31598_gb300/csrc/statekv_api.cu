@@ -605,7 +605,7 @@ statekv_status statekv_init(const statekv_config* cfg, void* device_arena, size_
 
     const int D = cfg->head_dim, B = cfg->state_capacity, Hkv = cfg->num_kv_heads;
     bool ok = attn_prepare(D) == cudaSuccess && select_prepare() == cudaSuccess &&
-              gemm_prepare() == cudaSuccess &&
+              gemm_prepare() == cudaSuccess && thin_prepare() == cudaSuccess &&
               decode_prepare() == cudaSuccess;
     if (ok && B > 0) {
         const cuuint64_t dims[4] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(B),
@@ -825,11 +825,18 @@ BlockBufs block_bufs(const statekv_config& c, const statekv_block_config& b, int
     o.attn = take(rows * hq * d * 2);
     o.gu = take(rows * 2 * static_cast<size_t>(b.intermediate) * 2);
     o.act = take(rows * static_cast<size_t>(b.intermediate) * 2);
-    // split-K partials of the largest split GEMM, and their tile counters
+    // split-K partials of the largest split GEMM, and the tile counters of
+    // the cooperative path (rows above kThinMaxRows)
     int nk[4][2];
     block_gemm_shapes(c, b, nk);
     size_t part = 0;
-    for (auto& g : nk) part = std::max(part, gemm_plan(static_cast<int>(rows), g[0], g[1], device_sm_count()).partial_bytes);
+    const int sms = device_sm_count();
+    for (int i = 0; i < 4; ++i) {
+        const int M = static_cast<int>(rows), N = nk[i][0], K = nk[i][1];
+        part = std::max(part, M <= kThinMaxRows
+                                  ? thin_plan(M, N, K, sms, i == 2 ? b.intermediate : 0).partial_bytes
+                                  : gemm_plan(M, N, K, sms).partial_bytes);
+    }
     o.gemm_part = take(part);
     o.gemm_cnt = take(static_cast<size_t>(4) * c.num_layers * kGemmCounterRegion * 4);
     o.total = off;
@@ -972,14 +979,64 @@ statekv_status statekv_block_frame(statekv_handle* h, const statekv_block_config
         gp.watchdog_ns = 1000000ull * (c.watchdog_ms ? c.watchdog_ms : 2000u);
         return timed(h, 3, st, [&] { return launch_gemm(tx, tw, gp, sms, st); }) == cudaSuccess;
     };
+    // Up to kThinMaxRows rows (one stream's frame) the projections run as thin
+    // GEMMs: each writes split-K partials (or, for gate/up unsplit, SiLU * up
+    // directly) and the next elementwise kernel adds them up -- the QKV sum
+    // in the RoPE kernel, the output and down projections' sums in the
+    // residual update, which also computes the following RMSNorm (the next
+    // layer's, when the call covers it).
+    float* part = reinterpret_cast<float*>(ws + bb.gemm_part);
+    const unsigned long long wd_ns = 1000000ull * (c.watchdog_ms ? c.watchdog_ms : 2000u);
+    auto thin_gemm = [&](const void* X, const void* Wt, int Nw, int K, int paired_I,
+                         __nv_bfloat16* act, int* splits_out) {
+        const ThinPlan g = thin_plan(rows, Nw, K, sms, paired_I);
+        CUtensorMap tx, tw;
+        const cuuint64_t dx[4] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(rows), 1, 1};
+        const cuuint64_t dw[4] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(Nw), 1, 1};
+        const cuuint64_t sx[3] = {static_cast<cuuint64_t>(K) * 2, static_cast<cuuint64_t>(K) * rows * 2,
+                                  static_cast<cuuint64_t>(K) * rows * 2};
+        const cuuint64_t sw[3] = {static_cast<cuuint64_t>(K) * 2, static_cast<cuuint64_t>(K) * Nw * 2,
+                                  static_cast<cuuint64_t>(K) * Nw * 2};
+        const cuuint32_t bx[4] = {static_cast<cuuint32_t>(kGemmBK), static_cast<cuuint32_t>(g.Mp), 1, 1};
+        const cuuint32_t bw[4] = {static_cast<cuuint32_t>(kGemmBK), 128, 1, 1};
+        if (!encode_4d(&tx, X, dx, sx, bx) || !encode_4d(&tw, Wt, dw, sw, bw)) return false;
+        ThinParams tp{};
+        tp.M = rows;
+        tp.Mp = g.Mp;
+        tp.Nw = Nw;
+        tp.K = K;
+        tp.k_steps = g.k_steps;
+        tp.kps = g.kps;
+        tp.splits = g.splits;
+        tp.stages = g.stages;
+        tp.paired_I = paired_I;
+        tp.act = (act && g.splits == 1) ? act : nullptr;
+        tp.partials = tp.act ? nullptr : part;
+        tp.status = h->status_dev;
+        tp.watchdog_ns = wd_ns;
+        *splits_out = tp.act ? 0 : g.splits;
+        return timed(h, 3, st, [&] { return launch_thin_gemm(tx, tw, tp, g.smem, st); }) == cudaSuccess;
+    };
+    const bool thin = rows <= kThinMaxRows;
     for (int l = layer_begin; l < layer_begin + layer_count; ++l) {
         const statekv_block_weights& w = weights[l];
-        if (timed(h, 4, st, [&] {
+        const bool last = l + 1 == layer_begin + layer_count;
+        int splits = 0;
+        // the thin path's previous layer already normalised x into h
+        if ((!thin || l == layer_begin) &&
+            timed(h, 4, st, [&] {
                 return launch_rmsnorm(x, static_cast<const __nv_bfloat16*>(w.norm_attn), b.rms_eps,
                                       buf(bb.h), rows, H, st);
             }) != cudaSuccess)
             return STATEKV_ERR_CUDA;
-        if (!gemm(buf(bb.h), w.w_qkv, w.b_qkv, buf(bb.qkv), false, W, H)) return STATEKV_ERR_CUDA;
+        if (thin) {
+            if (!thin_gemm(buf(bb.h), w.w_qkv, W, H, 0, nullptr, &splits)) return STATEKV_ERR_CUDA;
+            rp.part = part;
+            rp.splits = splits;
+            rp.bias = static_cast<const __nv_bfloat16*>(w.b_qkv);
+        } else if (!gemm(buf(bb.h), w.w_qkv, w.b_qkv, buf(bb.qkv), false, W, H)) {
+            return STATEKV_ERR_CUDA;
+        }
         rp.layer = l;
         if (timed(h, 4, st, [&] { return launch_qkv_rope(rp, st); }) != cudaSuccess)
             return STATEKV_ERR_CUDA;
@@ -988,6 +1045,30 @@ statekv_status statekv_block_frame(statekv_handle* h, const statekv_block_config
         a.layer_count = 1;
         const statekv_status r = run_step(h, a, st);
         if (r != STATEKV_OK) return r;
+        if (thin) {
+            if (!thin_gemm(buf(bb.attn), w.w_o, H, Hq * d, 0, nullptr, &splits) ||
+                timed(h, 4, st, [&] {
+                    return launch_residual_norm(part, splits, x,
+                                                static_cast<const __nv_bfloat16*>(w.norm_mlp),
+                                                b.rms_eps, buf(bb.h), rows, H, st);
+                }) != cudaSuccess)
+                return STATEKV_ERR_CUDA;
+            if (!thin_gemm(buf(bb.h), w.w_gate_up, 2 * I, H, I, buf(bb.act), &splits))
+                return STATEKV_ERR_CUDA;
+            if (splits > 0 &&
+                timed(h, 4, st, [&] { return launch_silu_partials(part, splits, buf(bb.act), rows, I, st); }) !=
+                    cudaSuccess)
+                return STATEKV_ERR_CUDA;
+            const __nv_bfloat16* next_norm =
+                last ? nullptr : static_cast<const __nv_bfloat16*>(weights[l + 1].norm_attn);
+            if (!thin_gemm(buf(bb.act), w.w_down, H, I, 0, nullptr, &splits) ||
+                timed(h, 4, st, [&] {
+                    return launch_residual_norm(part, splits, x, next_norm, b.rms_eps, buf(bb.h), rows,
+                                                H, st);
+                }) != cudaSuccess)
+                return STATEKV_ERR_CUDA;
+            continue;
+        }
         if (!gemm(buf(bb.attn), w.w_o, nullptr, x, true, H, Hq * d)) return STATEKV_ERR_CUDA;
         if (timed(h, 4, st, [&] {
                 return launch_rmsnorm(x, static_cast<const __nv_bfloat16*>(w.norm_mlp), b.rms_eps,

@@ -169,3 +169,61 @@ def test_block_ragged_widths_many_streams():
     stats = {}
     worst = run_block_parity(shape, BlockShape(136, 200, weight_std=0.08), 3, stats=stats)
     print("ragged block worst |dx|", worst, stats)
+
+
+@pytest.mark.gpu
+def test_block_ragged_widths_thin_rows():
+    """At most 256 rows (here 4 streams x 49 tokens = 196, one stream's row
+    count at 7B shape) the projections run as thin GEMMs writing split-K
+    partials that the RoPE, residual and SiLU kernels add up.  Hidden 136 and
+    MLP 200 give ragged W row blocks, a ragged last K step, and a gate/up
+    projection with only two row-block pairs, so it splits K and its SiLU
+    reads partials."""
+    from paper_2605_31598_gb300.inputs import BlockShape
+
+    _need_gpu()
+    shape = Shape(4, 2, 64, 49, 64, 3, num_layers=2, num_streams=4)
+    stats = {}
+    worst = run_block_parity(shape, BlockShape(136, 200, weight_std=0.08), 3, stats=stats)
+    print("ragged thin block worst |dx|", worst, stats)
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("streams,tokens", [(1, 196), (2, 16)])
+def test_block_multi_layer_call_equals_layer_calls(streams, tokens):
+    """One call over every layer (where the thin path computes layer l+1's
+    input RMSNorm inside layer l's residual update) gives bit for bit the
+    hidden states, states and caches of one call per layer."""
+    from paper_2605_31598_gb300.inputs import BlockShape
+
+    _need_gpu()
+    shape = Shape(4, 2, 64, tokens, 64, 3, num_layers=3, num_streams=streams)
+    block = BlockShape(256, 512, weight_std=0.08)
+    bc = statekv_block_config(block.hidden, block.intermediate, block.rms_eps, block.rope_theta,
+                              1.0, 0)
+    wts = block_weights(shape, block, device="cuda")
+    warr = block_weights_array(wts)
+    engs = [StateKV(make_config(shape)) for _ in range(2)]
+    wss = [torch.empty(e.block_workspace_bytes(bc), dtype=torch.uint8, device="cuda") for e in engs]
+    for n in range(1, 4):
+        x = block_input(shape, block, n, device="cuda")
+        y_all = torch.empty_like(x)
+        assert engs[0].block_frame(bc, warr, x, y_all, wss[0]) == 0
+        y = x.clone()
+        for l in range(shape.num_layers):
+            y_next = torch.empty_like(y)
+            assert engs[1].block_frame(bc, warr, y, y_next, wss[1], layer_begin=l, layer_count=1) == 0
+            y = y_next
+        torch.cuda.synchronize()
+        assert torch.equal(y_all, y), f"frame {n}"
+        for s in range(streams):
+            for l in range(shape.num_layers):
+                (ka, va, pa, _), (kb, vb, pb, _) = engs[0].state(s, l), engs[1].state(s, l)
+                assert torch.equal(pa, pb)
+                used = pa >= 0
+                assert torch.equal(ka[used], kb[used]) and torch.equal(va[used], vb[used])
+                ca, cb = engs[0].cache(s, l), engs[1].cache(s, l)
+                assert ca[2].length == cb[2].length == n * tokens
+                assert torch.equal(ca[0][:, :n * tokens], cb[0][:, :n * tokens])
+                assert torch.equal(ca[1][:, :n * tokens], cb[1][:, :n * tokens])
+    assert engs[0].sync() == 0 and engs[1].sync() == 0
