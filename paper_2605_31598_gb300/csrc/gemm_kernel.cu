@@ -22,6 +22,8 @@
 // the accumulators (one TMEM lane quadrant each, thread = row) and write D or
 // the fp32 partials.  Every mbarrier wait is bounded by the watchdog; on
 // expiry the CTA records DEV_TIMEOUT_GEMM, drains and exits.
+#include <algorithm>
+
 #include "sm103_ptx.cuh"
 #include "statekv_kernels.cuh"
 
@@ -423,19 +425,229 @@ __global__ void __launch_bounds__(kGThreads, 1)
 
 // ---------------------------------------------------------------- thin GEMM
 // M <= 256 rows.  The roles swap: W is the A operand (128 of its rows per
-// instruction, two row blocks per unit) and the whole of X, Mp rows, the B
-// operand (N = Mp), so each 64-wide K step loads two 16 KB W tiles and one
-// X tile of Mp x 128 B, and both accumulators (TMEM columns [0, Mp) and
-// [256, 256 + Mp)) share the X tile.  One unit per CTA: nothing waits on
-// another CTA.
+// instruction) and all of X, Mp rows, the B operand (N = Mp).  A unit is one
+// or two 128-row blocks of W -- two consecutive blocks, or for the gate/up
+// projection a gate block and the matching up block -- over one range of K;
+// the blocks share each X tile, so two blocks halve the X traffic per weight
+// byte.  Each 64-wide K step loads the unit's W tiles (16 KB each) and one X
+// tile of Mp x 128 B.  The `splits` units of a block (pair) are the CTAs of
+// one thread-block cluster: after the main loop each stages its fp32
+// accumulators in its own shared memory (the stage ring is idle by then; the
+// staging area may reach past it), and after a cluster barrier CTA r adds
+// rows [r M / S, (r + 1) M / S) over the S CTAs' copies in rank order,
+// applies the epilogue and writes bf16.  No partial sum leaves the cluster
+// and the result does not depend on timing.
 constexpr int kTTileW = 128 * kGemmBK * 2;  // 16 KB: 128 rows of W x 64 K
 constexpr int kTMaxStages = 8;
 constexpr int kTBarBytes = 256;             // barriers, TMEM slot, abort flag
 constexpr int kTSmemMax = 232448;
+constexpr int kTRegionMax = kTSmemMax - 1024 - kTBarBytes;  // ring / staging area
+// Every plan uses more than half of an SM's shared memory, so each SM holds
+// one CTA and no CTA waits on another cluster's for TMEM.
+static_assert(kTMaxStages * (kTTileW + 16 * kGemmBK * 2) > 233472 / 2, "one CTA per SM");
 
-__host__ __device__ constexpr int thin_stage_bytes(int Mp) { return 2 * kTTileW + Mp * kGemmBK * 2; }
+__host__ __device__ constexpr int thin_stage_bytes(int Mp, int wblocks)
+{
+    return wblocks * kTTileW + Mp * kGemmBK * 2;
+}
 
-__device__ __forceinline__ float silu_times(float g, float u) { return g / (1.f + expf(-g)) * u; }
+__host__ __device__ constexpr size_t thin_staging_bytes(int M, int wblocks)
+{
+    return static_cast<size_t>(wblocks) * M * 128 * 4;
+}
+
+// SiLU(g) * u with the fast exponential and division: straight-line code the
+// compiler interleaves across a thread's 32 values (the epilogue runs one
+// warp per SM sub-partition, so it is bound by dependent-instruction latency;
+// the library expf / IEEE division branch and serialise it).  Relative error
+// ~1e-6, far below the bf16 rounding of the result.
+__device__ __forceinline__ float silu_times(float g, float u) { return __fdividef(g, 1.f + __expf(-g)) * u; }
+
+// Round-to-nearest-even to bf16 of a finite float, as integer arithmetic on
+// its bits (full-rate ALU work, where the conversion instructions are not):
+// the same result as __float2bfloat16_rn for every finite input.
+__device__ __forceinline__ uint32_t bf16_rne_bits(float x)
+{
+    const uint32_t u = __float_as_uint(x);
+    return (u + 0x7FFFu + ((u >> 16) & 1u)) >> 16;
+}
+
+__device__ __forceinline__ float bf16_round(float x) { return __uint_as_float(bf16_rne_bits(x) << 16); }
+
+__device__ __forceinline__ void add4(float4& a, const float4& b)
+{
+    a.x += b.x;
+    a.y += b.y;
+    a.z += b.z;
+    a.w += b.w;
+}
+
+// four consecutive staged values of row t, summed over the cluster's S CTAs
+// in rank order (stage: fp32 [rows][128] at shared address `base` in every
+// CTA).  All S loads are issued before the first addition.
+template <int S>
+__device__ __forceinline__ float4 cluster_sum4(uint32_t base, int t, int col)
+{
+    const uint32_t a = base + static_cast<uint32_t>(t * 128 + col) * 4u;
+    float4 v[S];
+#pragma unroll
+    for (int r = 0; r < S; ++r) v[r] = ld_dsmem_f4(dsmem_addr(a, r));
+#pragma unroll
+    for (int r = 1; r < S; ++r) add4(v[0], v[r]);
+    return v[0];
+}
+
+__device__ __forceinline__ void store_bf16x4(__nv_bfloat16* dst, float a, float b, float c, float d)
+{
+    *reinterpret_cast<uint2*>(dst) = make_uint2(pack_bf16x2(a, b), pack_bf16x2(c, d));
+}
+
+// Residual epilogue of one staged block: out[t][wb + j] += sum, rows
+// [t0, t1), 4 columns per thread (e = 0..127: column group e mod 32, row
+// phase e / 32).  Rows go in batches whose loads (about 8 in flight per thread)
+// are all issued before the first use.
+template <int S>
+__device__ __forceinline__ void epi_residual(const ThinParams& p, uint32_t sbase, int wb, int nv, int t0,
+                                             int t1, int e)
+{
+    constexpr int kB = 8 / S > 0 ? 8 / S : 1;
+    const int j4 = 4 * (e & 31);
+    if (j4 >= nv) return;
+    for (int tb = t0 + (e >> 5); tb < t1; tb += 4 * kB) {
+        uint2 old[kB];
+        float4 a[kB];
+#pragma unroll
+        for (int b = 0; b < kB; ++b)
+            if (tb + 4 * b < t1)
+                old[b] = *reinterpret_cast<const uint2*>(p.out + static_cast<size_t>(tb + 4 * b) * p.Nw + wb + j4);
+#pragma unroll
+        for (int b = 0; b < kB; ++b)
+            if (tb + 4 * b < t1) a[b] = cluster_sum4<S>(sbase, tb + 4 * b, j4);
+#pragma unroll
+        for (int b = 0; b < kB; ++b)
+            if (tb + 4 * b < t1) {
+                const float2 lo = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&old[b].x));
+                const float2 hi = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&old[b].y));
+                store_bf16x4(p.out + static_cast<size_t>(tb + 4 * b) * p.Nw + wb + j4, lo.x + a[b].x,
+                             lo.y + a[b].y, hi.x + a[b].z, hi.y + a[b].w);
+            }
+    }
+}
+
+// QKV epilogue of one staged block (W rows wb.., whole heads): bias added and
+// rounded to bf16 where the projection would be stored, q and k heads
+// rotated by the rows' (cos, sin) table, written to q / k / v in [M][H][d].
+// 16 threads per row: thread g takes pairs (k, k + d/2), k = 4 (g mod d/8)
+// .. +3, of the block's head g / (d/8).
+template <int S>
+__device__ __forceinline__ void epi_qkv(const ThinParams& p, uint32_t sbase, int wb, int t0, int t1, int e)
+{
+    constexpr int kB = 8 / S > 0 ? 8 / S : 1;
+    const int half = p.d / 2, gph = half / 4;  // 4-pair groups per head
+    const int g = e & 15, lh = g / gph, k = 4 * (g - lh * gph);
+    const int c1 = lh * p.d + k, f1 = wb + c1;  // block column, W row of the first value
+    if (f1 >= p.Nw) return;
+    const int head = f1 / p.d;
+    const bool rotate = head < p.Hq + p.Hkv;
+    __nv_bfloat16* dst0 = head < p.Hq ? p.q + static_cast<size_t>(head) * p.d
+                        : rotate      ? p.k + static_cast<size_t>(head - p.Hq) * p.d
+                                      : p.v + static_cast<size_t>(head - p.Hq - p.Hkv) * p.d;
+    const int row_stride = (head < p.Hq ? p.Hq : p.Hkv) * p.d;
+    float b1[4], b2[4];  // this thread's bias values, the same for every row
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        b1[i] = p.bias ? __bfloat162float(p.bias[f1 + i]) : 0.f;
+        b2[i] = p.bias ? __bfloat162float(p.bias[f1 + half + i]) : 0.f;
+    }
+    for (int tb = t0 + (e >> 4); tb < t1; tb += 8 * kB) {
+        float4 a1[kB], a2[kB], cs[kB][2];
+#pragma unroll
+        for (int b = 0; b < kB; ++b) {
+            const int t = tb + 8 * b;
+            if (t < t1 && rotate) {
+                const float4* r4 = reinterpret_cast<const float4*>(p.rope + static_cast<size_t>(t) * half + k);
+                cs[b][0] = r4[0];  // (cos, sin) of pairs k, k + 1
+                cs[b][1] = r4[1];  // of pairs k + 2, k + 3
+            }
+        }
+#pragma unroll
+        for (int b = 0; b < kB; ++b) {
+            const int t = tb + 8 * b;
+            if (t < t1) {
+                a1[b] = cluster_sum4<S>(sbase, t, c1);
+                a2[b] = cluster_sum4<S>(sbase, t, c1 + half);
+            }
+        }
+#pragma unroll
+        for (int b = 0; b < kB; ++b) {
+            const int t = tb + 8 * b;
+            if (t >= t1) continue;
+            float x1[4] = {a1[b].x, a1[b].y, a1[b].z, a1[b].w}, x2[4] = {a2[b].x, a2[b].y, a2[b].z, a2[b].w};
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                x1[i] = bf16_round(x1[i] + b1[i]);
+                x2[i] = bf16_round(x2[i] + b2[i]);
+            }
+            if (rotate) {
+                const float c[4] = {cs[b][0].x, cs[b][0].z, cs[b][1].x, cs[b][1].z};
+                const float sn[4] = {cs[b][0].y, cs[b][0].w, cs[b][1].y, cs[b][1].w};
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const float o1 = x1[i] * c[i] - x2[i] * sn[i];
+                    const float o2 = x2[i] * c[i] + x1[i] * sn[i];
+                    x1[i] = o1;
+                    x2[i] = o2;
+                }
+            }
+            __nv_bfloat16* dst = dst0 + static_cast<size_t>(t) * row_stride;
+            store_bf16x4(dst + k, x1[0], x1[1], x1[2], x1[3]);
+            store_bf16x4(dst + k + half, x2[0], x2[1], x2[2], x2[3]);
+        }
+    }
+}
+
+// SiLU * up from the staged gate (sbase) and up (ubase) blocks, summed over
+// the cluster: out[t][col0 + j] for j < nv (layout as epi_residual's).
+template <int S>
+__device__ __forceinline__ void epi_silu(const ThinParams& p, uint32_t sbase, uint32_t ubase, int col0, int nv,
+                                         int t0, int t1, int e)
+{
+    constexpr int kB = 8 / S > 0 ? 8 / S : 1;
+    const int j4 = 4 * (e & 31);
+    if (j4 >= nv) return;
+    for (int tb = t0 + (e >> 5); tb < t1; tb += 4 * kB) {
+        float4 g[kB], u[kB];
+#pragma unroll
+        for (int b = 0; b < kB; ++b)
+            if (tb + 4 * b < t1) {
+                g[b] = cluster_sum4<S>(sbase, tb + 4 * b, j4);
+                u[b] = cluster_sum4<S>(ubase, tb + 4 * b, j4);
+            }
+#pragma unroll
+        for (int b = 0; b < kB; ++b)
+            if (tb + 4 * b < t1)
+                store_bf16x4(p.out + static_cast<size_t>(tb + 4 * b) * p.paired_I + col0 + j4,
+                             silu_times(bf16_round(g[b].x), bf16_round(u[b].x)),
+                             silu_times(bf16_round(g[b].y), bf16_round(u[b].y)),
+                             silu_times(bf16_round(g[b].z), bf16_round(u[b].z)),
+                             silu_times(bf16_round(g[b].w), bf16_round(u[b].w)));
+    }
+}
+
+// Part 2 of the epilogue for a cluster of S CTAs (S in {1, 2, 4, 8}).
+template <int S>
+__device__ __forceinline__ void epi_part2(const ThinParams& p, uint32_t base, uint32_t blk, int nacc, int wb0,
+                                          int wb1, int nv0, int nv1, int t0, int t1, int e)
+{
+    if (p.op == kThinSilu) {
+        epi_silu<S>(p, base, base + blk, wb0, nv0, t0, t1, e);
+        return;
+    }
+    for (int a = 0; a < nacc; ++a) {
+        if (p.op == kThinResidual) epi_residual<S>(p, base + a * blk, a ? wb1 : wb0, a ? nv1 : nv0, t0, t1, e);
+        else epi_qkv<S>(p, base + a * blk, a ? wb1 : wb0, t0, t1, e);
+    }
+}
 
 __global__ void __launch_bounds__(kGThreads, 1)
     gemm_thin_tc(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_w,
@@ -444,9 +656,11 @@ __global__ void __launch_bounds__(kGThreads, 1)
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
+    const bool paired = p.paired_I > 0;
     const int S = p.stages;
-    const int stage_bytes = thin_stage_bytes(p.Mp);
-    uint64_t* bars = reinterpret_cast<uint64_t*>(sm + S * stage_bytes);
+    const int stage_bytes = thin_stage_bytes(p.Mp, p.wblocks);
+    const int x_off = p.wblocks * kTTileW;  // the X tile's offset in a stage
+    uint64_t* bars = reinterpret_cast<uint64_t*>(sm + p.region);
     uint64_t* full = bars;            // stage loaded
     uint64_t* empty = bars + S;       // stage read by its MMAs
     uint64_t* acc_full = bars + 2 * S;
@@ -454,21 +668,21 @@ __global__ void __launch_bounds__(kGThreads, 1)
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
-    const int tile = blockIdx.x / p.splits, split = blockIdx.x - tile * p.splits;
+    const int tile = blockIdx.x / p.splits, split = blockIdx.x - tile * p.splits;  // split = cluster rank
     const int ks0 = split * p.kps, ks1 = min(p.k_steps, ks0 + p.kps);
-    // W row blocks of the unit and the rows of each that are outputs
+    // the unit's W row blocks and how many of their rows are outputs
     int wb0, wb1, nv0, nv1;
-    if (p.paired_I > 0) {
+    if (paired) {
         wb0 = 128 * tile;
-        wb1 = p.paired_I + 128 * tile;
-        nv0 = nv1 = min(128, p.paired_I - 128 * tile);
+        wb1 = p.paired_I + wb0;
+        nv0 = nv1 = min(128, p.paired_I - wb0);
     } else {
-        wb0 = 256 * tile;
+        wb0 = 128 * p.wblocks * tile;
         wb1 = wb0 + 128;
         nv0 = min(128, p.Nw - wb0);
-        nv1 = max(0, min(128, p.Nw - wb1));
+        nv1 = p.wblocks == 2 ? max(0, min(128, p.Nw - wb1)) : 0;
     }
-    const bool two = nv1 > 0;
+    const int nacc = nv1 > 0 ? 2 : 1;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (threadIdx.x == 0) {
@@ -497,12 +711,13 @@ __global__ void __launch_bounds__(kGThreads, 1)
     // before touching what this one writes)
     pdl_launch_dependents();
 
+    bool ok = true;
     if (warp == 0) {
         // ------------------------------------------------------------ TMA producer
         if (lane == 0) {
             tma_prefetch_desc(&tm_x);
             tma_prefetch_desc(&tm_w);
-            const uint32_t tx = (two ? 2 : 1) * kTTileW + p.Mp * kGemmBK * 2;
+            const uint32_t tx = nacc * kTTileW + p.Mp * kGemmBK * 2;
             // The weights do not depend on the previous kernel of the stream:
             // the first ring's worth of W tiles is requested before waiting
             // for it (a no-op unless launched programmatically), X after.
@@ -512,11 +727,11 @@ __global__ void __launch_bounds__(kGThreads, 1)
                 mbar_arrive_expect_tx(&full[n], tx);
                 const int kc = (ks0 + n) * kGemmBK;
                 tma_load_4d(base, &tm_w, &full[n], kc, wb0, 0, 0);
-                if (two) tma_load_4d(base + kTTileW, &tm_w, &full[n], kc, wb1, 0, 0);
+                if (nacc == 2) tma_load_4d(base + kTTileW, &tm_w, &full[n], kc, wb1, 0, 0);
             }
             pdl_wait();
             for (int n = 0; n < pre; ++n)
-                tma_load_4d(sm + n * stage_bytes + 2 * kTTileW, &tm_x, &full[n], (ks0 + n) * kGemmBK, 0, 0, 0);
+                tma_load_4d(sm + n * stage_bytes + x_off, &tm_x, &full[n], (ks0 + n) * kGemmBK, 0, 0, 0);
             int n = pre;
             for (int ks = ks0 + pre; ks < ks1; ++ks, ++n) {
                 if (*abort_flag) break;
@@ -529,11 +744,11 @@ __global__ void __launch_bounds__(kGThreads, 1)
                 mbar_arrive_expect_tx(&full[s], tx);
                 const int kc = ks * kGemmBK;
                 tma_load_4d(base, &tm_w, &full[s], kc, wb0, 0, 0);
-                if (two) tma_load_4d(base + kTTileW, &tm_w, &full[s], kc, wb1, 0, 0);
-                tma_load_4d(base + 2 * kTTileW, &tm_x, &full[s], kc, 0, 0, 0);
+                if (nacc == 2) tma_load_4d(base + kTTileW, &tm_w, &full[s], kc, wb1, 0, 0);
+                tma_load_4d(base + x_off, &tm_x, &full[s], kc, 0, 0, 0);
             }
-            // let every copy land before the CTA's memory goes away: the last
-            // use of stage s is the largest use issued for it
+            // let every copy land before the stages are reused or the CTA's
+            // memory goes away: the last use of stage s is the largest one issued
             const unsigned long long dl = g_globaltimer() + p.watchdog_ns;
             for (int s = 0; s < S && s < n; ++s) g_wait(&full[s], ((n - 1 - s) / S) & 1, dl);
         }
@@ -543,7 +758,6 @@ __global__ void __launch_bounds__(kGThreads, 1)
         if (lane == 0) {
             const uint32_t id = idesc_bf16_f32(128, p.Mp, false, false);
             const uint32_t s0 = smem_addr(sm);
-            bool ok = true;
             int n = 0;
             for (int ks = ks0; ks < ks1; ++ks, ++n) {
                 const int s = n % S;
@@ -552,12 +766,12 @@ __global__ void __launch_bounds__(kGThreads, 1)
                 const uint32_t sa = s0 + s * stage_bytes;
                 const uint64_t da0 = sdesc_sw128(sa, 16, 1024);
                 const uint64_t da1 = sdesc_sw128(sa + kTTileW, 16, 1024);
-                const uint64_t dx = sdesc_sw128(sa + 2 * kTTileW, 16, 1024);
+                const uint64_t dx = sdesc_sw128(sa + x_off, 16, 1024);
 #pragma unroll
                 for (int kk = 0; kk < kGemmBK / 16; ++kk) {
                     const uint32_t acc = (ks > ks0 || kk > 0) ? 1u : 0u;
                     umma_bf16(tbase, da0 + 2 * kk, dx + 2 * kk, id, acc);
-                    if (two) umma_bf16(tbase + 256, da1 + 2 * kk, dx + 2 * kk, id, acc);
+                    if (nacc == 2) umma_bf16(tbase + 256, da1 + 2 * kk, dx + 2 * kk, id, acc);
                 }
                 umma_commit(&empty[s]);
             }
@@ -568,81 +782,79 @@ __global__ void __launch_bounds__(kGThreads, 1)
         }
         __syncwarp();
     } else {
-        // ------------------------------------------------------------ epilogue (warps 2..5)
-        // Thread = W row (TMEM lane); each 32-column TMEM load holds 32 rows of
-        // X for it.  The values go to shared memory as one output row per X
-        // row (the stage ring is free once the last MMA has completed), then
-        // one lane per warp copies whole rows out with bulk stores: a few
-        // large writes per row instead of one 128-byte store per warp and X
-        // row, which left the kernel's completion waiting long after its
-        // last instruction.
+        // ------------------------------------------------------------ epilogue (warps 2..5), part 1
+        // thread = W row (TMEM lane); each 32-column TMEM load holds 32 rows of X
         const int quad = warp & 3;
         const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
         const int r = quad * 32 + lane;
         const int chunks = (p.M + 31) / 32;
-        const bool ok = __all_sync(0xffffffffu, g_wait(acc_full, 0, deadline));
-        if (ok) {
-            tc_fence_after();
-            if (p.act) {
-                __nv_bfloat16* stage = reinterpret_cast<__nv_bfloat16*>(sm);  // [M][128]
+        ok = __all_sync(0xffffffffu, g_wait(acc_full, 0, deadline));
+        if (!ok) fail(8);
+        if (ok) tc_fence_after();
+        if (ok && p.op == kThinSilu && p.splits == 1) {
+            // the whole K range is here: SiLU(gate) * up straight from TMEM,
+            // staged as bf16 rows, then written out with 16-byte stores, 16
+            // threads per row
+            __nv_bfloat16* stage = reinterpret_cast<__nv_bfloat16*>(sm);  // [M][128]
+#pragma unroll 1
+            for (int c = 0; c < chunks; ++c) {
+                float g[32], u[32];
+                tmem_ld32(tbase + lane_off + 32 * c, g);
+                tmem_ld32(tbase + lane_off + 256 + 32 * c, u);
+                tmem_ld_wait();
+                // the 32 values first (independent chains the compiler can
+                // interleave), then the predicated stores
+#pragma unroll
+                for (int j = 0; j < 32; ++j) g[j] = silu_times(bf16_round(g[j]), bf16_round(u[j]));
+                uint16_t* srow = reinterpret_cast<uint16_t*>(stage) + (32 * c) * 128 + r;
+                if (32 * c + 32 <= p.M) {
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) srow[j * 128] = static_cast<uint16_t>(bf16_rne_bits(g[j]));
+                } else {
+#pragma unroll
+                    for (int j = 0; j < 32; ++j)
+                        if (32 * c + j < p.M) srow[j * 128] = static_cast<uint16_t>(bf16_rne_bits(g[j]));
+                }
+            }
+            epi_bar();
+            const int e = threadIdx.x - 64, c16 = e & 15;
+            if (8 * c16 < nv0)
+                for (int t = e >> 4; t < p.M; t += 8)
+                    *reinterpret_cast<uint4*>(p.out + static_cast<size_t>(t) * p.paired_I + wb0 + 8 * c16) =
+                        *reinterpret_cast<const uint4*>(stage + t * 128 + 8 * c16);
+        } else if (ok) {
+            float* stage = reinterpret_cast<float*>(sm);  // [nacc][M][128]
+            for (int a = 0; a < nacc; ++a)
 #pragma unroll 1
                 for (int c = 0; c < chunks; ++c) {
-                    float g[32], u[32];
-                    tmem_ld32(tbase + lane_off + 32 * c, g);
-                    tmem_ld32(tbase + lane_off + 256 + 32 * c, u);
+                    float v[32];
+                    tmem_ld32(tbase + lane_off + 256 * a + 32 * c, v);
                     tmem_ld_wait();
 #pragma unroll
                     for (int j = 0; j < 32; ++j) {
                         const int t = 32 * c + j;
-                        if (t < p.M) {
-                            // gate and up are rounded to bf16 first, as when
-                            // they are stored between kernels
-                            const float gb = __bfloat162float(__float2bfloat16_rn(g[j]));
-                            const float ub = __bfloat162float(__float2bfloat16_rn(u[j]));
-                            stage[t * 128 + r] = __float2bfloat16_rn(silu_times(gb, ub));
-                        }
+                        if (t < p.M) stage[(a * p.M + t) * 128 + r] = v[j];
                     }
                 }
-                fence_proxy_async_smem();
-                epi_bar();
-                if (lane == 0) {
-                    const uint32_t bytes = static_cast<uint32_t>(nv0) * 2;
-                    for (int t = quad; t < p.M; t += 4)
-                        bulk_store(p.act + static_cast<size_t>(t) * p.paired_I + 128 * tile, stage + t * 128, bytes);
-                    bulk_commit();
-                    bulk_wait();
-                }
-            } else {
-                float* stage = reinterpret_cast<float*>(sm);  // [M][128]
-                for (int b = 0; b < (two ? 2 : 1); ++b) {
-#pragma unroll 1
-                    for (int c = 0; c < chunks; ++c) {
-                        float v[32];
-                        tmem_ld32(tbase + lane_off + 256 * b + 32 * c, v);
-                        tmem_ld_wait();
-#pragma unroll
-                        for (int j = 0; j < 32; ++j) {
-                            const int t = 32 * c + j;
-                            if (t < p.M) stage[t * 128 + r] = v[j];
-                        }
-                    }
-                    fence_proxy_async_smem();
-                    epi_bar();
-                    if (lane == 0) {
-                        const uint32_t bytes = static_cast<uint32_t>(b ? nv1 : nv0) * 4;
-                        float* dst = p.partials + static_cast<size_t>(split) * p.M * p.Nw + (b ? wb1 : wb0);
-                        for (int t = quad; t < p.M; t += 4)
-                            bulk_store(dst + static_cast<size_t>(t) * p.Nw, stage + t * 128, bytes);
-                        bulk_commit();
-                        bulk_wait();  // the stage is rewritten for the next block
-                    }
-                    epi_bar();
-                }
-            }
-        } else {
-            fail(8);
         }
     }
+    // every CTA of the cluster has staged its accumulators
+    cluster_sync();
+    if (warp >= 2 && !(p.op == kThinSilu && p.splits == 1)) {
+        // ------------------------------------------------------------ epilogue, part 2
+        // this CTA's share of the rows, summed over the cluster in rank order
+        const int e = threadIdx.x - 64;  // 0..127
+        const int t0 = split * p.M / p.splits, t1 = (split + 1) * p.M / p.splits;
+        const uint32_t base = smem_addr(sm), blk = static_cast<uint32_t>(p.M) * 128u * 4u;
+        switch (p.splits) {
+            case 1: epi_part2<1>(p, base, blk, nacc, wb0, wb1, nv0, nv1, t0, t1, e); break;
+            case 2: epi_part2<2>(p, base, blk, nacc, wb0, wb1, nv0, nv1, t0, t1, e); break;
+            case 4: epi_part2<4>(p, base, blk, nacc, wb0, wb1, nv0, nv1, t0, t1, e); break;
+            default: epi_part2<8>(p, base, blk, nacc, wb0, wb1, nv0, nv1, t0, t1, e); break;
+        }
+    }
+    // no CTA leaves while the others may still read its shared memory
+    cluster_sync();
     tc_fence_before();
     __syncthreads();
     if (warp == 1) tmem_dealloc(tbase, 512);
@@ -693,54 +905,132 @@ cudaError_t launch_gemm(const CUtensorMap& tm_x, const CUtensorMap& tm_w, const 
                                        dim3(kGThreads), args, kGAlloc, st);
 }
 
+namespace {
+
+// clusters of each size (1..kThinMaxSplits CTAs) that one device holds at
+// once with the thin kernel's shared memory, measured at set-up per device
+constexpr int kThinMaxDevices = 64;
+int g_thin_clusters[kThinMaxDevices][kThinMaxSplits + 1] = {};
+
+int thin_max_clusters(int size, int sms)
+{
+    int dev = 0;
+    if (cudaGetDevice(&dev) == cudaSuccess && dev >= 0 && dev < kThinMaxDevices && g_thin_clusters[dev][size] > 0)
+        return g_thin_clusters[dev][size];
+    return sms / size / 2;  // not measured: assume half the SMs usable
+}
+
+}  // namespace
+
 ThinPlan thin_plan(int M, int Nw, int K, int sms, int paired_I)
 {
-    ThinPlan g{};
-    g.Mp = (M + 15) / 16 * 16;
-    g.tiles = paired_I > 0 ? (paired_I + 127) / 128 : (Nw + 255) / 256;
-    g.k_steps = (K + kGemmBK - 1) / kGemmBK;
-    // split K while the tiles alone leave SMs idle, into as many ranges as
-    // keep every unit in one wave
-    int splits = g.tiles >= sms ? 1 : sms / g.tiles;
-    splits = splits < 1 ? 1 : (splits > g.k_steps ? g.k_steps : splits);
-    g.kps = (g.k_steps + splits - 1) / splits;
-    g.splits = (g.k_steps + g.kps - 1) / g.kps;
-    g.units = g.tiles * g.splits;
-    const int sb = thin_stage_bytes(g.Mp);
-    g.stages = (kTSmemMax - 1024 - kTBarBytes) / sb;
-    g.stages = g.stages > kTMaxStages ? kTMaxStages : g.stages;
-    g.smem = static_cast<size_t>(g.stages) * sb + kTBarBytes + 1024;
-    g.partial_bytes = (paired_I > 0 && g.splits == 1) ? 0 : static_cast<size_t>(g.splits) * M * Nw * 4;
-    return g;
+    // The unit shape (one or two W blocks) and the split count (the cluster
+    // size) are chosen by a streaming model fitted to measured launches: the
+    // time is a fixed cost per launch plus the bytes the CTAs load -- every
+    // weight byte once, the X tile once per CTA and K step -- at
+    // min(CTAs x 65 GB/s, 7.3 TB/s), with a wave per max-active-cluster
+    // count of clusters.
+    const bool paired = paired_I > 0;
+    const int Mp = (M + 15) / 16 * 16;
+    const int k_steps = (K + kGemmBK - 1) / kGemmBK;
+    const double w_bytes = 2.0 * K * (paired ? 2.0 * paired_I : static_cast<double>(Nw));
+    ThinPlan best{};
+    double best_us = 1e30;
+    for (int wb = paired ? 2 : 1; wb <= 2; ++wb) {
+        const int tiles = paired ? (paired_I + 127) / 128 : (Nw + 128 * wb - 1) / (128 * wb);
+        const int sb = thin_stage_bytes(Mp, wb);
+        const int stages = std::min(kTMaxStages, kTRegionMax / sb);
+        if (stages < 2) continue;
+        for (int s = 1; s <= kThinMaxSplits; s *= 2) {
+            const int kps = (k_steps + s - 1) / s;
+            if ((s - 1) * kps >= k_steps) continue;  // every split gets K steps
+            const bool staged = !(paired && s == 1);
+            if (staged && thin_staging_bytes(M, wb) > static_cast<size_t>(kTRegionMax)) continue;
+            const int ctas = tiles * s;
+            const int per_wave = std::max(1, thin_max_clusters(s, sms));
+            const int waves = (tiles + per_wave - 1) / per_wave;
+            const int active = std::min(tiles, per_wave) * s;
+            const double bytes = w_bytes + static_cast<double>(ctas) * Mp * kps * kGemmBK * 2;
+            const double rate = std::min(active * 65e3, 7.3e6);  // bytes per us
+            const double us = 4.0 * waves + (s > 1 ? 1.0 : 0.0) + bytes / rate;
+            if (us < best_us - 0.05) {
+                best_us = us;
+                best.tiles = tiles;
+                best.k_steps = k_steps;
+                best.kps = kps;
+                best.splits = s;
+                best.Mp = Mp;
+                best.stages = stages;
+                best.wblocks = wb;
+                const size_t ring = static_cast<size_t>(stages) * sb;
+                best.region = std::max(ring, staged ? thin_staging_bytes(M, wb) : 0);
+                best.region = (best.region + 1023) / 1024 * 1024;
+                best.smem = best.region + kTBarBytes + 1024;
+            }
+        }
+    }
+    return best;
 }
 
 cudaError_t thin_prepare()
 {
-    return cudaFuncSetAttribute(gemm_thin_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, kTSmemMax);
+    cudaError_t e = cudaFuncSetAttribute(gemm_thin_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, kTSmemMax);
+    if (e != cudaSuccess) return e;
+    int dev = 0;
+    if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+    if (dev < 0 || dev >= kThinMaxDevices) return cudaSuccess;  // plans fall back to a guess
+    for (int s = 1; s <= kThinMaxSplits; ++s) {
+        cudaLaunchConfig_t cfg{};
+        cfg.gridDim = dim3(s);
+        cfg.blockDim = dim3(kGThreads);
+        cfg.dynamicSmemBytes = kTSmemMax;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = s;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        int n = 0;
+        if ((e = cudaOccupancyMaxActiveClusters(&n, gemm_thin_tc, &cfg)) != cudaSuccess) return e;
+        g_thin_clusters[dev][s] = n;
+    }
+    return cudaSuccess;
 }
 
 cudaError_t launch_thin_gemm(const CUtensorMap& tm_x, const CUtensorMap& tm_w, const ThinParams& p,
                              size_t smem, cudaStream_t st)
 {
-    const int units = (p.paired_I > 0 ? (p.paired_I + 127) / 128 : (p.Nw + 255) / 256) * p.splits;
-    if (units <= 0) return cudaSuccess;
+    const bool paired = p.paired_I > 0;
+    if (p.wblocks != 1 && p.wblocks != 2) return cudaErrorInvalidValue;
+    const int tiles = paired ? (p.paired_I + 127) / 128 : (p.Nw + 128 * p.wblocks - 1) / (128 * p.wblocks);
+    if (tiles <= 0) return cudaSuccess;
+    const size_t ring = static_cast<size_t>(p.stages) * thin_stage_bytes(p.Mp, p.wblocks);
+    const bool staged = !(p.op == kThinSilu && p.splits == 1);
     if (p.M < 1 || p.M > kThinMaxRows || p.Mp != (p.M + 15) / 16 * 16 || p.stages < 2 ||
-        p.stages > kTMaxStages || (p.act && (p.paired_I <= 0 || p.splits != 1)) || (!p.act && !p.partials) ||
-        (p.paired_I > 0 ? (p.paired_I & 7) : (p.Nw & 3)) != 0 ||
-        static_cast<size_t>(p.M) * 128 * 4 > static_cast<size_t>(p.stages) * thin_stage_bytes(p.Mp) ||
-        smem > static_cast<size_t>(kTSmemMax) ||
-        static_cast<size_t>(p.stages) * thin_stage_bytes(p.Mp) + kTBarBytes + 1024 > smem)
+        p.stages > kTMaxStages || (p.splits != 1 && p.splits != 2 && p.splits != 4 && p.splits != 8) ||
+        (p.splits - 1) * p.kps >= p.k_steps || p.splits * p.kps < p.k_steps ||
+        (!p.out && p.op != kThinQkvRope) || (p.op == kThinSilu) != paired || (paired && p.wblocks != 2) ||
+        (paired && (p.paired_I & 7) != 0) || (!paired && (p.Nw & 3) != 0) ||
+        (p.op == kThinQkvRope && (!p.q || !p.k || !p.v || !p.rope || (p.d != 64 && p.d != 128) ||
+                                  p.Nw != (p.Hq + 2 * p.Hkv) * p.d)) ||
+        ring > p.region || (staged && thin_staging_bytes(p.M, p.wblocks) > p.region) || p.region % 1024 != 0 ||
+        p.region + kTBarBytes + 1024 > smem || smem > static_cast<size_t>(kTSmemMax))
         return cudaErrorInvalidValue;
     cudaLaunchConfig_t cfg{};
-    cfg.gridDim = dim3(units);
+    cfg.gridDim = dim3(tiles * p.splits);
     cfg.blockDim = dim3(kGThreads);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = st;
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
+    attr[1].id = cudaLaunchAttributeClusterDimension;
+    attr[1].val.clusterDim.x = p.splits;
+    attr[1].val.clusterDim.y = 1;
+    attr[1].val.clusterDim.z = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = 2;
     return cudaLaunchKernelEx(&cfg, gemm_thin_tc, tm_x, tm_w, p);
 }
 

@@ -782,7 +782,7 @@ namespace {
 
 // Workspace carve-up of one block call (all offsets 256-byte aligned).
 struct BlockBufs {
-    size_t h, qkv, q, k, v, attn, gu, act, gemm_part, gemm_cnt, total;
+    size_t h, qkv, q, k, v, attn, gu, act, rope, gemm_part, gemm_cnt, total;
 };
 
 // split-K tile counters: one region per projection GEMM of a block call (a
@@ -825,18 +825,17 @@ BlockBufs block_bufs(const statekv_config& c, const statekv_block_config& b, int
     o.attn = take(rows * hq * d * 2);
     o.gu = take(rows * 2 * static_cast<size_t>(b.intermediate) * 2);
     o.act = take(rows * static_cast<size_t>(b.intermediate) * 2);
+    o.rope = take(rows * (d / 2) * 8);  // (cos, sin) per row and rotated pair
     // split-K partials of the largest split GEMM, and the tile counters of
-    // the cooperative path (rows above kThinMaxRows)
+    // the cooperative path (rows above kThinMaxRows; the thin path adds its
+    // splits up inside a thread-block cluster and needs neither)
     int nk[4][2];
     block_gemm_shapes(c, b, nk);
     size_t part = 0;
     const int sms = device_sm_count();
-    for (int i = 0; i < 4; ++i) {
-        const int M = static_cast<int>(rows), N = nk[i][0], K = nk[i][1];
-        part = std::max(part, M <= kThinMaxRows
-                                  ? thin_plan(M, N, K, sms, i == 2 ? b.intermediate : 0).partial_bytes
-                                  : gemm_plan(M, N, K, sms).partial_bytes);
-    }
+    if (rows > static_cast<size_t>(kThinMaxRows))
+        for (int i = 0; i < 4; ++i)
+            part = std::max(part, gemm_plan(static_cast<int>(rows), nk[i][0], nk[i][1], sms).partial_bytes);
     o.gemm_part = take(part);
     o.gemm_cnt = take(static_cast<size_t>(4) * c.num_layers * kGemmCounterRegion * 4);
     o.total = off;
@@ -980,15 +979,14 @@ statekv_status statekv_block_frame(statekv_handle* h, const statekv_block_config
         return timed(h, 3, st, [&] { return launch_gemm(tx, tw, gp, sms, st); }) == cudaSuccess;
     };
     // Up to kThinMaxRows rows (one stream's frame) the projections run as thin
-    // GEMMs: each writes split-K partials (or, for gate/up unsplit, SiLU * up
-    // directly) and the next elementwise kernel adds them up -- the QKV sum
-    // in the RoPE kernel, the output and down projections' sums in the
-    // residual update, which also computes the following RMSNorm (the next
-    // layer's, when the call covers it).
-    float* part = reinterpret_cast<float*>(ws + bb.gemm_part);
+    // GEMMs whose epilogues finish the job: QKV adds the bias, rotates q and k
+    // with the table the preceding RMSNorm wrote and stores q, k, v in the
+    // step's layout; the output and down projections add into the residual
+    // x; gate/up stores SiLU(gate) * up.
     const unsigned long long wd_ns = 1000000ull * (c.watchdog_ms ? c.watchdog_ms : 2000u);
-    auto thin_gemm = [&](const void* X, const void* Wt, int Nw, int K, int paired_I,
-                         __nv_bfloat16* act, int* splits_out) {
+    float2* rope_tab = reinterpret_cast<float2*>(ws + bb.rope);
+    auto thin_gemm = [&](const void* X, const void* Wt, int Nw, int K, int paired_I, int op,
+                         __nv_bfloat16* out, const void* bias) {
         const ThinPlan g = thin_plan(rows, Nw, K, sms, paired_I);
         CUtensorMap tx, tw;
         const cuuint64_t dx[4] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(rows), 1, 1};
@@ -1010,62 +1008,55 @@ statekv_status statekv_block_frame(statekv_handle* h, const statekv_block_config
         tp.splits = g.splits;
         tp.stages = g.stages;
         tp.paired_I = paired_I;
-        tp.act = (act && g.splits == 1) ? act : nullptr;
-        tp.partials = tp.act ? nullptr : part;
+        tp.wblocks = g.wblocks;
+        tp.region = g.region;
+        tp.op = op;
+        tp.out = out;
+        tp.bias = static_cast<const __nv_bfloat16*>(bias);
+        tp.q = buf(bb.q);
+        tp.k = buf(bb.k);
+        tp.v = buf(bb.v);
+        tp.rope = rope_tab;
+        tp.Hq = Hq;
+        tp.Hkv = Hkv;
+        tp.d = d;
         tp.status = h->status_dev;
         tp.watchdog_ns = wd_ns;
-        *splits_out = tp.act ? 0 : g.splits;
         return timed(h, 3, st, [&] { return launch_thin_gemm(tx, tw, tp, g.smem, st); }) == cudaSuccess;
     };
     const bool thin = rows <= kThinMaxRows;
     for (int l = layer_begin; l < layer_begin + layer_count; ++l) {
         const statekv_block_weights& w = weights[l];
-        const bool last = l + 1 == layer_begin + layer_count;
-        int splits = 0;
-        // the thin path's previous layer already normalised x into h
-        if ((!thin || l == layer_begin) &&
-            timed(h, 4, st, [&] {
-                return launch_rmsnorm(x, static_cast<const __nv_bfloat16*>(w.norm_attn), b.rms_eps,
-                                      buf(bb.h), rows, H, st);
-            }) != cudaSuccess)
-            return STATEKV_ERR_CUDA;
+        rp.layer = l;
         if (thin) {
-            if (!thin_gemm(buf(bb.h), w.w_qkv, W, H, 0, nullptr, &splits)) return STATEKV_ERR_CUDA;
-            rp.part = part;
-            rp.splits = splits;
-            rp.bias = static_cast<const __nv_bfloat16*>(w.b_qkv);
-        } else if (!gemm(buf(bb.h), w.w_qkv, w.b_qkv, buf(bb.qkv), false, W, H)) {
+            // the norm also writes the rows' RoPE table for the QKV epilogue
+            if (timed(h, 4, st, [&] {
+                    return launch_rmsnorm_rope(x, static_cast<const __nv_bfloat16*>(w.norm_attn), b.rms_eps,
+                                               buf(bb.h), rows, H, rp, rope_tab, st);
+                }) != cudaSuccess ||
+                !thin_gemm(buf(bb.h), w.w_qkv, W, H, 0, kThinQkvRope, nullptr, w.b_qkv))
+                return STATEKV_ERR_CUDA;
+        } else if (timed(h, 4, st, [&] {
+                       return launch_rmsnorm(x, static_cast<const __nv_bfloat16*>(w.norm_attn), b.rms_eps,
+                                             buf(bb.h), rows, H, st);
+                   }) != cudaSuccess ||
+                   !gemm(buf(bb.h), w.w_qkv, w.b_qkv, buf(bb.qkv), false, W, H) ||
+                   timed(h, 4, st, [&] { return launch_qkv_rope(rp, st); }) != cudaSuccess) {
             return STATEKV_ERR_CUDA;
         }
-        rp.layer = l;
-        if (timed(h, 4, st, [&] { return launch_qkv_rope(rp, st); }) != cudaSuccess)
-            return STATEKV_ERR_CUDA;
         statekv_frame_args a = probe;
         a.layer_begin = l;
         a.layer_count = 1;
         const statekv_status r = run_step(h, a, st);
         if (r != STATEKV_OK) return r;
         if (thin) {
-            if (!thin_gemm(buf(bb.attn), w.w_o, H, Hq * d, 0, nullptr, &splits) ||
+            if (!thin_gemm(buf(bb.attn), w.w_o, H, Hq * d, 0, kThinResidual, x, nullptr) ||
                 timed(h, 4, st, [&] {
-                    return launch_residual_norm(part, splits, x,
-                                                static_cast<const __nv_bfloat16*>(w.norm_mlp),
-                                                b.rms_eps, buf(bb.h), rows, H, st);
-                }) != cudaSuccess)
-                return STATEKV_ERR_CUDA;
-            if (!thin_gemm(buf(bb.h), w.w_gate_up, 2 * I, H, I, buf(bb.act), &splits))
-                return STATEKV_ERR_CUDA;
-            if (splits > 0 &&
-                timed(h, 4, st, [&] { return launch_silu_partials(part, splits, buf(bb.act), rows, I, st); }) !=
-                    cudaSuccess)
-                return STATEKV_ERR_CUDA;
-            const __nv_bfloat16* next_norm =
-                last ? nullptr : static_cast<const __nv_bfloat16*>(weights[l + 1].norm_attn);
-            if (!thin_gemm(buf(bb.act), w.w_down, H, I, 0, nullptr, &splits) ||
-                timed(h, 4, st, [&] {
-                    return launch_residual_norm(part, splits, x, next_norm, b.rms_eps, buf(bb.h), rows,
-                                                H, st);
-                }) != cudaSuccess)
+                    return launch_rmsnorm(x, static_cast<const __nv_bfloat16*>(w.norm_mlp), b.rms_eps,
+                                          buf(bb.h), rows, H, st);
+                }) != cudaSuccess ||
+                !thin_gemm(buf(bb.h), w.w_gate_up, 2 * I, H, I, kThinSilu, buf(bb.act), nullptr) ||
+                !thin_gemm(buf(bb.act), w.w_down, H, I, 0, kThinResidual, x, nullptr))
                 return STATEKV_ERR_CUDA;
             continue;
         }

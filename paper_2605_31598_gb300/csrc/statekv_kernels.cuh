@@ -154,12 +154,6 @@ cudaError_t launch_state_metrics(const uint8_t* mask_n, const uint8_t* mask_n1, 
 // Per-frame transformer block (block_kernel.cu).
 struct RopeParams {
     const __nv_bfloat16* qkv;   // [S*T][(Hq + 2 Hkv) * d]: q heads, k heads, v heads
-    // or, when part is set, the QKV projection as `splits` fp32 split-K
-    // partials [splits][S*T][(Hq + 2 Hkv) * d] plus the nullable bias, summed
-    // in split order and rounded to bf16 (the same rounding point as qkv)
-    const float* part;
-    int splits;
-    const __nv_bfloat16* bias;
     __nv_bfloat16* q;           // [S][T][Hq][d]
     __nv_bfloat16* k;           // [S][T][Hkv][d]
     __nv_bfloat16* v;           // [S][T][Hkv][d]
@@ -174,16 +168,6 @@ cudaError_t launch_rmsnorm(const __nv_bfloat16* x, const __nv_bfloat16* g, float
 cudaError_t launch_qkv_rope(const RopeParams& p, cudaStream_t st);
 cudaError_t launch_silu_mul(const __nv_bfloat16* gu, __nv_bfloat16* a, long long rows, int I,
                             cudaStream_t st);
-// x[r] = bf16(x[r] + sum of `splits` fp32 partials [splits][rows][H] in split
-// order); then, when g is set, y[r] = RMSNorm(x[r]) g with the same arithmetic
-// (and order) as launch_rmsnorm.
-cudaError_t launch_residual_norm(const float* part, int splits, __nv_bfloat16* x,
-                                 const __nv_bfloat16* g, float eps, __nv_bfloat16* y, int rows,
-                                 int H, cudaStream_t st);
-// a = bf16(SiLU(bf16(gate)) bf16(up)) from `splits` fp32 partials
-// [splits][rows][2I] (gate in columns [0, I), up in [I, 2I)).
-cudaError_t launch_silu_partials(const float* part, int splits, __nv_bfloat16* a, int rows, int I,
-                                 cudaStream_t st);
 // Projection GEMMs of the block (gemm_kernel.cu): D[M][N] = X[M][K] W[N][K]^T
 // (+ bias[N]) (+ D when add), bf16, fp32 accumulation on tcgen05.  A unit is
 // a 128-column tile of W for a pair of 128-row tiles of X over kps 64-wide K
@@ -211,31 +195,52 @@ struct GemmParams {
 cudaError_t gemm_prepare();
 cudaError_t launch_gemm(const CUtensorMap& tm_x, const CUtensorMap& tm_w, const GemmParams& p,
                         int sms, cudaStream_t st);
-// Thin projections (M <= kThinMaxRows, gemm_kernel.cu): W is the MMA's A
-// operand (two 128-row blocks per unit) and all of X (Mp = M rounded up to 16
-// rows, one TMA box of 64 K-columns x Mp rows) its B operand.  A unit is one
-// pair of W row blocks over one range of K; each CTA takes one unit.  Output:
-// fp32 partials [splits][M][Nw] (feature = W row), or with `act` set (paired
-// gate/up, one split) act[M][I] = bf16(SiLU(bf16(gate)) bf16(up)).  Paired
-// (paired_I > 0): block 0 = gate rows [128 t, 128 t + 128), block 1 = the up
-// rows I + 128 t onward; otherwise rows [256 t, 256 t + 256).  No CTA waits
-// on another.
+// Thin projections (M <= kThinMaxRows rows, gemm_kernel.cu): W is the MMA's
+// A operand and all of X (Mp = M rounded up to 16 rows, one TMA box of 64
+// K-columns x Mp rows) its B operand.  A unit is `wblocks` 128-row blocks of
+// W (rows [256 t, 256 t + 256) for two; for the gate/up projection a gate
+// block and the matching up block) over one range of K; the `splits` units of
+// a tile form a thread-block cluster, which adds its accumulators in
+// distributed shared memory in rank order, each CTA finishing a 1/splits
+// share of the rows of X:
+//   kThinResidual  out[m][n] = bf16(out[m][n] + sum)        (out: [M][Nw])
+//   kThinQkvRope   bias added, rounded to bf16, q and k heads rotated with the
+//                  cos/sin table `rope` ([M][d/2] float2, scale applied), v
+//                  copied, written in the [M][H][d] layouts of q, k, v
+//   kThinSilu      out[m][j] = bf16(SiLU(bf16(gate)) bf16(up)) (out: [M][I];
+//                  paired_I = I: gate rows [0, I), up rows [I, 2I) of W)
+// The X tensor map's box is 64 x Mp, the W map's 64 x 128 (128-byte swizzle).
 constexpr int kThinMaxRows = 256;
+constexpr int kThinMaxSplits = 8;
+enum ThinOp : int { kThinResidual = 0, kThinQkvRope = 1, kThinSilu = 2 };
 struct ThinPlan {
-    int tiles, k_steps, kps, splits, units, Mp, stages;
-    size_t smem, partial_bytes;
+    int tiles, k_steps, kps, splits, Mp, stages, wblocks;
+    size_t region, smem;  // ring / staging bytes; dynamic shared memory of the launch
 };
 ThinPlan thin_plan(int M, int Nw, int K, int sms, int paired_I);
 struct ThinParams {
-    int M, Mp, Nw, K, k_steps, kps, splits, stages, paired_I;
-    float* partials;            // [splits][M][Nw], when act is null
-    __nv_bfloat16* act;         // [M][paired_I]: paired, splits == 1
+    int M, Mp, Nw, K, k_steps, kps, splits, stages, paired_I, op, wblocks;
+    size_t region;
+    __nv_bfloat16* out;             // residual / silu output
+    const __nv_bfloat16* bias;      // qkv: nullable [Nw]
+    __nv_bfloat16 *q, *k, *v;       // qkv: [M][Hq][d], [M][Hkv][d], [M][Hkv][d]
+    const float2* rope;             // qkv: [M][d / 2] (cos, sin)
+    int Hq, Hkv, d;
     int32_t* status;
     unsigned long long watchdog_ns;
 };
+// Sets the kernel's shared-memory limit and measures, on the current device,
+// how many clusters of each size fit at once (the plans use it).
 cudaError_t thin_prepare();
 cudaError_t launch_thin_gemm(const CUtensorMap& tm_x, const CUtensorMap& tm_w, const ThinParams& p,
                              size_t smem, cudaStream_t st);
+// RMSNorm as launch_rmsnorm, and, when rp is set, the RoPE table of the next
+// QKV projection: rope[r][k] = (cos, sin)(p * freq[k]) * scale for row r's
+// virtual position p (the same fp64 angle and fp32 sin/cos as the rotation
+// kernel).
+cudaError_t launch_rmsnorm_rope(const __nv_bfloat16* x, const __nv_bfloat16* g, float eps,
+                                __nv_bfloat16* y, int rows, int H, const RopeParams& rp, float2* rope,
+                                cudaStream_t st);
 
 
 // One-pass split-K decoding over the cache (decode_kernel.cu): for up to
