@@ -336,9 +336,19 @@ typedef struct {
 
 /* Borrowed device pointers into the arena, valid until statekv_destroy.  The
  * contents are current once the stream of the last prefill call is
- * synchronised; the counters are host-side and current immediately. */
+ * synchronised; the counters are host-side and current immediately.
+ *
+ * statekv_state_view: the compressed state of one (stream, layer) -- Sec. 3.3,
+ * Eq. 6's S_n, the B tokens per KV head kept by the top-B selection, with
+ * their virtual positions (Sec. 3.3: token t of frame n sits at (n-1) T + t)
+ * and the virtual length L_n.  Errors: INVALID_ARG for a null handle or
+ * output, or a (stream, layer) outside the configuration. */
 statekv_status statekv_state_view(const statekv_handle* h, int32_t stream, int32_t layer,
                                   statekv_state_info* out);
+/* statekv_cache_view: the detailed state of one (stream, layer) -- Sec. 3.2,
+ * Eq. 4's D_n, every frame's K/V rows appended in order (then any decoded
+ * tokens), which decoding attends to.  Errors: INVALID_ARG for a null handle
+ * or output, or a (stream, layer) outside the configuration. */
 statekv_status statekv_cache_view(const statekv_handle* h, int32_t stream, int32_t layer,
                                   statekv_cache_info* out);
 
