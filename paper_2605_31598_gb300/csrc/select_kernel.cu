@@ -248,8 +248,10 @@ __global__ void __launch_bounds__(kSelThreads)
             }
             const unsigned long long diff = a ^ o;  // bits in which some keys differ
             const int hb = diff ? 63 - __clzll(static_cast<long long>(diff)) : 0;
-            const int shift0 = (hb / 8) * 8;
-            const unsigned long long above = shift0 >= 56 ? 0ull : ~((1ull << (shift0 + 8)) - 1);
+            // the first digit is the 8 bits ending at that bit, so every bit it
+            // holds can differ (a digit below bit 0 is cut to its bits >= 0)
+            const int shift0 = hb - 7;
+            const unsigned long long above = hb >= 63 ? 0ull : ~((2ull << hb) - 1);
             sh_shift = shift0;
             sh_prefix = o & above;  // = a & above
             sh_mask = above;
@@ -260,12 +262,14 @@ __global__ void __launch_bounds__(kSelThreads)
         __syncthreads();
         prefix = sh_prefix;
         mask = sh_mask;
-        for (int shift = sh_shift, pass = 0; shift >= 0; shift -= 8, ++pass) {
+        for (int shift = sh_shift, pass = 0; shift > -8; shift -= 8, ++pass) {
             unsigned* hist = hist2[pass & 1];
+            const int dsh = shift < 0 ? 0 : shift;                                 // the digit's lowest bit
+            const unsigned long long dmask = shift < 0 ? (0xFFull >> -shift) : 0xFFull;  // its bits, at dsh
             for (int i0 = 0; i0 < n; i0 += kSelThreads) {
                 const int i = i0 + tid;
                 int digit = -1;
-                if (i < n && (key[i] & mask) == prefix) digit = (key[i] >> shift) & 0xFF;
+                if (i < n && (key[i] & mask) == prefix) digit = static_cast<int>((key[i] >> dsh) & dmask);
                 const unsigned peers = __match_any_sync(0xffffffffu, digit);
                 if (digit >= 0 && lane == __ffs(peers) - 1) atomicAdd(&hist[digit], __popc(peers));
             }
@@ -296,8 +300,8 @@ __global__ void __launch_bounds__(kSelThreads)
                         if (above + c[j] >= static_cast<unsigned>(k)) {
                             const unsigned d = 255 - 8 * lane - j;
                             const int k_rem = k - static_cast<int>(above);
-                            sh_prefix = prefix | (static_cast<unsigned long long>(d) << shift);
-                            sh_mask = mask | (0xFFull << shift);
+                            sh_prefix = prefix | (static_cast<unsigned long long>(d) << dsh);
+                            sh_mask = mask | (dmask << dsh);
                             sh_k = k_rem;
                             sh_done = (c[j] == static_cast<unsigned>(k_rem)) ? 1 : 0;
                             break;
