@@ -217,9 +217,12 @@ statekv_status statekv_state_metrics(const uint8_t* mask_n, const uint8_t* mask_
  *        the layer's state and decode cache advance by one frame)
  *   x1 = x + o W_o^T
  *   x2 = x1 + (SiLU(h2 W_gate^T) * (h2 W_up^T)) W_down^T,  h2 = RMSNorm(x1) * norm_mlp
- * bf16 storage between steps, fp32 arithmetic; the projections are plain
- * cuBLASLt GEMMs.  Weight matrices are row-major [out features][in features]
- * (torch.nn.Linear layout). */
+ * bf16 storage between steps, fp32 arithmetic.  The projections run on the
+ * library's own tensor-core GEMMs: for up to 256 rows (one stream's frame) a
+ * split-K kernel whose clusters add their partial sums in distributed shared
+ * memory, with bias + RoPE, the residual add and SiLU * up in its epilogues;
+ * above that a cooperative split-K kernel.  Weight matrices are row-major
+ * [out features][in features] (torch.nn.Linear layout). */
 typedef struct {
     int32_t hidden;            /* model width (multiple of 8, at most 8192) */
     int32_t intermediate;      /* MLP width (multiple of 8) */
@@ -257,13 +260,12 @@ statekv_status statekv_block_workspace_bytes(const statekv_handle* h,
  *            layer layer_begin; not modified
  *   x_out    bf16 [stream_count][T][hidden] (device): layer
  *            layer_begin + layer_count - 1's output (may equal x_in)
- * Every covered (stream, layer) advances by one frame.  The first call for a
- * given stream count times cuBLASLt's candidate algorithms for each projection
- * shape on the call's operands and keeps the fastest; that call synchronises
- * the stream (so it cannot be captured into a CUDA graph), later calls do not.
- * Errors as statekv_prefill_frame, INVALID_ARG for a bad block config
- * (head_dim > 128 pairs, sizes not multiples of 8), UNSUPPORTED if cuBLASLt
- * finds no GEMM plan; nothing is enqueued on an argument error. */
+ * Every covered (stream, layer) advances by one frame.  The call only
+ * enqueues work on `stream` (no synchronisation).  Errors as
+ * statekv_prefill_frame, INVALID_ARG for a bad block config (head_dim / 2 >
+ * 64 rotation pairs, sizes not multiples of 8, hidden > 8192) or a workspace
+ * smaller than statekv_block_workspace_bytes(); nothing is enqueued on an
+ * argument error, CUDA if a launch fails. */
 statekv_status statekv_block_frame(statekv_handle* h, const statekv_block_config* bc,
                                    const statekv_block_weights* weights, int32_t stream_begin,
                                    int32_t stream_count, int32_t layer_begin, int32_t layer_count,
