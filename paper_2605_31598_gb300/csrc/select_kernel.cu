@@ -16,6 +16,7 @@
 //      keys are distinct and exactly B members are kept;
 //   3. evicted / empty slots (ascending) receive the admitted frame tokens
 //      (ascending) as 128-bit row copies, and their positions are updated.
+#include "sm103_ptx.cuh"
 #include "statekv_kernels.cuh"
 
 #include <algorithm>
@@ -110,6 +111,11 @@ __global__ void __launch_bounds__(kSelThreads)
     state_select_gather(const SelectParams p)
 {
     extern __shared__ __align__(16) uint8_t smem_raw[];
+    // A kernel launched programmatically behind this one (the transformer
+    // block's output projection) may start now: it requests its first weight
+    // tiles, which nothing here writes, and waits for this grid's completion
+    // before it reads anything else.
+    ptx::pdl_launch_dependents();
     const int T = p.T, B = p.B, P = p.P, D = p.D;
     uint64_t* key = reinterpret_cast<uint64_t*>(smem_raw);            // [P]
     int* free_slot = reinterpret_cast<int*>(key + P);                  // [T]
