@@ -26,6 +26,7 @@ namespace {
 
 constexpr int kSelThreads = 640;
 constexpr int kSelWarps = kSelThreads / 32;
+static_assert(kSelWarps <= 32, "one warp combines the warps' values");
 
 // Exclusive block-wide scan of one int per thread; returns the total.
 __device__ __forceinline__ int block_exclusive_scan(int x, int* warp_sums, int& excl)
@@ -158,8 +159,9 @@ __global__ void __launch_bounds__(kSelThreads)
             int ps[4];
 #pragma unroll
             for (int e = 0; e < 4; ++e) {  // positions first: their loads overlap the sums'
+                // (bounded by B, not by the count, so they do not wait for the count's load)
                 const int c = c0 + e;
-                ps[e] = c < count ? pos[c] : L + (c - B);
+                ps[e] = c < B ? pos[c] : 0;
             }
             const float4 s4 = rows_sum4(part, p.MT, P, c0);
             float4 r4 = s4;
@@ -179,8 +181,9 @@ __global__ void __launch_bounds__(kSelThreads)
                 const int c = c0 + e;
                 const int i = c < count ? c : (c >= B && c - B < T) ? count + (c - B) : -1;
                 if (i < 0) continue;
+                const int pe = c < count ? ps[e] : L + (c - B);
                 const uint64_t kk = (static_cast<uint64_t>(__float_as_uint(rv[e])) << 32) |
-                                    static_cast<uint32_t>(0xFFFFFFFFu - static_cast<uint32_t>(ps[e]));
+                                    static_cast<uint32_t>(0xFFFFFFFFu - static_cast<uint32_t>(pe));
                 key[i] = kk;
                 kand &= kk;
                 kor |= kk;
@@ -246,23 +249,30 @@ __global__ void __launch_bounds__(kSelThreads)
             }
         }
         __syncthreads();
-        if (tid == 0) {
-            unsigned long long a = ~0ull, o = 0ull;
-            for (int w = 0; w < kSelWarps; ++w) {
-                a &= warp_and[w];
-                o |= warp_or[w];
-            }
+        if (tid < 32) {  // warp 0 combines the warps' values
+            const unsigned long long wa = lane < kSelWarps ? warp_and[lane] : ~0ull;
+            const unsigned long long wo = lane < kSelWarps ? warp_or[lane] : 0ull;
+            const unsigned long long a =
+                (static_cast<unsigned long long>(__reduce_and_sync(0xffffffffu, static_cast<uint32_t>(wa >> 32)))
+                 << 32) |
+                __reduce_and_sync(0xffffffffu, static_cast<uint32_t>(wa));
+            const unsigned long long o =
+                (static_cast<unsigned long long>(__reduce_or_sync(0xffffffffu, static_cast<uint32_t>(wo >> 32)))
+                 << 32) |
+                __reduce_or_sync(0xffffffffu, static_cast<uint32_t>(wo));
             const unsigned long long diff = a ^ o;  // bits in which some keys differ
             const int hb = diff ? 63 - __clzll(static_cast<long long>(diff)) : 0;
             // the first digit is the 8 bits ending at that bit, so every bit it
             // holds can differ (a digit below bit 0 is cut to its bits >= 0)
             const int shift0 = hb - 7;
             const unsigned long long above = hb >= 63 ? 0ull : ~((2ull << hb) - 1);
-            sh_shift = shift0;
-            sh_prefix = o & above;  // = a & above
-            sh_mask = above;
-            sh_k = B;
-            sh_done = 0;
+            if (lane == 0) {
+                sh_shift = shift0;
+                sh_prefix = o & above;  // = a & above
+                sh_mask = above;
+                sh_k = B;
+                sh_done = 0;
+            }
         }
         for (int i = tid; i < 512; i += kSelThreads) hist2[i >> 8][i & 255] = 0;
         __syncthreads();
