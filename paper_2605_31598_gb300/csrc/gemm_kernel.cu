@@ -10,11 +10,16 @@
 //     tiles of X (both accumulators live in TMEM, so a W tile is loaded once
 //     for up to 256 rows), over one contiguous range of K;
 //   - when the (column tile, row pair) grid alone would leave SMs idle, K is
-//     split into ranges: every split writes an fp32 partial of its tile, and
-//     the last split to finish (an atomic counter per tile, no waiting) adds
-//     the partials in split order, so the result does not depend on timing;
+//     split into ranges: every split writes an fp32 partial of its tile; the
+//     launch is cooperative, so the splits of a tile wait for one another (an
+//     atomic counter per tile, bounded by the watchdog), then split s adds its
+//     share of the rows over every split in split order, so the result does
+//     not depend on timing;
 //   - one CTA per SM walks the units; TMEM holds two accumulator sets, so the
-//     epilogue of one unit overlaps the main loop of the next.
+//     epilogue of one unit overlaps the main loop of the next;
+//   - GEMMs with enough 256-wide tiles to fill every SM by themselves (the
+//     gate/up projection at two or more streams) use W tiles of 256 rows: one
+//     accumulator set fills TMEM, and each staged byte feeds 1.5x the MMA work.
 // 192 threads: warp 0 issues the TMA loads (a four-stage ring of 48 KB: X rows
 // m0..m0+127, X rows m0+128..m0+255, W rows n0..n0+127, 64 K-columns each,
 // 128-byte swizzle), warp 1 allocates TMEM and issues tcgen05.mma
@@ -33,23 +38,36 @@ namespace {
 using namespace ptx;
 
 constexpr int kGThreads = 192;
-constexpr int kGStages = 4;
 constexpr int kGTileA = kGemmBM * kGemmBK * 2;        // 16 KB: 128 rows of X x 64 K
-constexpr int kGTileB = kGemmBN * kGemmBK * 2;        // 16 KB: 128 rows of W x 64 K
-constexpr int kGStageBytes = 2 * kGTileA + kGTileB;   // 48 KB
 // epilogue staging: per epilogue warp a 32 x 36 fp32 block (row-major, 16-byte
 // rows padded by one float4 against bank conflicts) turns thread-per-row TMEM
 // reads into row-contiguous global stores
 constexpr int kGStageLd = 36;
 constexpr int kRG = 8;  // rows per group of the split-K reduction (2 kRG loads in flight)
-constexpr int kGOffEpi = kGStages * kGStageBytes;
-constexpr int kGOffBar = kGOffEpi + 4 * 32 * kGStageLd * 4;
-constexpr int kGNumBars = 2 * kGStages + 5;           // full[4] empty[4] acc_full[2] acc_empty[2] drain
-constexpr int kGOffMisc = kGOffBar + kGNumBars * 8;
-constexpr int kGBytes = kGOffMisc + 16;
-constexpr int kGAlloc = kGBytes + 1024;               // room to align the base to 1 KB
-static_assert(kGAlloc <= 232448, "shared memory budget");
-static_assert(kGStageBytes % 1024 == 0 && kGTileA % 1024 == 0, "swizzle atoms stay aligned");
+
+// Shared memory and TMEM plan for a tile of 256 rows of X x BN rows of W.
+// BN = 128: a four-stage ring of 48 KB and two accumulator sets (2 x 128
+// TMEM columns each), so a unit's epilogue overlaps the next unit's main loop.
+// BN = 256: a three-stage ring of 64 KB (W tile 32 KB) and one set filling
+// TMEM's 512 columns; each byte staged feeds 1.5x the MMA work of BN = 128,
+// for GEMMs large enough to be bound by the L2-to-SM traffic.
+template <int BN>
+struct GLayout {
+    static constexpr int kStages = BN == 256 ? 3 : 4;
+    static constexpr int kAccSets = BN == 256 ? 1 : 2;
+    static constexpr int kTileB = BN * kGemmBK * 2;
+    static constexpr int kStageBytes = 2 * kGTileA + kTileB;
+    static constexpr int kOffEpi = kStages * kStageBytes;
+    static constexpr int kOffBar = kOffEpi + 4 * 32 * kGStageLd * 4;
+    static constexpr int kNumBars = 2 * kStages + 5;  // full[S] empty[S] acc_full[2] acc_empty[2] drain
+    static constexpr int kOffMisc = kOffBar + kNumBars * 8;
+    static constexpr int kBytes = kOffMisc + 16;
+    static constexpr int kAlloc = kBytes + 1024;      // room to align the base to 1 KB
+    static_assert(BN == 128 || BN == 256, "tile width");
+    static_assert(kAccSets * 2 * BN <= 512, "TMEM columns");
+    static_assert(kAlloc <= 232448, "shared memory budget");
+    static_assert(kStageBytes % 1024 == 0 && kGTileA % 1024 == 0, "swizzle atoms stay aligned");
+};
 
 __device__ __forceinline__ unsigned long long g_globaltimer()
 {
@@ -75,12 +93,13 @@ struct GemmUnit {
     bool two;  // the pair's second 128-row tile holds rows below M
 };
 
+template <int BN>
 __device__ __forceinline__ GemmUnit gemm_unit(const GemmParams& p, int w)
 {
     GemmUnit x;
     x.tile = w / p.splits;
     x.split = w - x.tile * p.splits;
-    x.n0 = (x.tile % p.n_tiles) * kGemmBN;
+    x.n0 = (x.tile % p.n_tiles) * BN;
     x.m0 = (x.tile / p.n_tiles) * 2 * kGemmBM;
     x.ks0 = x.split * p.kps;
     x.ks1 = min(p.k_steps, x.ks0 + p.kps);
@@ -167,22 +186,27 @@ __device__ __forceinline__ void store_rows_strided(const GemmParams& p, int m0, 
     store4_rows<NR>(p, m0, mstep, nrows, n, a);
 }
 
+template <int BN>
 __global__ void __launch_bounds__(kGThreads, 1)
     gemm_bf16_tc(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_w,
                  const GemmParams p)
 {
+    using L = GLayout<BN>;
+    constexpr int kGStages = L::kStages, kGStageBytes = L::kStageBytes, kGTileB = L::kTileB;
+    constexpr int NB = L::kAccSets;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-    uint64_t* bars = reinterpret_cast<uint64_t*>(sm + kGOffBar);
+    uint64_t* bars = reinterpret_cast<uint64_t*>(sm + L::kOffBar);
     uint64_t* full = bars;                     // stage loaded
     uint64_t* empty = bars + kGStages;         // stage read by its MMAs
     uint64_t* acc_full = bars + 2 * kGStages;  // accumulator set complete
     uint64_t* acc_empty = acc_full + 2;        // accumulator set read out
     uint64_t* drain = acc_full + 4;            // every MMA of the CTA has completed
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + kGOffMisc);
-    volatile int* abort_flag = reinterpret_cast<volatile int*>(sm + kGOffMisc + 4);
-    volatile int* last_flag = reinterpret_cast<volatile int*>(sm + kGOffMisc + 8);
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + L::kOffMisc);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(sm + L::kOffMisc + 4);
+    volatile int* last_flag = reinterpret_cast<volatile int*>(sm + L::kOffMisc + 8);
+    const bool split = BN == 128 && p.splits > 1;  // the plan splits K only with 128-wide tiles
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (threadIdx.x == 0) {
@@ -221,7 +245,7 @@ __global__ void __launch_bounds__(kGThreads, 1)
             bool ok = true;
             int n = 0;
             for (int w = blockIdx.x; ok && w < p.units; w += gridDim.x) {
-                const GemmUnit x = gemm_unit(p, w);
+                const GemmUnit x = gemm_unit<BN>(p, w);
                 const unsigned long long deadline = g_globaltimer() + p.watchdog_ns;
                 for (int ks = x.ks0; ks < x.ks1; ++ks, ++n) {
                     if (*abort_flag) {
@@ -252,18 +276,18 @@ __global__ void __launch_bounds__(kGThreads, 1)
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0) {
-            constexpr uint32_t kId = idesc_bf16_f32(kGemmBM, kGemmBN, false, false);
+            constexpr uint32_t kId = idesc_bf16_f32(kGemmBM, BN, false, false);
             const uint32_t s0 = smem_addr(sm);
             bool ok = true;
             int n = 0, u = 0, site = 3;
             for (int w = blockIdx.x; ok && w < p.units; w += gridDim.x, ++u) {
-                const GemmUnit x = gemm_unit(p, w);
+                const GemmUnit x = gemm_unit<BN>(p, w);
                 const unsigned long long deadline = g_globaltimer() + p.watchdog_ns;
-                const int buf = u & 1;
+                const int buf = u % NB;
                 site = 4;
-                if (u >= 2 && !(ok = g_wait(&acc_empty[buf], ((u - 2) >> 1) & 1, deadline))) break;
+                if (u >= NB && !(ok = g_wait(&acc_empty[buf], ((u - NB) / NB) & 1, deadline))) break;
                 tc_fence_after();
-                const uint32_t acc0 = tbase + buf * 256, acc1 = acc0 + 128;
+                const uint32_t acc0 = tbase + buf * 2 * BN, acc1 = acc0 + BN;
                 for (int ks = x.ks0; ks < x.ks1; ++ks, ++n) {
                     const int s = n % kGStages;
                     site = 3;
@@ -295,29 +319,29 @@ __global__ void __launch_bounds__(kGThreads, 1)
         // ------------------------------------------------------------ epilogue (warps 2..5)
         const int quad = warp & 3;  // TMEM lane quadrant: rows 32 quad .. 32 quad + 31 of a tile
         const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
-        float* stg = reinterpret_cast<float*>(sm + kGOffEpi) + (warp - 2) * 32 * kGStageLd;
+        float* stg = reinterpret_cast<float*>(sm + L::kOffEpi) + (warp - 2) * 32 * kGStageLd;
         const int sub = lane >> 3, c4 = lane & 7;  // staging read-out: 4 rows x 8 float4 per instruction
         bool ok = true;
         int u = 0;
         for (int w = blockIdx.x; w < p.units; w += gridDim.x, ++u) {
-            const GemmUnit x = gemm_unit(p, w);
+            const GemmUnit x = gemm_unit<BN>(p, w);
             const unsigned long long deadline = g_globaltimer() + p.watchdog_ns;
-            const int buf = u & 1;
-            if (ok) ok = __all_sync(0xffffffffu, g_wait(&acc_full[buf], (u >> 1) & 1, deadline));
+            const int buf = u % NB;
+            if (ok) ok = __all_sync(0xffffffffu, g_wait(&acc_full[buf], (u / NB) & 1, deadline));
             if (ok) {
                 tc_fence_after();
                 for (int mt = 0; mt < (x.two ? 2 : 1); ++mt) {
                     const int mrow0 = x.m0 + mt * kGemmBM + quad * 32;  // this warp's first row
                     const int rmax = min(32, p.M - mrow0);             // rows below M
-                    float* part = p.splits > 1
+                    float* part = split
                                       ? p.partials + ((static_cast<size_t>(w) * 2 + mt) * kGemmBM + quad * 32) * kGemmBN
                                       : nullptr;
 #pragma unroll 1
-                    for (int c = 0; c < kGemmBN / 32; ++c) {
+                    for (int c = 0; c < BN / 32; ++c) {
                         // thread = row in TMEM -> a row-major 32 x 32 block in shared
                         // memory -> 4 rows of 8 float4 per warp instruction
                         float v[32];
-                        tmem_ld32(tbase + lane_off + buf * 256 + mt * 128 + c * 32, v);
+                        tmem_ld32(tbase + lane_off + buf * 2 * BN + mt * BN + c * 32, v);
                         tmem_ld_wait();
 #pragma unroll
                         for (int i = 0; i < 8; ++i)
@@ -346,7 +370,7 @@ __global__ void __launch_bounds__(kGThreads, 1)
             }
             tc_fence_before();
             mbar_arrive(&acc_empty[buf]);  // the MMA may refill this accumulator set
-            if (p.splits > 1) {
+            if (split) {
                 // Publish this split's partial: the barrier orders the CTA's partial
                 // stores before one thread's fence and counter increment.  The launch
                 // is cooperative (every unit's CTA is resident), so each split can
@@ -865,9 +889,15 @@ __global__ void __launch_bounds__(kGThreads, 1)
 GemmPlan gemm_plan(int M, int N, int K, int sms)
 {
     GemmPlan g{};
-    g.n_tiles = (N + kGemmBN - 1) / kGemmBN;
     g.m_pairs = (M + 2 * kGemmBM - 1) / (2 * kGemmBM);
     g.k_steps = (K + kGemmBK - 1) / kGemmBK;
+    // 256-wide tiles where they alone fill every SM (no K split needed) and K
+    // is long enough to hide the epilogue they cannot overlap (one accumulator
+    // set), with 128-byte aligned rows (measured at M = 1568, N = 37888,
+    // K = 3584: 380 -> 350 us; at K = 200, or with K = 3592, slower)
+    const int wide = (N + 255) / 256 * g.m_pairs;
+    g.bn = (wide >= sms && g.k_steps >= 32 && (K % 64) == 0) ? 256 : kGemmBN;
+    g.n_tiles = (N + g.bn - 1) / g.bn;
     const int tiles = g.n_tiles * g.m_pairs;
     // split K only while the tiles alone leave SMs idle, into as many ranges as
     // keep every unit in one wave
@@ -883,16 +913,26 @@ GemmPlan gemm_plan(int M, int N, int K, int sms)
 
 cudaError_t gemm_prepare()
 {
-    return cudaFuncSetAttribute(gemm_bf16_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, kGAlloc);
+    const cudaError_t e = cudaFuncSetAttribute(gemm_bf16_tc<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                               GLayout<128>::kAlloc);
+    if (e != cudaSuccess) return e;
+    return cudaFuncSetAttribute(gemm_bf16_tc<256>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                GLayout<256>::kAlloc);
 }
 
 cudaError_t launch_gemm(const CUtensorMap& tm_x, const CUtensorMap& tm_w, const GemmParams& p,
                         int sms, cudaStream_t st)
 {
     if (p.units <= 0) return cudaSuccess;
+    if (p.bn != 128 && p.bn != 256) return cudaErrorInvalidValue;
     const int grid = p.units < sms ? p.units : sms;
+    if (p.bn == 256) {
+        if (p.splits != 1) return cudaErrorInvalidValue;
+        gemm_bf16_tc<256><<<grid, kGThreads, GLayout<256>::kAlloc, st>>>(tm_x, tm_w, p);
+        return cudaGetLastError();
+    }
     if (p.splits == 1) {
-        gemm_bf16_tc<<<grid, kGThreads, kGAlloc, st>>>(tm_x, tm_w, p);
+        gemm_bf16_tc<128><<<grid, kGThreads, GLayout<128>::kAlloc, st>>>(tm_x, tm_w, p);
         return cudaGetLastError();
     }
     // split K: the splits of a tile wait for one another, so every unit's CTA
@@ -901,8 +941,8 @@ cudaError_t launch_gemm(const CUtensorMap& tm_x, const CUtensorMap& tm_w, const 
     CUtensorMap a = tm_x, b = tm_w;
     GemmParams q = p;
     void* args[] = {&a, &b, &q};
-    return cudaLaunchCooperativeKernel(reinterpret_cast<const void*>(gemm_bf16_tc), dim3(grid),
-                                       dim3(kGThreads), args, kGAlloc, st);
+    return cudaLaunchCooperativeKernel(reinterpret_cast<const void*>(gemm_bf16_tc<128>), dim3(grid),
+                                       dim3(kGThreads), args, GLayout<128>::kAlloc, st);
 }
 
 namespace {

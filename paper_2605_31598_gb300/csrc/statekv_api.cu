@@ -959,11 +959,13 @@ statekv_status statekv_block_frame(statekv_handle* h, const statekv_block_config
         const cuuint64_t sw[3] = {static_cast<cuuint64_t>(K) * 2, static_cast<cuuint64_t>(K) * N * 2,
                                   static_cast<cuuint64_t>(K) * N * 2};
         const cuuint32_t box[4] = {static_cast<cuuint32_t>(kGemmBK), static_cast<cuuint32_t>(kGemmBM), 1, 1};
-        if (!encode_4d(&tx, X, dx, sx, box) || !encode_4d(&tw, Wt, dw, sw, box)) return false;
+        const cuuint32_t wbox[4] = {static_cast<cuuint32_t>(kGemmBK), static_cast<cuuint32_t>(g.bn), 1, 1};
+        if (!encode_4d(&tx, X, dx, sx, box) || !encode_4d(&tw, Wt, dw, sw, wbox)) return false;
         GemmParams gp{};
         gp.M = rows;
         gp.N = N;
         gp.K = K;
+        gp.bn = g.bn;
         gp.n_tiles = g.n_tiles;
         gp.k_steps = g.k_steps;
         gp.kps = g.kps;

@@ -177,12 +177,14 @@ cudaError_t launch_silu_mul(const __nv_bfloat16* gu, __nv_bfloat16* a, long long
 // tile's rows over all splits in split order.
 constexpr int kGemmBM = 128, kGemmBN = 128, kGemmBK = 64;
 struct GemmPlan {
+    int bn;                     // W rows per tile: 128, or 256 for GEMMs with many tiles (no K split)
     int n_tiles, m_pairs, k_steps, kps, splits, units, counters;
     size_t partial_bytes;
 };
 GemmPlan gemm_plan(int M, int N, int K, int sms);
 struct GemmParams {
     int M, N, K;
+    int bn;                     // the plan's tile width; the W tensor map's box has bn rows
     int n_tiles, k_steps, kps, splits, units;
     const __nv_bfloat16* bias;  // nullable [N]
     __nv_bfloat16* D;           // [M][N]

@@ -189,6 +189,22 @@ def test_block_ragged_widths_thin_rows():
 
 
 @pytest.mark.gpu
+def test_block_wide_tiles_for_the_gate_up_projection():
+    """Two streams of 196 tokens (392 rows: the cooperative GEMM path), hidden
+    2048 and MLP 9728: the gate/up projection (N = 19456, K = 2048) has 76 x 2
+    tiles of 256 W rows, one per SM of a 152-SM GB300, so it runs with
+    256-wide tiles and one accumulator set; the other projections keep
+    128-wide tiles and split K."""
+    from paper_2605_31598_gb300.inputs import BlockShape
+
+    _need_gpu()
+    shape = Shape(16, 2, 128, 196, 256, 3, num_layers=1, num_streams=2)
+    stats = {}
+    worst = run_block_parity(shape, BlockShape(2048, 9728), 2, stats=stats)
+    print("wide-tile block worst |dx|", worst, stats)
+
+
+@pytest.mark.gpu
 @pytest.mark.parametrize("streams,tokens", [(1, 196), (2, 16)])
 def test_block_multi_layer_call_equals_layer_calls(streams, tokens):
     """One call over every layer (where the thin path computes layer l+1's
