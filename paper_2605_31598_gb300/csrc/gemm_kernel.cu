@@ -891,12 +891,15 @@ GemmPlan gemm_plan(int M, int N, int K, int sms)
     GemmPlan g{};
     g.m_pairs = (M + 2 * kGemmBM - 1) / (2 * kGemmBM);
     g.k_steps = (K + kGemmBK - 1) / kGemmBK;
-    // 256-wide tiles where they alone fill every SM (no K split needed) and K
-    // is long enough to hide the epilogue they cannot overlap (one accumulator
-    // set), with 128-byte aligned rows (measured at M = 1568, N = 37888,
-    // K = 3584: 380 -> 350 us; at K = 200, or with K = 3592, slower)
-    const int wide = (N + 255) / 256 * g.m_pairs;
-    g.bn = (wide >= sms && g.k_steps >= 32 && (K % 64) == 0) ? 256 : kGemmBN;
+    // 256-wide tiles when the 128-wide ones take several rounds and fewer
+    // rounds of 256-wide ones cost less: a 256-wide unit measured 1.82x a
+    // 128-wide one (twice the work; M = 1568, N = 37888, K = 3584: 380 ->
+    // 350 us).  Only with K long enough to hide the epilogue they cannot
+    // overlap (one accumulator set) and 128-byte aligned rows (at K = 200, or
+    // with K = 3592, they were slower).
+    const int narrow = (N + kGemmBN - 1) / kGemmBN * g.m_pairs, wide = (N + 255) / 256 * g.m_pairs;
+    const int r128 = (narrow + sms - 1) / sms, r256 = (wide + sms - 1) / sms;
+    g.bn = (narrow >= sms && 1.85 * r256 < r128 && g.k_steps >= 32 && (K % 64) == 0) ? 256 : kGemmBN;
     g.n_tiles = (N + g.bn - 1) / g.bn;
     const int tiles = g.n_tiles * g.m_pairs;
     // split K only while the tiles alone leave SMs idle, into as many ranges as
