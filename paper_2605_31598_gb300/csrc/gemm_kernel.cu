@@ -17,9 +17,10 @@
 //     not depend on timing;
 //   - one CTA per SM walks the units; TMEM holds two accumulator sets, so the
 //     epilogue of one unit overlaps the main loop of the next;
-//   - GEMMs with enough 256-wide tiles to fill every SM by themselves (the
-//     gate/up projection at two or more streams) use W tiles of 256 rows: one
-//     accumulator set fills TMEM, and each staged byte feeds 1.5x the MMA work.
+//   - GEMMs whose 128-wide tiles would take several rounds on the SMs use W
+//     tiles of 192 or 256 rows when fewer rounds of those cost less (every
+//     projection at eight streams, gate/up from two): one accumulator set, and
+//     each staged byte feeds up to 1.5x the MMA work.
 // 192 threads: warp 0 issues the TMA loads (a four-stage ring of 48 KB: X rows
 // m0..m0+127, X rows m0+128..m0+255, W rows n0..n0+127, 64 K-columns each,
 // 128-byte swizzle), warp 1 allocates TMEM and issues tcgen05.mma
@@ -48,13 +49,16 @@ constexpr int kRG = 8;  // rows per group of the split-K reduction (2 kRG loads 
 // Shared memory and TMEM plan for a tile of 256 rows of X x BN rows of W.
 // BN = 128: a four-stage ring of 48 KB and two accumulator sets (2 x 128
 // TMEM columns each), so a unit's epilogue overlaps the next unit's main loop.
-// BN = 256: a three-stage ring of 64 KB (W tile 32 KB) and one set filling
-// TMEM's 512 columns; each byte staged feeds 1.5x the MMA work of BN = 128,
-// for GEMMs large enough to be bound by the L2-to-SM traffic.
+// BN = 192 / 256: a three-stage ring of 56 / 64 KB and one set, its two
+// 128-row accumulators at TMEM columns 0 and 256; each byte staged feeds up to
+// 1.5x the MMA work of BN = 128, and the wider tiles change how many rounds a
+// GEMM's tiles take on the SMs.
 template <int BN>
 struct GLayout {
-    static constexpr int kStages = BN == 256 ? 3 : 4;
-    static constexpr int kAccSets = BN == 256 ? 1 : 2;
+    static constexpr int kStages = BN == 128 ? 4 : 3;
+    static constexpr int kAccSets = BN == 128 ? 2 : 1;
+    static constexpr int kMtStride = BN == 128 ? 128 : 256;  // TMEM columns between the two row tiles
+    static constexpr int kSetStride = 256;                   // TMEM columns between accumulator sets
     static constexpr int kTileB = BN * kGemmBK * 2;
     static constexpr int kStageBytes = 2 * kGTileA + kTileB;
     static constexpr int kOffEpi = kStages * kStageBytes;
@@ -63,8 +67,8 @@ struct GLayout {
     static constexpr int kOffMisc = kOffBar + kNumBars * 8;
     static constexpr int kBytes = kOffMisc + 16;
     static constexpr int kAlloc = kBytes + 1024;      // room to align the base to 1 KB
-    static_assert(BN == 128 || BN == 256, "tile width");
-    static_assert(kAccSets * 2 * BN <= 512, "TMEM columns");
+    static_assert(BN == 128 || BN == 192 || BN == 256, "tile width");
+    static_assert((kAccSets - 1) * kSetStride + kMtStride + BN <= 512, "TMEM columns");
     static_assert(kAlloc <= 232448, "shared memory budget");
     static_assert(kStageBytes % 1024 == 0 && kGTileA % 1024 == 0, "swizzle atoms stay aligned");
 };
@@ -287,7 +291,7 @@ __global__ void __launch_bounds__(kGThreads, 1)
                 site = 4;
                 if (u >= NB && !(ok = g_wait(&acc_empty[buf], ((u - NB) / NB) & 1, deadline))) break;
                 tc_fence_after();
-                const uint32_t acc0 = tbase + buf * 2 * BN, acc1 = acc0 + BN;
+                const uint32_t acc0 = tbase + buf * L::kSetStride, acc1 = acc0 + L::kMtStride;
                 for (int ks = x.ks0; ks < x.ks1; ++ks, ++n) {
                     const int s = n % kGStages;
                     site = 3;
@@ -341,7 +345,7 @@ __global__ void __launch_bounds__(kGThreads, 1)
                         // thread = row in TMEM -> a row-major 32 x 32 block in shared
                         // memory -> 4 rows of 8 float4 per warp instruction
                         float v[32];
-                        tmem_ld32(tbase + lane_off + buf * 2 * BN + mt * BN + c * 32, v);
+                        tmem_ld32(tbase + lane_off + buf * L::kSetStride + mt * L::kMtStride + c * 32, v);
                         tmem_ld_wait();
 #pragma unroll
                         for (int i = 0; i < 8; ++i)
@@ -891,15 +895,27 @@ GemmPlan gemm_plan(int M, int N, int K, int sms)
     GemmPlan g{};
     g.m_pairs = (M + 2 * kGemmBM - 1) / (2 * kGemmBM);
     g.k_steps = (K + kGemmBK - 1) / kGemmBK;
-    // 256-wide tiles when the 128-wide ones take several rounds and fewer
-    // rounds of 256-wide ones cost less: a 256-wide unit measured 1.82x a
-    // 128-wide one (twice the work; M = 1568, N = 37888, K = 3584: 380 ->
-    // 350 us).  Only with K long enough to hide the epilogue they cannot
-    // overlap (one accumulator set) and 128-byte aligned rows (at K = 200, or
-    // with K = 3592, they were slower).
-    const int narrow = (N + kGemmBN - 1) / kGemmBN * g.m_pairs, wide = (N + 255) / 256 * g.m_pairs;
-    const int r128 = (narrow + sms - 1) / sms, r256 = (wide + sms - 1) / sms;
-    g.bn = (narrow >= sms && 1.85 * r256 < r128 && g.k_steps >= 32 && (K % 64) == 0) ? 256 : kGemmBN;
+    // Wider tiles (192 or 256 W rows) when the 128-wide ones take several
+    // rounds on the SMs and fewer rounds of wider ones cost less: a 256-wide
+    // unit measured 1.82x a 128-wide one (twice the work), a 192-wide one
+    // 1.41x.  Only with K long enough to hide the epilogue they cannot overlap
+    // (one accumulator set) and 128-byte aligned rows (at K = 200, or with
+    // K = 3592, they were slower).
+    g.bn = kGemmBN;
+    const int narrow = (N + kGemmBN - 1) / kGemmBN * g.m_pairs;
+    if (narrow >= sms && g.k_steps >= 32 && (K % 64) == 0) {
+        double best = (narrow + sms - 1) / sms;
+        const int widths[2] = {192, 256};
+        const double unit_cost[2] = {1.41, 1.82};
+        for (int i = 0; i < 2; ++i) {
+            const int t = (N + widths[i] - 1) / widths[i] * g.m_pairs;
+            const double cost = ((t + sms - 1) / sms) * unit_cost[i];
+            if (cost < best - 0.05) {
+                best = cost;
+                g.bn = widths[i];
+            }
+        }
+    }
     g.n_tiles = (N + g.bn - 1) / g.bn;
     const int tiles = g.n_tiles * g.m_pairs;
     // split K only while the tiles alone leave SMs idle, into as many ranges as
@@ -916,8 +932,11 @@ GemmPlan gemm_plan(int M, int N, int K, int sms)
 
 cudaError_t gemm_prepare()
 {
-    const cudaError_t e = cudaFuncSetAttribute(gemm_bf16_tc<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                               GLayout<128>::kAlloc);
+    cudaError_t e = cudaFuncSetAttribute(gemm_bf16_tc<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         GLayout<128>::kAlloc);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(gemm_bf16_tc<192>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 GLayout<192>::kAlloc);
     if (e != cudaSuccess) return e;
     return cudaFuncSetAttribute(gemm_bf16_tc<256>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 GLayout<256>::kAlloc);
@@ -927,11 +946,14 @@ cudaError_t launch_gemm(const CUtensorMap& tm_x, const CUtensorMap& tm_w, const 
                         int sms, cudaStream_t st)
 {
     if (p.units <= 0) return cudaSuccess;
-    if (p.bn != 128 && p.bn != 256) return cudaErrorInvalidValue;
+    if (p.bn != 128 && p.bn != 192 && p.bn != 256) return cudaErrorInvalidValue;
     const int grid = p.units < sms ? p.units : sms;
-    if (p.bn == 256) {
+    if (p.bn != 128) {
         if (p.splits != 1) return cudaErrorInvalidValue;
-        gemm_bf16_tc<256><<<grid, kGThreads, GLayout<256>::kAlloc, st>>>(tm_x, tm_w, p);
+        if (p.bn == 192)
+            gemm_bf16_tc<192><<<grid, kGThreads, GLayout<192>::kAlloc, st>>>(tm_x, tm_w, p);
+        else
+            gemm_bf16_tc<256><<<grid, kGThreads, GLayout<256>::kAlloc, st>>>(tm_x, tm_w, p);
         return cudaGetLastError();
     }
     if (p.splits == 1) {

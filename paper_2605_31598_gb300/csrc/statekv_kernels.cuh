@@ -177,7 +177,7 @@ cudaError_t launch_silu_mul(const __nv_bfloat16* gu, __nv_bfloat16* a, long long
 // tile's rows over all splits in split order.
 constexpr int kGemmBM = 128, kGemmBN = 128, kGemmBK = 64;
 struct GemmPlan {
-    int bn;                     // W rows per tile: 128, or 256 for GEMMs with many tiles (no K split)
+    int bn;                     // W rows per tile: 128, or 192 / 256 for GEMMs with many tiles (no K split)
     int n_tiles, m_pairs, k_steps, kps, splits, units, counters;
     size_t partial_bytes;
 };

@@ -189,19 +189,21 @@ def test_block_ragged_widths_thin_rows():
 
 
 @pytest.mark.gpu
-def test_block_wide_tiles_for_the_gate_up_projection():
-    """Two streams of 196 tokens (392 rows: the cooperative GEMM path), hidden
-    2048 and MLP 9728: the gate/up projection (N = 19456, K = 2048) has 76 x 2
-    tiles of 256 W rows, one per SM of a 152-SM GB300, so it runs with
-    256-wide tiles and one accumulator set; the other projections keep
-    128-wide tiles and split K."""
+@pytest.mark.parametrize("intermediate", [9728, 6144])
+def test_block_wide_tiles_of_the_cooperative_path(intermediate):
+    """Two streams of 196 tokens (392 rows: the cooperative GEMM path) and
+    hidden 2048.  The gate/up projection (K = 2048) would take two rounds of
+    128-wide tiles on a 152-SM GB300 and takes one round of wider ones: with
+    MLP 9728 (N = 19456) 76 x 2 tiles of 256 W rows, with MLP 6144
+    (N = 12288) 64 x 2 tiles of 192 W rows; one accumulator set.  The other
+    projections keep 128-wide tiles and split K."""
     from paper_2605_31598_gb300.inputs import BlockShape
 
     _need_gpu()
     shape = Shape(16, 2, 128, 196, 256, 3, num_layers=1, num_streams=2)
     stats = {}
-    worst = run_block_parity(shape, BlockShape(2048, 9728), 2, stats=stats)
-    print("wide-tile block worst |dx|", worst, stats)
+    worst = run_block_parity(shape, BlockShape(2048, intermediate), 2, stats=stats)
+    print(f"wide-tile block (MLP {intermediate}) worst |dx|", worst, stats)
 
 
 @pytest.mark.gpu
