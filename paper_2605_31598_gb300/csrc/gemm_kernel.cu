@@ -97,13 +97,31 @@ struct GemmUnit {
     bool two;  // the pair's second 128-row tile holds rows below M
 };
 
+// SiLU(g) * u with the fast exponential and division: straight-line code the
+// compiler interleaves across a thread's 32 values (the epilogue runs one
+// warp per SM sub-partition, so it is bound by dependent-instruction latency;
+// the library expf / IEEE division branch and serialise it).  Relative error
+// ~1e-6, far below the bf16 rounding of the result.
+__device__ __forceinline__ float silu_times(float g, float u) { return __fdividef(g, 1.f + __expf(-g)) * u; }
+
+// Round-to-nearest-even to bf16 of a finite float, as integer arithmetic on
+// its bits (full-rate ALU work, where the conversion instructions are not):
+// the same result as __float2bfloat16_rn for every finite input.
+__device__ __forceinline__ uint32_t bf16_rne_bits(float x)
+{
+    const uint32_t u = __float_as_uint(x);
+    return (u + 0x7FFFu + ((u >> 16) & 1u)) >> 16;
+}
+
+__device__ __forceinline__ float bf16_round(float x) { return __uint_as_float(bf16_rne_bits(x) << 16); }
+
 template <int BN>
 __device__ __forceinline__ GemmUnit gemm_unit(const GemmParams& p, int w)
 {
     GemmUnit x;
     x.tile = w / p.splits;
     x.split = w - x.tile * p.splits;
-    x.n0 = (x.tile % p.n_tiles) * BN;
+    x.n0 = (x.tile % p.n_tiles) * (p.paired_I ? BN / 2 : BN);  // paired: the output column base
     x.m0 = (x.tile / p.n_tiles) * 2 * kGemmBM;
     x.ks0 = x.split * p.kps;
     x.ks1 = min(p.k_steps, x.ks0 + p.kps);
@@ -267,7 +285,12 @@ __global__ void __launch_bounds__(kGThreads, 1)
                     const int kc = ks * kGemmBK;
                     tma_load_4d(base, &tm_x, &full[s], kc, x.m0, 0, 0);
                     if (x.two) tma_load_4d(base + kGTileA, &tm_x, &full[s], kc, x.m0 + kGemmBM, 0, 0);
-                    tma_load_4d(base + 2 * kGTileA, &tm_w, &full[s], kc, x.n0, 0, 0);
+                    if (p.paired_I) {  // BN / 2 gate rows, then the same up rows
+                        tma_load_4d(base + 2 * kGTileA, &tm_w, &full[s], kc, x.n0, 0, 0);
+                        tma_load_4d(base + 2 * kGTileA + kGTileB / 2, &tm_w, &full[s], kc, x.n0, 1, 0);
+                    } else {
+                        tma_load_4d(base + 2 * kGTileA, &tm_w, &full[s], kc, x.n0, 0, 0);
+                    }
                     last_use[s] = use;
                 }
             }
@@ -340,12 +363,22 @@ __global__ void __launch_bounds__(kGThreads, 1)
                     float* part = split
                                       ? p.partials + ((static_cast<size_t>(w) * 2 + mt) * kGemmBM + quad * 32) * kGemmBN
                                       : nullptr;
+                    const uint32_t tacc = tbase + lane_off + buf * L::kSetStride + mt * L::kMtStride;
 #pragma unroll 1
-                    for (int c = 0; c < BN / 32; ++c) {
+                    for (int c = 0; c < (p.paired_I ? BN / 64 : BN / 32); ++c) {
                         // thread = row in TMEM -> a row-major 32 x 32 block in shared
                         // memory -> 4 rows of 8 float4 per warp instruction
                         float v[32];
-                        tmem_ld32(tbase + lane_off + buf * L::kSetStride + mt * L::kMtStride + c * 32, v);
+                        tmem_ld32(tacc + c * 32, v);
+                        if (p.paired_I) {
+                            // gate column j and up column j + BN / 2: SiLU(gate) * up,
+                            // each rounded to bf16 first as the unfused path stores them
+                            float u[32];
+                            tmem_ld32(tacc + BN / 2 + c * 32, u);
+                            tmem_ld_wait();
+#pragma unroll
+                            for (int i = 0; i < 32; ++i) v[i] = silu_times(bf16_round(v[i]), bf16_round(u[i]));
+                        }
                         tmem_ld_wait();
 #pragma unroll
                         for (int i = 0; i < 8; ++i)
@@ -483,24 +516,6 @@ __host__ __device__ constexpr size_t thin_staging_bytes(int M, int wblocks)
 {
     return static_cast<size_t>(wblocks) * M * 128 * 4;
 }
-
-// SiLU(g) * u with the fast exponential and division: straight-line code the
-// compiler interleaves across a thread's 32 values (the epilogue runs one
-// warp per SM sub-partition, so it is bound by dependent-instruction latency;
-// the library expf / IEEE division branch and serialise it).  Relative error
-// ~1e-6, far below the bf16 rounding of the result.
-__device__ __forceinline__ float silu_times(float g, float u) { return __fdividef(g, 1.f + __expf(-g)) * u; }
-
-// Round-to-nearest-even to bf16 of a finite float, as integer arithmetic on
-// its bits (full-rate ALU work, where the conversion instructions are not):
-// the same result as __float2bfloat16_rn for every finite input.
-__device__ __forceinline__ uint32_t bf16_rne_bits(float x)
-{
-    const uint32_t u = __float_as_uint(x);
-    return (u + 0x7FFFu + ((u >> 16) & 1u)) >> 16;
-}
-
-__device__ __forceinline__ float bf16_round(float x) { return __uint_as_float(bf16_rne_bits(x) << 16); }
 
 __device__ __forceinline__ void add4(float4& a, const float4& b)
 {
@@ -947,6 +962,7 @@ cudaError_t launch_gemm(const CUtensorMap& tm_x, const CUtensorMap& tm_w, const 
 {
     if (p.units <= 0) return cudaSuccess;
     if (p.bn != 128 && p.bn != 192 && p.bn != 256) return cudaErrorInvalidValue;
+    if (p.paired_I && (p.splits != 1 || p.paired_I != p.N || p.bias || p.add)) return cudaErrorInvalidValue;
     const int grid = p.units < sms ? p.units : sms;
     if (p.bn != 128) {
         if (p.splits != 1) return cudaErrorInvalidValue;

@@ -946,39 +946,48 @@ statekv_status statekv_block_frame(statekv_handle* h, const statekv_block_config
         return STATEKV_ERR_CUDA;
     int gemm_seq = 0;  // the call's projection GEMMs in order: each has its own counters
     // D[rows][N] = X[rows][K] W[N][K]^T (+ bias) (+ D), on the tensor cores
+    // With pair_I > 0 (gate/up: N = 2 pair_I) and a plan without K split, D
+    // receives SiLU(gate) * up [rows][pair_I] from the GEMM's epilogue and the
+    // call returns 2; otherwise it returns 1 after storing the plain product.
     auto gemm = [&](const void* X, const void* Wt, const void* bias, __nv_bfloat16* D, bool add,
-                    int N, int K) {
+                    int N, int K, int pair_I = 0, __nv_bfloat16* D_pair = nullptr) -> int {
         const GemmPlan g = gemm_plan(rows, N, K, sms);
-        if (g.counters > kGemmCounterRegion) return false;
+        if (g.counters > kGemmCounterRegion) return 0;
+        const bool paired = pair_I > 0 && g.splits == 1;
         int* counters = gemm_cnt + static_cast<size_t>(gemm_seq++) * kGemmCounterRegion;
         CUtensorMap tx, tw;
         const cuuint64_t dx[4] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(rows), 1, 1};
-        const cuuint64_t dw[4] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(N), 1, 1};
+        const cuuint64_t dw[4] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(paired ? pair_I : N),
+                                  static_cast<cuuint64_t>(paired ? 2 : 1), 1};
         const cuuint64_t sx[3] = {static_cast<cuuint64_t>(K) * 2, static_cast<cuuint64_t>(K) * rows * 2,
                                   static_cast<cuuint64_t>(K) * rows * 2};
-        const cuuint64_t sw[3] = {static_cast<cuuint64_t>(K) * 2, static_cast<cuuint64_t>(K) * N * 2,
+        const cuuint64_t sw[3] = {static_cast<cuuint64_t>(K) * 2,
+                                  static_cast<cuuint64_t>(K) * (paired ? pair_I : N) * 2,
                                   static_cast<cuuint64_t>(K) * N * 2};
         const cuuint32_t box[4] = {static_cast<cuuint32_t>(kGemmBK), static_cast<cuuint32_t>(kGemmBM), 1, 1};
-        const cuuint32_t wbox[4] = {static_cast<cuuint32_t>(kGemmBK), static_cast<cuuint32_t>(g.bn), 1, 1};
+        const cuuint32_t wbox[4] = {static_cast<cuuint32_t>(kGemmBK),
+                                    static_cast<cuuint32_t>(paired ? g.bn / 2 : g.bn), 1, 1};
         if (!encode_4d(&tx, X, dx, sx, box) || !encode_4d(&tw, Wt, dw, sw, wbox)) return false;
         GemmParams gp{};
         gp.M = rows;
-        gp.N = N;
+        gp.N = paired ? pair_I : N;
         gp.K = K;
         gp.bn = g.bn;
-        gp.n_tiles = g.n_tiles;
+        gp.paired_I = paired ? pair_I : 0;
+        gp.n_tiles = paired ? (pair_I + g.bn / 2 - 1) / (g.bn / 2) : g.n_tiles;
         gp.k_steps = g.k_steps;
         gp.kps = g.kps;
         gp.splits = g.splits;
-        gp.units = g.units;
+        gp.units = paired ? gp.n_tiles * g.m_pairs : g.units;
         gp.bias = static_cast<const __nv_bfloat16*>(bias);
-        gp.D = D;
+        gp.D = paired ? D_pair : D;
         gp.add = add ? 1 : 0;
         gp.partials = reinterpret_cast<float*>(ws + bb.gemm_part);
         gp.counters = counters;
         gp.status = h->status_dev;
         gp.watchdog_ns = 1000000ull * (c.watchdog_ms ? c.watchdog_ms : 2000u);
-        return timed(h, 3, st, [&] { return launch_gemm(tx, tw, gp, sms, st); }) == cudaSuccess;
+        if (timed(h, 3, st, [&] { return launch_gemm(tx, tw, gp, sms, st); }) != cudaSuccess) return 0;
+        return paired ? 2 : 1;
     };
     // Up to kThinMaxRows rows (one stream's frame) the projections run as thin
     // GEMMs whose epilogues finish the job: QKV adds the bias, rotates q and k
@@ -1068,9 +1077,12 @@ statekv_status statekv_block_frame(statekv_handle* h, const statekv_block_config
                                       buf(bb.h), rows, H, st);
             }) != cudaSuccess)
             return STATEKV_ERR_CUDA;
-        if (!gemm(buf(bb.h), w.w_gate_up, nullptr, buf(bb.gu), false, 2 * I, H)) return STATEKV_ERR_CUDA;
-        if (timed(h, 4, st, [&] { return launch_silu_mul(buf(bb.gu), buf(bb.act), rows, I, st); }) !=
-            cudaSuccess)
+        // gate/up: SiLU(gate) * up in the GEMM's epilogue when its plan does not
+        // split K, else the plain product and the elementwise kernel
+        const int gu = gemm(buf(bb.h), w.w_gate_up, nullptr, buf(bb.gu), false, 2 * I, H, I, buf(bb.act));
+        if (gu == 0) return STATEKV_ERR_CUDA;
+        if (gu == 1 && timed(h, 4, st, [&] { return launch_silu_mul(buf(bb.gu), buf(bb.act), rows, I, st); }) !=
+                           cudaSuccess)
             return STATEKV_ERR_CUDA;
         if (!gemm(buf(bb.act), w.w_down, nullptr, x, true, H, I)) return STATEKV_ERR_CUDA;
     }

@@ -186,6 +186,9 @@ struct GemmParams {
     int M, N, K;
     int bn;                     // the plan's tile width; the W tensor map's box has bn rows
     int n_tiles, k_steps, kps, splits, units;
+    int paired_I;               // > 0: W = gate rows [0, I) then up rows [I, 2 I), D = SiLU(gate) * up
+                                // [M][I] (N = I); the W map is [2][I][K] with boxes of bn / 2 rows,
+                                // tile t covers output columns [t bn / 2, (t + 1) bn / 2); splits = 1
     const __nv_bfloat16* bias;  // nullable [N]
     __nv_bfloat16* D;           // [M][N]
     int add;                    // 1: D += X W^T

@@ -189,14 +189,15 @@ def test_block_ragged_widths_thin_rows():
 
 
 @pytest.mark.gpu
-@pytest.mark.parametrize("intermediate", [9728, 6144])
+@pytest.mark.parametrize("intermediate", [9728, 6144, 4864])
 def test_block_wide_tiles_of_the_cooperative_path(intermediate):
     """Two streams of 196 tokens (392 rows: the cooperative GEMM path) and
-    hidden 2048.  The gate/up projection (K = 2048) would take two rounds of
-    128-wide tiles on a 152-SM GB300 and takes one round of wider ones: with
+    hidden 2048.  The gate/up projection (K = 2048) takes one round of tiles
+    on a 152-SM GB300 without splitting K, so SiLU(gate) * up is formed in its
+    epilogue (each unit holds a block of gate rows and the same up rows): with
     MLP 9728 (N = 19456) 76 x 2 tiles of 256 W rows, with MLP 6144
-    (N = 12288) 64 x 2 tiles of 192 W rows; one accumulator set.  The other
-    projections keep 128-wide tiles and split K."""
+    (N = 12288) 64 x 2 tiles of 192, with MLP 4864 (N = 9728) 76 x 2 tiles of
+    128.  The other projections keep 128-wide tiles and split K."""
     from paper_2605_31598_gb300.inputs import BlockShape
 
     _need_gpu()
