@@ -115,14 +115,20 @@ __device__ __forceinline__ uint32_t bf16_rne_bits(float x)
 
 __device__ __forceinline__ float bf16_round(float x) { return __uint_as_float(bf16_rne_bits(x) << 16); }
 
+// Tiles are numbered row pair fastest: the CTAs running at the same time
+// share W tiles (each W tile is read from HBM about once and served from L2 to
+// its other row pairs) while the X rows, far smaller, stay in L2.  Numbered
+// column fastest, a GEMM whose W exceeds L2 re-read it from HBM once per row
+// pair (1.94 GB of DRAM traffic for the 0.34 GB of the 8-stream gate/up).
 template <int BN>
 __device__ __forceinline__ GemmUnit gemm_unit(const GemmParams& p, int w)
 {
     GemmUnit x;
     x.tile = w / p.splits;
     x.split = w - x.tile * p.splits;
-    x.n0 = (x.tile % p.n_tiles) * (p.paired_I ? BN / 2 : BN);  // paired: the output column base
-    x.m0 = (x.tile / p.n_tiles) * 2 * kGemmBM;
+    const int m_pairs = (p.M + 2 * kGemmBM - 1) / (2 * kGemmBM);
+    x.n0 = (x.tile / m_pairs) * (p.paired_I ? BN / 2 : BN);  // paired: the output column base
+    x.m0 = (x.tile % m_pairs) * 2 * kGemmBM;
     x.ks0 = x.split * p.kps;
     x.ks1 = min(p.k_steps, x.ks0 + p.kps);
     x.two = x.m0 + kGemmBM < p.M;
