@@ -67,6 +67,8 @@ struct GLayout {
     static constexpr int kOffMisc = kOffBar + kNumBars * 8;
     static constexpr int kBytes = kOffMisc + 16;
     static constexpr int kAlloc = kBytes + 1024;      // room to align the base to 1 KB
+    // the epilogue reads the accumulators in 32-column chunks (paired: 32 gate and 32 up
+    // columns at a time), so BN is a multiple of 64
     static_assert(BN == 128 || BN == 192 || BN == 256, "tile width");
     static_assert((kAccSets - 1) * kSetStride + kMtStride + BN <= 512, "TMEM columns");
     static_assert(kAlloc <= 232448, "shared memory budget");
